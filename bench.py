@@ -1,0 +1,396 @@
+#!/usr/bin/env python
+"""Decode-attention benchmark over DynaCalKV latent caches on GB300.
+
+One step = one pass of the whole hot path over one decode batch:
+  1. latent append of the batch's new tokens (x [B, D] . [A_k | A_v] written
+     to each sequence's last cache row), then
+  2. decode attention (key reconstruction on tensor cores, RoPE, online
+     softmax, value absorption, split merge and B_v projection)
+for every layer of the workload.  Default workload: the Llama-2-7B-like MHA
+layer (D 4096, 32 heads of 128, 8 uneven key groups, sum r_g = 1024,
+r_v = 1024) at batch 16 x 4096-token contexts, bf16 latents.
+
+Metric: decode tokens/s (B queries per step), plus latent-cache GB/s and the
+fraction of the HBM roofline of the main attention kernel.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config C] [--impl dck|reference]
+
+With N > 1 (torchrun), every rank runs its own copy of the workload (the
+path shards by sequence with no exchange): weak scaling, value = all ranks'
+tokens / max-over-ranks time.  `--impl reference` times the fp64 CPU oracle
+(the only baseline that exists: the paper has no decode kernel).
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode attn tokens/s and latent-cache HBM GB/s (% of roofline) vs context length"
+UNIT = "tokens/s"
+L2_FLUSH_BYTES = 512 << 20
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            m = json.load(f)
+        return {"hbm_gbs": m["hbm_gbs"], "bf16_tflops": m["bf16_tflops"],
+                "bf16_tflops_sustained": m.get("bf16_tflops_sustained", m["bf16_tflops"]), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+def kernel_source_sha():
+    h = hashlib.sha256()
+    for fn in ("decode_tc.cu", "decode_simt.cu", "common.cuh"):
+        p = os.path.join(ROOT, "paper_2607_24331_gb300", "csrc", fn)
+        if os.path.exists(p):
+            h.update(open(p, "rb").read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(cfg):
+    """DRAM bytes per launch of the main decode kernel from the committed ncu summary, if current."""
+    p = os.path.join(ROOT, "profiles", "decode_main_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(str(cfg))
+    if not e or e.get("source_sha") != kernel_source_sha():
+        return None
+    return e.get("bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def gpu_identifier(torch, dev):
+    try:
+        u = str(torch.cuda.get_device_properties(dev).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        return str(dev)
+
+
+# ---------------------------------------------------------------------------
+# the oracle as CPU baseline (rank 0 only)
+# ---------------------------------------------------------------------------
+
+def oracle_sample_seconds(w, budget_s, min_pairs=2, max_pairs=4096):
+    """Times the fp64 oracle on (sequence, head) pairs of layer 0 until `budget_s` elapse.
+    Returns (pairs, seconds, description)."""
+    import numpy as np
+    import oracle
+    from paper_2607_24331_gb300 import synth as S
+
+    spec = w.layer
+    starts = S.seq_starts(w.seq_lens)
+    q = S.gaussian(S.stream_key(w.seed, 0, S.TID["q"]), (w.batch, spec.n_q_heads, spec.head_dim), 1.0, spec.dtype)
+    Bk, Bv = S.make_bk(spec, w.seed, 0), S.make_bv(spec, w.seed, 0)
+    rng = np.random.default_rng(0)
+    pairs, secs, cache = 0, 0.0, {}
+    while (secs < budget_s or pairs < min_pairs) and pairs < max_pairs:
+        b = int(rng.integers(w.batch))
+        j = int(rng.integers(spec.n_q_heads))
+        if b not in cache:
+            L = w.seq_lens[b]
+            cache = {b: (S.cache_rows(spec, w.seed, 0, "kcache", int(starts[b]), L),
+                         S.cache_rows(spec, w.seed, 0, "vcache", int(starts[b]), L))}
+        kc, vc = cache[b]
+        t0 = time.perf_counter()
+        oracle.decode_attention(spec, q[b:b + 1], kc, vc, Bk, Bv, np.array([0]), np.array([w.seq_lens[b]]),
+                                heads=[j])
+        secs += time.perf_counter() - t0
+        pairs += 1
+    desc = (f"{pairs} (sequence, query-head) pairs of layer 0 over their full contexts, fp64 numpy "
+            f"(BLAS threads = host cores); tokens/s = pairs / Hq / seconds")
+    return pairs, secs, desc
+
+
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(w, budget_s=12.0):
+    pairs, secs, desc = oracle_sample_seconds(w, budget_s)
+    tok_s = (pairs / w.layer.n_q_heads) / secs / w.n_layers
+    return {"value": tok_s, "unit": UNIT, "cores": host_cores(), "kind": "oracle", "sample": desc}
+
+
+def run_reference(args):
+    from paper_2607_24331_gb300 import synth as S
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = S.workload(args.config, args.batch)
+    for _ in range(args.warmup):
+        oracle_sample_seconds(w, 0.0, min_pairs=1, max_pairs=1)
+    t_steps, tot_pairs = [], 0
+    for _ in range(args.steps):
+        pairs, secs, desc = oracle_sample_seconds(w, 0.0, min_pairs=2, max_pairs=2)
+        t_steps.append(secs)
+        tot_pairs += pairs
+    secs = sum(t_steps)
+    value = (tot_pairs / w.layer.n_q_heads) / secs / w.n_layers
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "impl": "reference", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "batch": w.batch, "context": list(sorted(set(w.seq_lens)))[:4],
+                       "layers": w.n_layers},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+                             "sample": f"each step: 2 (sequence, query-head) pairs over full contexts, fp64 numpy"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# the GPU arm
+# ---------------------------------------------------------------------------
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", type=int, default=1)
+    ap.add_argument("--batch", type=int, default=None, help="batch of the 32-layer workload (config 4)")
+    ap.add_argument("--impl", default="dck", choices=["dck", "reference"])
+    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time for cpu_baseline")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    if args.impl == "reference":
+        run_reference(args)
+        return
+
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_2607_24331_gb300 import dck, device
+    from paper_2607_24331_gb300 import synth as S
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    w = S.workload(args.config, args.batch)
+    spec = w.layer
+    B = w.batch
+    dt = device.TORCH_DTYPE[spec.dtype]
+    layers = []
+    for l in range(w.n_layers):
+        buf = device.DecodeBuffers(spec, w.seq_lens, device=dev).synth(seed=w.seed + rank * 1000, layer=l)
+        A_k = torch.empty((spec.hidden, spec.rank_k), dtype=dt, device=dev)
+        A_v = torch.empty((spec.hidden, spec.rank_v), dtype=dt, device=dev)
+        device.synth_fill(A_k, S.stream_key(w.seed, l, S.TID["A_k"]), 1.0 / math.sqrt(spec.hidden))
+        device.synth_fill(A_v, S.stream_key(w.seed, l, S.TID["A_v"]), 1.0 / math.sqrt(spec.hidden))
+        x = torch.empty((B, spec.hidden), dtype=dt, device=dev)
+        device.synth_fill(x, S.stream_key(w.seed, l, S.TID["x_step"]), 1.0)
+        rows = (buf.seq_start + buf.seq_len.to(torch.int64) - 1).contiguous()
+        ws_a = dck.dck_latent_append_workspace_size(buf.layer, B)
+        wsa = torch.empty(max(ws_a, 256), dtype=torch.uint8, device=dev)
+        layers.append((buf, A_k, A_v, x, rows, wsa, ws_a))
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    launches = [0]
+
+    def step(q_src=None, x_src=None):
+        for l, (buf, A_k, A_v, x, rows, wsa, ws_a) in enumerate(layers):
+            xx = x if x_src is None else x_src[l]
+            dck.check(dck.dck_latent_append(buf.layer, xx, B, A_k, A_v, rows, buf.kcache, buf.vcache, buf.n_rows,
+                                            wsa, ws_a, stream), "append")
+            launches[0] += dck.dck_last_launch_count()
+            qq = buf.q if q_src is None else q_src[l]
+            dck.check(dck.dck_decode_attention(buf.layer, qq, buf.kcache, buf.vcache, buf.n_rows, buf.B_k, buf.B_v,
+                                               buf.seq_start, buf.seq_len, B, spec.rope_theta, buf.out,
+                                               buf.workspace, buf.ws_bytes, stream), "decode")
+            launches[0] += dck.dck_last_launch_count()
+
+    for _ in range(args.warmup):
+        flush.fill_(1)
+        step()
+    torch.cuda.synchronize()
+    assert dck.dck_last_device_error(stream) == dck.DCK_OK
+
+    # ---- device-resident timed region ----
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    clocks = ClockSampler(gpu_identifier(torch, local))
+    clocks.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    launches[0] = 0
+    for k in range(K):
+        flush.fill_(k & 0xFF)
+        dck.check(dck.dck_set_timing_events(*kev[k]), "timing events")
+        ev[k][0].record(stream)
+        step()
+        ev[k][1].record(stream)
+    torch.cuda.synchronize()
+    dck.check(dck.dck_set_timing_events(None, None), "timing events")
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    gpu_launches = launches[0]
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    kern_ms = [a.elapsed_time(b) for a, b in kev]
+    t_ms = sum(step_ms)
+    if world > 1:
+        tt = torch.tensor([t_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t_ms = float(tt.item())
+    ms_per_step = t_ms / K
+    value = world * B * K / (t_ms / 1e3)
+
+    # ---- end to end: host inputs -> device -> result back, every step ----
+    q_host = [torch.empty(buf.q.shape, dtype=dt, pin_memory=True) for (buf, *_r) in layers]
+    x_host = [torch.empty(x.shape, dtype=dt, pin_memory=True) for (_b, _a, _v, x, *_r) in layers]
+    out_host = [torch.empty(buf.out.shape, dtype=dt, pin_memory=True) for (buf, *_r) in layers]
+    for l, (buf, _a, _v, x, *_r) in enumerate(layers):
+        q_host[l].copy_(buf.q)
+        x_host[l].copy_(x)
+    q_dev = [torch.empty_like(buf.q) for (buf, *_r) in layers]
+    x_dev = [torch.empty_like(x) for (_b, _a, _v, x, *_r) in layers]
+    h2d = sum(t.numel() * t.element_size() for t in q_host + x_host)
+    d2h = sum(t.numel() * t.element_size() for t in out_host)
+
+    def e2e_step():
+        for l in range(len(layers)):
+            q_dev[l].copy_(q_host[l], non_blocking=True)
+            x_dev[l].copy_(x_host[l], non_blocking=True)
+        step(q_dev, x_dev)
+        for l, (buf, *_r) in enumerate(layers):
+            out_host[l].copy_(buf.out, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    eev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    if world > 1:
+        dist.barrier()
+    for k in range(K):
+        flush.fill_(k & 0xFF)
+        eev[k][0].record(stream)
+        e2e_step()
+        eev[k][1].record(stream)
+        eev[k][1].synchronize()   # the result is on the host before the next step starts
+    e2e_ms = sum(a.elapsed_time(b) for a, b in eev)
+    if world > 1:
+        tt = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    e2e_value = world * B * K / (e2e_ms / 1e3)
+
+    # ---- roofline of the main attention kernel (one launch = one layer) ----
+    peaks = load_peaks()
+    buf0 = layers[-1][0]
+    alg_bytes = buf0.algorithmic_bytes()
+    flops = buf0.tensor_flops()
+    k_avg_s = statistics.mean(kern_ms) / 1e3
+    achieved_gbs = alg_bytes / k_avg_s / 1e9
+    tflops = flops / k_avg_s / 1e12
+    step_alg_bytes = sum(b.algorithmic_bytes() for (b, *_r) in layers) + \
+        sum((a.numel() + v.numel()) * a.element_size() for (_b, a, v, *_r) in layers)
+    roof = {"bound": "hbm", "achieved": achieved_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": achieved_gbs / peaks["hbm_gbs"], "traffic": profiled_traffic(args.config),
+            "kernel": "main decode-attention kernel", "kernel_us": 1e6 * k_avg_s,
+            "alg_bytes_per_launch": alg_bytes, "peak_source": peaks["source"],
+            "tensor_tflops": tflops, "tensor_frac": tflops / peaks["bf16_tflops"],
+            "roofline_us": 1e6 * max(alg_bytes / (peaks["hbm_gbs"] * 1e9), flops / (peaks["bf16_tflops"] * 1e12))}
+
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
+            "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if spec.dtype == "bf16" else "f32", "data": "synthetic (seeded Gaussian latents/factors)",
+            "config": {"workload": w.name, "batch": B, "context": sorted(set(w.seq_lens))[:4]
+                       if w.n_layers == 1 else f"ragged U[1024,16384], mean {np.mean(w.seq_lens):.0f}",
+                       "layers": w.n_layers, "step": "latent append of B tokens + decode attention, per layer",
+                       "l2": "flushed between steps (512 MB write outside the timed events)",
+                       "parallelism": f"replicas x{world}"},
+            "latent_gbs": step_alg_bytes / (ms_per_step / 1e3) / 1e9,
+            "roofline": roof, "clocks": clk,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": gpu_launches}
+    if rank == 0 and world == 1:
+        line["cpu_baseline"] = cpu_baseline(w, args.cpu_budget)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

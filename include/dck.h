@@ -1,0 +1,188 @@
+/*
+ * dck.h - C ABI of libdck: decode attention over a DynaCalKV compressed KV cache
+ * on NVIDIA GB300 (sm_103a).
+ *
+ * The method (DynaCalKV, arXiv 2607.24331):
+ *   Sec. III-A  a rank-r factorisation W ~ L R caches z = x L (r numbers per
+ *               token) instead of x W and rebuilds x W ~ z R at attention time.
+ *   Sec. III-C  the key projection is split column-wise into head groups of
+ *               varying size; group g keeps its own factors L_g (D x r_g) and
+ *               R_g (r_g x n_g*d), so each token caches one key latent
+ *               c_t^g = x_t L_g per group, of rank r_g.
+ *   Sec. III-D  the value projection is factorised as a whole, W^(v) ~ L_v R_v,
+ *               so each token caches one value latent v_t = x_t L_v of rank r_v.
+ * Here A_g = L_g, B_g = R_g, A_v = L_v and B_v = R_v.
+ *
+ * Decode attention (one query per sequence, at position L_b - 1, the decode
+ * step's own token being the last cache row): for query head j with KV head
+ * h = floor(j * Hkv / Hq) in group g at column-block slot s,
+ *   k_t   = c_t^g B_g[:, s*d:(s+1)*d],  RoPE (rotate-half pairs (i, i+d/2),
+ *           omega_i = theta^(-2i/d)) at position t; q_j rotated at L_b - 1;
+ *   p     = softmax_t(<q_j', k_t'> / sqrt(d));
+ *   o_j   = (sum_t p_t v_t) B_v[:, h*d:(h+1)*d]
+ * (values are absorbed in latent space: sum_t p_t (v_t B_v) = (sum_t p_t v_t) B_v).
+ * The paper describes neither decode nor RoPE; these conventions are the
+ * library's and are stated here in full.
+ *
+ * Conventions of every entry point
+ *   - Pointers named d_* and all tensor pointers are DEVICE pointers on the
+ *     current CUDA device; descriptor arrays are HOST pointers, read during
+ *     the call only.
+ *   - The caller owns every buffer, including the workspace.  No entry point
+ *     allocates device memory or synchronises the stream; all work is
+ *     enqueued on `stream` (a cudaStream_t; NULL = legacy default stream).
+ *   - Host-side validation failures return a negative status before any
+ *     launch.  A failed launch returns DCK_ERR_CUDA.  Device-side checks
+ *     (lengths and rows outside the cache) record an error word that
+ *     dck_last_device_error() reports; the offending sequence is treated as
+ *     empty and its output is zero.
+ *   - No exception crosses the ABI.  Calls on distinct streams may run
+ *     concurrently if they use distinct workspaces.
+ *   - Tensors are dense row-major; element type is the descriptor's dtype
+ *     (bf16 or fp32) unless stated otherwise.
+ */
+#ifndef DCK_H_
+#define DCK_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  DCK_OK = 0,
+  DCK_ERR_INVALID = -1,     /* null pointer, bad size, malformed descriptor */
+  DCK_ERR_UNSUPPORTED = -2, /* well-formed but outside what the kernels implement */
+  DCK_ERR_WORKSPACE = -3,   /* workspace missing or smaller than the size query */
+  DCK_ERR_CUDA = -4,        /* a CUDA runtime call or kernel launch failed */
+  DCK_ERR_TIMEOUT = -5      /* a bounded device-side wait gave up */
+} dck_status;
+
+typedef enum { DCK_BF16 = 0, DCK_F32 = 1 } dck_dtype;
+
+/*
+ * One attention layer with a DynaCalKV cache (Sec. III-C key groups,
+ * Sec. III-D whole-matrix value factor).
+ *   hidden        D, the model width (rows of A_k and A_v)
+ *   n_q_heads     Hq; n_kv_heads Hkv divides Hq; consecutive query heads
+ *                 share a KV head
+ *   head_dim      d (64 or 128)
+ *   n_groups      G >= 1 key groups
+ *   group_offsets host [G+1], prefix offsets into group_heads (0 ... Hkv)
+ *   group_heads   host [Hkv], the KV heads of each group in the column-block
+ *                 order of B_g; together a permutation of 0 .. Hkv-1
+ *   ranks         host [G], r_g >= 16, a multiple of 16
+ *   rank_v        r_v >= 16, a multiple of 16
+ *   dtype         element type of q, caches, factors, x and out
+ * R_k = sum_g r_g.  Key latent of group g occupies columns
+ * [sum_{g'<g} r_g', +r_g) of a key-cache row.
+ */
+typedef struct {
+  int32_t hidden;
+  int32_t n_q_heads;
+  int32_t n_kv_heads;
+  int32_t head_dim;
+  int32_t n_groups;
+  const int32_t* group_offsets;
+  const int32_t* group_heads;
+  const int32_t* ranks;
+  int32_t rank_v;
+  int32_t dtype; /* dck_dtype */
+} dck_layer_desc;
+
+/* Text of a status code (static storage). */
+const char* dck_status_string(int32_t status);
+
+/* Checks a descriptor without launching anything. */
+dck_status dck_validate_desc(const dck_layer_desc* desc);
+
+/*
+ * Latent append (Sec. III-A z = x L; Sec. III-C L_g; Sec. III-D L_v).
+ *   x       [n_tok, D] new tokens' hidden states
+ *   A_k     [D, R_k] the key down-factors A_g side by side in group order
+ *   A_v     [D, r_v]
+ *   d_rows  device int64 [n_tok]: cache row that receives token i
+ *   kcache  [n_rows, R_k]  <- row d_rows[i] = x_i A_k   (rounded to dtype)
+ *   vcache  [n_rows, r_v]  <- row d_rows[i] = x_i A_v
+ * Accumulation is fp32.  Rows outside [0, n_rows) are skipped and recorded
+ * as a device error.  n_tok = 0 is a no-op.  The workspace (size from
+ * dck_latent_append_workspace_size, may be 0) is scratch owned by the caller.
+ */
+size_t dck_latent_append_workspace_size(const dck_layer_desc* desc, int32_t n_tok);
+dck_status dck_latent_append(const dck_layer_desc* desc, const void* x, int32_t n_tok,
+                             const void* A_k, const void* A_v, const int64_t* d_rows,
+                             void* kcache, void* vcache, int64_t n_rows,
+                             void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Decode attention over the latent caches (formula at the top of this file).
+ *   q           [B, Hq, d] queries before RoPE
+ *   kcache      [n_rows, R_k] key latents; vcache [n_rows, r_v] value latents
+ *   B_k         packed key up-factors: group g's block B_g [r_g, n_g*d]
+ *               (row-major) at element offset sum_{g'<g} r_g' n_g' d
+ *   B_v         [r_v, Hkv*d]
+ *   d_seq_start device int64 [B]: first cache row of sequence b
+ *   d_seq_len   device int32 [B]: L_b; rows d_seq_start[b] .. +L_b-1 are
+ *               sequence b's tokens at positions 0 .. L_b-1.  L_b = 0 gives a
+ *               zero output row.
+ *   rope_theta  RoPE base theta > 0
+ *   out         [B, Hq, d]
+ *   workspace   scratch of at least dck_decode_workspace_size(desc, B) bytes,
+ *               256-byte aligned; its contents need no initialisation
+ * Work is balanced over the device's SMs by 128-token tiles; the split
+ * partials live in the workspace and are merged by a second kernel on the
+ * same stream.
+ */
+size_t dck_decode_workspace_size(const dck_layer_desc* desc, int32_t batch);
+dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q,
+                                const void* kcache, const void* vcache, int64_t n_rows,
+                                const void* B_k, const void* B_v,
+                                const int64_t* d_seq_start, const int32_t* d_seq_len,
+                                int32_t batch, float rope_theta, void* out,
+                                void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Synchronises `stream`, then returns and clears the device error word of the
+ * current device: DCK_OK, DCK_ERR_INVALID (a length or row was outside the
+ * cache) or DCK_ERR_TIMEOUT (a bounded wait inside a kernel gave up).
+ */
+dck_status dck_last_device_error(void* stream);
+
+/*
+ * Kernel selection for the decode path (testing and measurement):
+ *   0 = automatic (tensor-core kernel where supported, else the CUDA-core kernel)
+ *   1 = CUDA-core kernel only
+ * Returns the previous value.  Affects subsequent calls in this process.
+ */
+int32_t dck_set_decode_kernel(int32_t which);
+
+/*
+ * Measurement hook: when both are non-NULL, every later dck_decode_attention
+ * call records the CUDA event ev_start (a cudaEvent_t) on its stream right
+ * before its main attention kernel and ev_stop right after it, so a caller
+ * can time that kernel alone.  NULL, NULL turns the hook off.  The events are
+ * owned by the caller.
+ */
+dck_status dck_set_timing_events(void* ev_start, void* ev_stop);
+
+/* Number of kernels the last decode / append call launched on the host side. */
+int32_t dck_last_launch_count(void);
+
+/*
+ * Seeded synthetic input (not part of the method): fills n elements of `dst`
+ * with the counter-based Gaussian stream `key` starting at element `start`:
+ * SplitMix64 draws 2i and 2i+1, the sum of their eight 16-bit fields s,
+ * value = float32(2s - 8*65535) * scale (one IEEE fp32 multiply), rounded to
+ * bf16 (nearest-even) when dtype is DCK_BF16.  Bit-identical to the Python
+ * generator used by the tests.
+ */
+dck_status dck_synth_gaussian(void* dst, int64_t n, uint64_t key, int64_t start,
+                              float scale, int32_t dtype, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DCK_H_ */

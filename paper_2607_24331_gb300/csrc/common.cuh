@@ -1,0 +1,159 @@
+// Internal declarations shared by the libdck translation units.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/dck.h"
+
+namespace dck {
+
+constexpr int kMaxKvHeads = 128;
+constexpr int kMaxGroups = 128;
+constexpr int kMaxQPerKv = 8;     // query heads per KV head handled by the kernels
+constexpr int kMaxRankV = 2048;
+constexpr int kMaxBatch = 4096;
+constexpr int kTile = 128;        // tokens per work tile (one UMMA M block)
+
+// Device error word values (bit flags).
+constexpr int kErrBadSeq = 1;     // a sequence's rows fall outside the cache
+constexpr int kErrBadRow = 2;     // an append destination row is outside the cache
+constexpr int kErrTimeout = 4;    // a bounded wait gave up
+
+// Group table and shapes of one layer, passed by value to the kernels.
+struct LayerTable {
+  int32_t Hq, Hkv, d, G, Rk, rv, qpg;
+  int32_t head_group[kMaxKvHeads];  // KV head -> group
+  int32_t head_slot[kMaxKvHeads];   // KV head -> column-block slot in its group
+  int32_t grp_rank[kMaxGroups];     // r_g
+  int32_t grp_roff[kMaxGroups];     // first key-cache column of group g
+  int32_t grp_nh[kMaxGroups];       // n_g
+  int64_t grp_boff[kMaxGroups];     // element offset of B_g in the packed B_k
+};
+
+// Work decomposition of a decode call: every sequence is cut into 128-token
+// tiles; the flattened tile list is split into n_items contiguous ranges
+// (item c: tiles [floor(c*NT/n), floor((c+1)*NT/n))).  Item c writes one
+// partial per sequence b it touches, in slot c + b.
+struct DecodeArgs {
+  const void* q;
+  const void* kc;
+  const void* vc;
+  const void* Bk;
+  const void* Bv;
+  const int64_t* seq_start;
+  const int32_t* seq_len;
+  int64_t n_rows;
+  int32_t B;
+  int32_t n_items;
+  float theta;
+  float* part_u;   // [n_slots, Hq, rv]
+  float* part_ml;  // [n_slots, Hq, 2]  (running max in log2 units, sum)
+  void* out;       // [B, Hq, d]
+  int* err;
+};
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Host launchers (each defined in its own translation unit).
+cudaError_t launch_decode_simt(const LayerTable& lt, const DecodeArgs& a, int dtype, cudaStream_t s);
+cudaError_t launch_combine(const LayerTable& lt, const DecodeArgs& a, int dtype, cudaStream_t s);
+cudaError_t launch_append_simt(const void* x, int n_tok, int D, const void* A_k, const void* A_v, int Rk,
+                               int rv, const int64_t* rows, void* kc, void* vc, int64_t n_rows, int dtype,
+                               int* err, cudaStream_t s);
+cudaError_t launch_synth_gaussian(void* dst, int64_t n, uint64_t key, int64_t start, float scale, int dtype,
+                                  cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// device helpers
+// ---------------------------------------------------------------------------
+
+template <typename T>
+__device__ __forceinline__ float to_f32(T v);
+template <>
+__device__ __forceinline__ float to_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+template <typename T>
+__device__ __forceinline__ T from_f32(float v);
+template <>
+__device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+
+// Number of 128-token tiles of every sequence, as an exclusive prefix in
+// shared memory prefix[0..B].  Sequences whose rows fall outside the cache
+// count as empty and raise kErrBadSeq.  Must be called by the whole block.
+// Returns the total tile count NT.
+__device__ __forceinline__ int build_tile_prefix(const int32_t* __restrict__ seq_len,
+                                                 const int64_t* __restrict__ seq_start, int B,
+                                                 int64_t n_rows, int* prefix, int* scratch, int* err,
+                                                 bool report) {
+  const int nt = blockDim.x;
+  const int per = (B + nt - 1) / nt;
+  const int b0 = threadIdx.x * per;
+  int local = 0;
+  for (int b = b0; b < b0 + per && b < B; ++b) {
+    int64_t L = seq_len[b];
+    int64_t st = seq_start[b];
+    if (L < 0 || st < 0 || st + L > n_rows) {
+      if (report) atomicOr(err, kErrBadSeq);
+      L = 0;
+    }
+    local += (int)((L + kTile - 1) / kTile);
+  }
+  scratch[threadIdx.x] = local;
+  __syncthreads();
+  // Hillis-Steele inclusive scan over the per-thread sums
+  for (int off = 1; off < nt; off <<= 1) {
+    int v = threadIdx.x >= off ? scratch[threadIdx.x - off] : 0;
+    __syncthreads();
+    scratch[threadIdx.x] += v;
+    __syncthreads();
+  }
+  int run = threadIdx.x ? scratch[threadIdx.x - 1] : 0;
+  for (int b = b0; b < b0 + per && b < B; ++b) {
+    prefix[b] = run;
+    int64_t L = seq_len[b];
+    int64_t st = seq_start[b];
+    if (L < 0 || st < 0 || st + L > n_rows) L = 0;
+    run += (int)((L + kTile - 1) / kTile);
+  }
+  int total = scratch[nt - 1];
+  if (threadIdx.x == 0) prefix[B] = total;
+  __syncthreads();
+  return total;
+}
+
+// Length of sequence b as used by the kernels (0 when its rows are invalid).
+__device__ __forceinline__ int valid_len(const int32_t* seq_len, const int64_t* seq_start, int b,
+                                         int64_t n_rows) {
+  int64_t L = seq_len[b];
+  int64_t st = seq_start[b];
+  if (L < 0 || st < 0 || st + L > n_rows) return 0;
+  return (int)L;
+}
+
+__device__ __forceinline__ int item_begin(int c, int NT, int n_items) {
+  return (int)(((int64_t)c * NT) / n_items);
+}
+
+// The item whose tile range contains tile x (0 <= x < NT).
+__device__ __forceinline__ int item_of_tile(int x, int NT, int n_items) {
+  return (int)((((int64_t)(x + 1) * n_items) + NT - 1) / NT) - 1;
+}
+
+// Sequence owning flattened tile x: largest b with prefix[b] <= x and a
+// non-empty tile range.
+__device__ __forceinline__ int seq_of_tile(const int* prefix, int B, int x) {
+  int lo = 0, hi = B - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (prefix[mid] <= x) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+}  // namespace dck

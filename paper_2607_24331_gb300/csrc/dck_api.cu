@@ -1,0 +1,271 @@
+// C ABI of libdck: argument validation, work planning and kernel dispatch.
+// The formulas and conventions are documented in include/dck.h.
+#include <atomic>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+
+#include "common.cuh"
+
+namespace dck {
+bool simt_supports(const LayerTable& lt);
+bool tc_decode_supports(const LayerTable& lt, int dtype);
+cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s);
+bool tc_append_supports(int D, int Rk, int rv, int dtype);
+size_t tc_append_workspace(int n_tok, int Rk, int rv);
+cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, const void* A_v, int Rk, int rv,
+                             const int64_t* rows, void* kc, void* vc, int64_t n_rows, void* ws, size_t ws_bytes,
+                             int* err, cudaStream_t s);
+}  // namespace dck
+
+using namespace dck;
+
+namespace {
+
+// Sticky device error word; its device address is looked up per device.
+__device__ int g_dck_error_word;
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+int* g_err_ptr[kMaxDevices] = {};
+int g_sm_count[kMaxDevices] = {};
+std::atomic<int> g_decode_kernel{0};
+std::atomic<int> g_last_launches{0};
+std::atomic<void*> g_ev_start{nullptr};
+std::atomic<void*> g_ev_stop{nullptr};
+
+bool device_state(int** err, int* sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return false;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_err_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_dck_error_word) != cudaSuccess) return false;
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return false;
+    g_err_ptr[dev] = static_cast<int*>(p);
+    g_sm_count[dev] = n;
+  }
+  if (err) *err = g_err_ptr[dev];
+  if (sms) *sms = g_sm_count[dev];
+  return true;
+}
+
+dck_status check_desc(const dck_layer_desc* d) {
+  if (!d) return DCK_ERR_INVALID;
+  if (d->hidden <= 0 || d->n_q_heads <= 0 || d->n_kv_heads <= 0 || d->head_dim <= 0 || d->n_groups <= 0 ||
+      d->rank_v <= 0)
+    return DCK_ERR_INVALID;
+  if (d->dtype != DCK_BF16 && d->dtype != DCK_F32) return DCK_ERR_INVALID;
+  if (d->n_q_heads % d->n_kv_heads != 0 || (d->head_dim & 1)) return DCK_ERR_INVALID;
+  if (!d->group_offsets || !d->group_heads || !d->ranks) return DCK_ERR_INVALID;
+  if (d->n_kv_heads > kMaxKvHeads || d->n_groups > kMaxGroups) return DCK_ERR_UNSUPPORTED;
+  if (d->group_offsets[0] != 0 || d->group_offsets[d->n_groups] != d->n_kv_heads) return DCK_ERR_INVALID;
+  for (int g = 0; g < d->n_groups; ++g) {
+    if (d->group_offsets[g + 1] <= d->group_offsets[g]) return DCK_ERR_INVALID;
+    if (d->ranks[g] <= 0) return DCK_ERR_INVALID;
+  }
+  bool seen[kMaxKvHeads] = {};
+  for (int i = 0; i < d->n_kv_heads; ++i) {
+    const int h = d->group_heads[i];
+    if (h < 0 || h >= d->n_kv_heads || seen[h]) return DCK_ERR_INVALID;
+    seen[h] = true;
+  }
+  if (d->head_dim != 64 && d->head_dim != 128) return DCK_ERR_UNSUPPORTED;
+  if (d->n_q_heads / d->n_kv_heads > kMaxQPerKv) return DCK_ERR_UNSUPPORTED;
+  if (d->rank_v % 16 || d->rank_v > kMaxRankV) return DCK_ERR_UNSUPPORTED;
+  for (int g = 0; g < d->n_groups; ++g)
+    if (d->ranks[g] % 16) return DCK_ERR_UNSUPPORTED;
+  return DCK_OK;
+}
+
+LayerTable make_table(const dck_layer_desc* d) {
+  LayerTable lt;
+  std::memset(&lt, 0, sizeof(lt));
+  lt.Hq = d->n_q_heads;
+  lt.Hkv = d->n_kv_heads;
+  lt.d = d->head_dim;
+  lt.G = d->n_groups;
+  lt.rv = d->rank_v;
+  lt.qpg = d->n_q_heads / d->n_kv_heads;
+  int roff = 0;
+  int64_t boff = 0;
+  for (int g = 0; g < d->n_groups; ++g) {
+    const int n = d->group_offsets[g + 1] - d->group_offsets[g];
+    lt.grp_rank[g] = d->ranks[g];
+    lt.grp_roff[g] = roff;
+    lt.grp_nh[g] = n;
+    lt.grp_boff[g] = boff;
+    for (int s = 0; s < n; ++s) {
+      const int h = d->group_heads[d->group_offsets[g] + s];
+      lt.head_group[h] = g;
+      lt.head_slot[h] = s;
+    }
+    roff += d->ranks[g];
+    boff += (int64_t)d->ranks[g] * n * d->head_dim;
+  }
+  lt.Rk = roff;
+  return lt;
+}
+
+size_t decode_ws_bytes(const LayerTable& lt, int batch, int n_items) {
+  const size_t slots = (size_t)n_items + (batch > 0 ? batch - 1 : 0);
+  return align_up(slots * lt.Hq * lt.rv * sizeof(float), 256) + align_up(slots * lt.Hq * 2 * sizeof(float), 256);
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+}  // namespace
+
+extern "C" {
+
+const char* dck_status_string(int32_t s) {
+  switch (s) {
+    case DCK_OK: return "ok";
+    case DCK_ERR_INVALID: return "invalid argument";
+    case DCK_ERR_UNSUPPORTED: return "unsupported shape or dtype";
+    case DCK_ERR_WORKSPACE: return "workspace missing or too small";
+    case DCK_ERR_CUDA: return "CUDA error";
+    case DCK_ERR_TIMEOUT: return "device-side wait timed out";
+    default: return "unknown status";
+  }
+}
+
+dck_status dck_validate_desc(const dck_layer_desc* desc) { return check_desc(desc); }
+
+int32_t dck_set_decode_kernel(int32_t which) { return g_decode_kernel.exchange(which); }
+
+int32_t dck_last_launch_count(void) { return g_last_launches.load(); }
+
+dck_status dck_set_timing_events(void* ev_start, void* ev_stop) {
+  if ((ev_start == nullptr) != (ev_stop == nullptr)) return DCK_ERR_INVALID;
+  g_ev_start = ev_start;
+  g_ev_stop = ev_stop;
+  return DCK_OK;
+}
+
+size_t dck_decode_workspace_size(const dck_layer_desc* desc, int32_t batch) {
+  if (check_desc(desc) != DCK_OK || batch < 0) return 0;
+  int sms = 0;
+  if (!device_state(nullptr, &sms)) return 0;
+  return decode_ws_bytes(make_table(desc), batch, sms);
+}
+
+dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const void* kcache, const void* vcache,
+                                int64_t n_rows, const void* B_k, const void* B_v, const int64_t* d_seq_start,
+                                const int32_t* d_seq_len, int32_t batch, float rope_theta, void* out,
+                                void* workspace, size_t ws_bytes, void* stream) {
+  g_last_launches = 0;
+  dck_status st = check_desc(desc);
+  if (st != DCK_OK) return st;
+  if (batch < 0 || batch > kMaxBatch || n_rows < 0) return DCK_ERR_INVALID;
+  if (!(rope_theta > 0.f) || !std::isfinite(rope_theta)) return DCK_ERR_INVALID;
+  if (batch == 0) return DCK_OK;
+  if (!q || !kcache || !vcache || !B_k || !B_v || !d_seq_start || !d_seq_len || !out) return DCK_ERR_INVALID;
+  const size_t el = desc->dtype == DCK_F32 ? 4 : 2;
+  if (!aligned(q, el) || !aligned(out, el) || !aligned(kcache, 16) || !aligned(vcache, 16) || !aligned(B_k, 16) ||
+      !aligned(B_v, 16))
+    return DCK_ERR_INVALID;
+  int* err = nullptr;
+  int sms = 0;
+  if (!device_state(&err, &sms)) return DCK_ERR_CUDA;
+  const LayerTable lt = make_table(desc);
+  const size_t need = decode_ws_bytes(lt, batch, sms);
+  if (!workspace || ws_bytes < need || !aligned(workspace, 256)) return DCK_ERR_WORKSPACE;
+  if (!simt_supports(lt)) return DCK_ERR_UNSUPPORTED;
+
+  DecodeArgs a;
+  a.q = q;
+  a.kc = kcache;
+  a.vc = vcache;
+  a.Bk = B_k;
+  a.Bv = B_v;
+  a.seq_start = d_seq_start;
+  a.seq_len = d_seq_len;
+  a.n_rows = n_rows;
+  a.B = batch;
+  a.n_items = sms;
+  a.theta = rope_theta;
+  const size_t slots = (size_t)sms + batch - 1;
+  a.part_u = static_cast<float*>(workspace);
+  a.part_ml = reinterpret_cast<float*>(static_cast<char*>(workspace) +
+                                       align_up(slots * lt.Hq * lt.rv * sizeof(float), 256));
+  a.out = out;
+  a.err = err;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  const bool use_tc = g_decode_kernel.load() == 0 && tc_decode_supports(lt, desc->dtype);
+  cudaEvent_t ev0 = static_cast<cudaEvent_t>(g_ev_start.load());
+  cudaEvent_t ev1 = static_cast<cudaEvent_t>(g_ev_stop.load());
+  if (ev0 && ev1 && cudaEventRecord(ev0, s) != cudaSuccess) return DCK_ERR_CUDA;
+  if (use_tc) e = launch_decode_tc(lt, a, s);
+  else e = launch_decode_simt(lt, a, desc->dtype, s);
+  if (e != cudaSuccess) return DCK_ERR_CUDA;
+  if (ev0 && ev1 && cudaEventRecord(ev1, s) != cudaSuccess) return DCK_ERR_CUDA;
+  e = launch_combine(lt, a, desc->dtype, s);
+  if (e != cudaSuccess) return DCK_ERR_CUDA;
+  g_last_launches = 2;
+  return DCK_OK;
+}
+
+size_t dck_latent_append_workspace_size(const dck_layer_desc* desc, int32_t n_tok) {
+  if (check_desc(desc) != DCK_OK || n_tok < 0) return 0;
+  const LayerTable lt = make_table(desc);
+  if (tc_append_supports(desc->hidden, lt.Rk, lt.rv, desc->dtype)) return tc_append_workspace(n_tok, lt.Rk, lt.rv);
+  return 0;
+}
+
+dck_status dck_latent_append(const dck_layer_desc* desc, const void* x, int32_t n_tok, const void* A_k,
+                             const void* A_v, const int64_t* d_rows, void* kcache, void* vcache, int64_t n_rows,
+                             void* workspace, size_t ws_bytes, void* stream) {
+  g_last_launches = 0;
+  dck_status st = check_desc(desc);
+  if (st != DCK_OK) return st;
+  if (n_tok < 0 || n_rows < 0) return DCK_ERR_INVALID;
+  if (n_tok == 0) return DCK_OK;
+  if (!x || !A_k || !A_v || !d_rows || !kcache || !vcache) return DCK_ERR_INVALID;
+  if (!aligned(x, 16) || !aligned(A_k, 16) || !aligned(A_v, 16) || !aligned(kcache, 16) || !aligned(vcache, 16))
+    return DCK_ERR_INVALID;
+  int* err = nullptr;
+  if (!device_state(&err, nullptr)) return DCK_ERR_CUDA;
+  const LayerTable lt = make_table(desc);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (tc_append_supports(desc->hidden, lt.Rk, lt.rv, desc->dtype)) {
+    const size_t need = tc_append_workspace(n_tok, lt.Rk, lt.rv);
+    if (need && (!workspace || ws_bytes < need || !aligned(workspace, 256))) return DCK_ERR_WORKSPACE;
+    e = launch_append_tc(x, n_tok, desc->hidden, A_k, A_v, lt.Rk, lt.rv, d_rows, kcache, vcache, n_rows, workspace,
+                         ws_bytes, err, s);
+  } else {
+    e = launch_append_simt(x, n_tok, desc->hidden, A_k, A_v, lt.Rk, lt.rv, d_rows, kcache, vcache, n_rows,
+                           desc->dtype, err, s);
+  }
+  if (e != cudaSuccess) return DCK_ERR_CUDA;
+  g_last_launches = 1;
+  return DCK_OK;
+}
+
+dck_status dck_last_device_error(void* stream) {
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return DCK_ERR_CUDA;
+  int* p = nullptr;
+  if (!device_state(&p, nullptr)) return DCK_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpyFromSymbol(&v, g_dck_error_word, sizeof(int)) != cudaSuccess) return DCK_ERR_CUDA;
+  const int zero = 0;
+  if (cudaMemcpyToSymbol(g_dck_error_word, &zero, sizeof(int)) != cudaSuccess) return DCK_ERR_CUDA;
+  if (v & kErrTimeout) return DCK_ERR_TIMEOUT;
+  if (v) return DCK_ERR_INVALID;
+  return DCK_OK;
+}
+
+dck_status dck_synth_gaussian(void* dst, int64_t n, uint64_t key, int64_t start, float scale, int32_t dtype,
+                              void* stream) {
+  if (n < 0 || start < 0 || (dtype != DCK_BF16 && dtype != DCK_F32)) return DCK_ERR_INVALID;
+  if (n == 0) return DCK_OK;
+  if (!dst || !aligned(dst, dtype == DCK_F32 ? 4 : 2)) return DCK_ERR_INVALID;
+  return launch_synth_gaussian(dst, n, key, start, scale, dtype, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? DCK_OK
+             : DCK_ERR_CUDA;
+}
+
+}  // extern "C"

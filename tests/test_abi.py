@@ -1,0 +1,70 @@
+"""The C ABI library loads, exports every declared entry point, and rejects
+malformed descriptors on the host (no GPU needed: nothing is launched)."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2607_24331_gb300 import dck
+from paper_2607_24331_gb300 import synth as S
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    names = []
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            txt = open(os.path.join(ROOT, "include", fn)).read()
+            txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+            names += re.findall(r"\b(dck_[a-z0-9_]+)\s*\(", txt)
+    return sorted(set(names))
+
+
+def test_library_exports_every_declared_symbol():
+    L = dck.lib()
+    names = declared_functions()
+    assert "dck_decode_attention" in names and "dck_latent_append" in names
+    for n in names:
+        assert hasattr(L, n), n
+    assert set(names) <= set(dck.EXPORTED)
+
+
+def test_status_strings():
+    for s in (0, -1, -2, -3, -4, -5):
+        assert dck.status_string(s)
+    assert dck.status_string(-99) == "unknown status"
+
+
+def _layer(**kw):
+    spec = dict(hidden=4096, n_q_heads=32, n_kv_heads=8, head_dim=128, groups=[[0, 1], [2, 3, 4], [5, 6, 7]],
+                ranks=[192, 256, 256], rank_v=384, dtype="bf16")
+    spec.update(kw)
+    return dck.Layer(**spec)
+
+
+def test_valid_descriptors():
+    for cfg in range(5):
+        assert dck.dck_validate_desc(dck.Layer.from_spec(S.workload(cfg).layer)) == dck.DCK_OK
+
+
+@pytest.mark.parametrize("kw,expect", [
+    (dict(n_q_heads=30), dck.DCK_ERR_INVALID),                         # Hq not a multiple of Hkv
+    (dict(groups=[[0, 1], [2, 3, 4], [5, 6, 6]]), dck.DCK_ERR_INVALID),  # not a permutation
+    (dict(groups=[[0, 1], [2, 3, 4], [5, 6]], ranks=[192, 256, 256]), dck.DCK_ERR_INVALID),
+    (dict(ranks=[192, 250, 256]), dck.DCK_ERR_UNSUPPORTED),           # rank not a multiple of 16
+    (dict(ranks=[192, 0, 256]), dck.DCK_ERR_INVALID),
+    (dict(rank_v=100), dck.DCK_ERR_UNSUPPORTED),
+    (dict(head_dim=96), dck.DCK_ERR_UNSUPPORTED),
+    (dict(head_dim=0), dck.DCK_ERR_INVALID),
+    (dict(hidden=0), dck.DCK_ERR_INVALID),
+    (dict(n_q_heads=128), dck.DCK_ERR_UNSUPPORTED),                    # 16 query heads per KV head
+])
+def test_malformed_descriptors(kw, expect):
+    assert dck.dck_validate_desc(_layer(**kw)) == expect
+
+
+def test_null_descriptor():
+    assert dck.lib().dck_validate_desc(None) == dck.DCK_ERR_INVALID
