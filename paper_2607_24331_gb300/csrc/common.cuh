@@ -52,6 +52,8 @@ struct DecodeArgs {
   float* part_ml;  // [n_slots, Hq, 2]  (running max in log2 units, sum)
   void* out;       // [B, Hq, d]
   int* err;
+  void* ev0;       // optional cudaEvent_t recorded right before / after the main kernel
+  void* ev1;
 };
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }

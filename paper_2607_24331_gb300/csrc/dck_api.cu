@@ -194,14 +194,13 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const
   a.err = err;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e;
-  const bool use_tc = g_decode_kernel.load() == 0 && tc_decode_supports(lt, desc->dtype);
-  cudaEvent_t ev0 = static_cast<cudaEvent_t>(g_ev_start.load());
-  cudaEvent_t ev1 = static_cast<cudaEvent_t>(g_ev_stop.load());
-  if (ev0 && ev1 && cudaEventRecord(ev0, s) != cudaSuccess) return DCK_ERR_CUDA;
+  const bool use_tc = g_decode_kernel.load() == 0 && n_rows < (int64_t(1) << 31) - 256 &&
+                      tc_decode_supports(lt, desc->dtype);
+  a.ev0 = g_ev_start.load();
+  a.ev1 = g_ev_stop.load();
   if (use_tc) e = launch_decode_tc(lt, a, s);
   else e = launch_decode_simt(lt, a, desc->dtype, s);
   if (e != cudaSuccess) return DCK_ERR_CUDA;
-  if (ev0 && ev1 && cudaEventRecord(ev1, s) != cudaSuccess) return DCK_ERR_CUDA;
   e = launch_combine(lt, a, desc->dtype, s);
   if (e != cudaSuccess) return DCK_ERR_CUDA;
   g_last_launches = 2;

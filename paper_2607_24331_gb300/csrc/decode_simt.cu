@@ -211,8 +211,11 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid(a.n_items, lt.Hkv);
+  if (a.ev0 && cudaEventRecordWithFlags(static_cast<cudaEvent_t>(a.ev0), s, cudaEventRecordExternal) != cudaSuccess) return cudaErrorUnknown;
   k<<<grid, kThreads, smem, s>>>(lt, a);
-  return cudaGetLastError();
+  e = cudaGetLastError();
+  if (e == cudaSuccess && a.ev1) e = cudaEventRecordWithFlags(static_cast<cudaEvent_t>(a.ev1), s, cudaEventRecordExternal);
+  return e;
 }
 
 }  // namespace

@@ -1,7 +1,756 @@
-// Tensor-core (tcgen05) decode attention: placeholder until the kernel lands.
+// Tensor-core (tcgen05) decode attention over DynaCalKV latent caches, bf16.
+//
+// One persistent CTA per SM walks its share of 128-token tiles (see
+// DecodeArgs).  For every tile and every key group g (Sec. III-C):
+//   K^_h = C_g[tile] . B_g[:, slot(h)]   for each KV head h of the group:
+//          tcgen05.mma, M = 128 tokens, N = d = 128, K = r_g, fp32 in TMEM;
+//   RoPE of K^_h in registers, scores against the rotated queries of h
+//          (log2 units), online softmax with a lazily moved reference max;
+// and once per tile the value latents are absorbed in latent space
+// (Sec. III-D, x W^(v) ~ z_v R_v applied after the sum):
+//   U[:, j] += C_v[tile]^T . P[:, j]     tcgen05.mma, M = 128 rv rows,
+//          N = query heads (padded to 16), K = tokens; U stays in TMEM.
+// At the end of each sequence segment U, the reference max and the row sum
+// are written as a split partial; the combine kernel merges splits and
+// applies B_v.
+//
+// Warp roles (320 threads):
+//   warp 0     TMA producer: latent pieces of C_g (ring A), B_g head slices
+//              and C_v pieces (ring S), all through mbarrier rings;
+//   warp 1     TMEM owner and tcgen05.mma issuer (one elected lane);
+//   warps 2-9  epilogue: each TMEM lane quadrant (32 tokens) is served by two
+//              warps that split the 64 RoPE frequency pairs of a head and
+//              add their partial scores through shared memory.
+// Every wait is bounded (2 s); on expiry the CTA stops issuing work, records
+// kErrTimeout and still releases TMEM.
+//
+// Shared-memory layouts (all 128B-swizzled unless noted):
+//   A slot  [128 tokens][w ranks] K-major, w in {64, 32, 16} with 128/64/32B
+//           swizzle: UMMA operand A of the key reconstruction;
+//   S slot  two boxes [64 rows][64 cols]: a B_g head slice (rows = ranks,
+//           cols = head dims; MN-major operand B) or a C_v piece (rows =
+//           tokens, cols = rv; MN-major operand A of the value absorption);
+//   P       [2 token atoms][Hq_pad heads][64 tokens] bf16, K-major operand B.
+#include <algorithm>
+#include <cstring>
+#include <mutex>
+
 #include "common.cuh"
+#include "sm100.cuh"
+#include "tmap.h"
 
 namespace dck {
-bool tc_decode_supports(const LayerTable&, int) { return false; }
-cudaError_t launch_decode_tc(const LayerTable&, const DecodeArgs&, cudaStream_t) { return cudaErrorNotSupported; }
+namespace {
+
+using namespace sm100;
+
+constexpr int kD = 128;
+constexpr int kNA = 5;
+constexpr int kNS = 5;
+constexpr int kSlot = 16384;
+constexpr int kMaxGroupsTc = 16;
+constexpr int kMaxPieces = 5;
+constexpr int kThreads = 320;
+constexpr int kEpiThreads = 256;
+constexpr int kMaxHqTc = 32;
+constexpr float kRescaleThr = 8.f;  // log2 units: probabilities stay <= 256
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kUCol = 256;     // first TMEM column of the U accumulators
+constexpr float kTwoPi = 6.28318530717958647692f;
+constexpr float kInvTwoPi = 0.15915494309189533577f;
+
+struct Pieces {
+  int8_t n[kMaxGroupsTc];
+  int8_t w[kMaxGroupsTc][kMaxPieces];
+  int16_t k[kMaxGroupsTc][kMaxPieces];
+};
+
+struct Maps {
+  CUtensorMap kc64, kc32, kc16, vc;
+  CUtensorMap bk[kMaxGroupsTc];
+};
+
+struct TcArgs {
+  int hq_pad;
+  int n_chunks;                  // rv / 128
+  Pieces pc;
+  int16_t order[kMaxKvHeads];    // KV head at each (group, slot) position, group-major
+};
+
+struct Smem {
+  uint8_t a[kNA][kSlot];
+  uint8_t s[kNS][kSlot];
+  uint8_t p[2][2 * kMaxHqTc * 128];
+  float qr[kMaxHqTc * kD];        // rotated queries * log2(e)/sqrt(d)
+  float x[kMaxHqTc * 128];        // scores [head][token]
+  float y[4][2][kMaxQPerKv][32];  // partial-score exchange of a quadrant's warp pair
+  double om64[kD / 2];
+  float om32[kD / 2];
+  float beta[kD / 2];
+  float redm[4][kMaxHqTc];
+  float redl[4][kMaxHqTc];
+  float alpha[kMaxHqTc];
+  uint64_t a_full[kNA], a_empty[kNA], s_full[kNS], s_empty[kNS];
+  uint64_t k_full[2], k_empty[2], p_full[2], p_empty[2], u_ready, u_free;
+  uint64_t epi_bar;             // all epilogue warps
+  uint64_t x_full[4][2], x_empty[4][2];  // partial-score exchange of a quadrant's warp pair
+  uint32_t tmem_base;
+  int abort_flag;
+  int b_first, pre_first, nt_total;
+  int a_issued, s_issued, a_used, s_used;
+};
+
+// Bounded wait whose outcome is the same in every lane of the warp.
+__device__ __forceinline__ bool wwait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+  const bool r = mbar_wait(bar, parity, abort_flag);
+  return __all_sync(0xffffffffu, r);
+}
+
+__device__ __forceinline__ int ntiles_of(const DecodeArgs& a, int b) {
+  const int L = valid_len(a.seq_len, a.seq_start, b, a.n_rows);
+  return (L + kTile - 1) / kTile;
+}
+
+struct Segment {
+  int b, L, t_begin, t_end, ntiles;
+  int64_t row0;
+};
+
+// Walks the sequences overlapping tiles [x, x1) in order.
+struct Walker {
+  int b, pre, x, x1;
+  __device__ bool next(const DecodeArgs& a, Segment& sg) {
+    while (x < x1 && b < a.B) {
+      const int nt = ntiles_of(a, b);
+      if (x >= pre + nt) {
+        pre += nt;
+        ++b;
+        continue;
+      }
+      const int xe = min(x1, pre + nt);
+      sg.b = b;
+      sg.L = valid_len(a.seq_len, a.seq_start, b, a.n_rows);
+      sg.row0 = a.seq_start[b];
+      sg.t_begin = (x - pre) * kTile;
+      sg.t_end = min(sg.L, (xe - pre) * kTile);
+      sg.ntiles = xe - x;
+      x = xe;
+      return true;
+    }
+    return false;
+  }
+};
+
+__device__ __forceinline__ uint32_t swz_of(int w) { return w == 64 ? kSw128 : (w == 32 ? kSw64 : kSw32); }
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Byte offset of P element (head j, token t) inside one P buffer.
+__device__ __forceinline__ uint32_t p_off(int j, int t, int hq_pad) {
+  const int atom = t >> 6, col = t & 63;
+  return atom * (hq_pad * 128) + (j >> 3) * 1024 + (j & 7) * 128 + ((((col >> 3) ^ (j & 7))) << 4) + ((col & 7) << 1);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    decode_tc_kernel(const __grid_constant__ Maps maps, const LayerTable lt, const DecodeArgs a, const TcArgs ta) {
+  extern __shared__ uint8_t smem_raw[];
+  Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  volatile int* abort_flag = &sm.abort_flag;
+  const int hq_pad = ta.hq_pad;
+  const int Hq = lt.Hq, qpg = lt.qpg;
+
+  // ---- setup -------------------------------------------------------------
+  if (tid == 0) {
+    for (int i = 0; i < kNA; ++i) {
+      mbar_init(&sm.a_full[i], 1);
+      mbar_init(&sm.a_empty[i], 1);
+    }
+    for (int i = 0; i < kNS; ++i) {
+      mbar_init(&sm.s_full[i], 1);
+      mbar_init(&sm.s_empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.k_full[i], 1);
+      mbar_init(&sm.k_empty[i], kEpiThreads / 32);
+      mbar_init(&sm.p_full[i], kEpiThreads / 32);
+      mbar_init(&sm.p_empty[i], 1);
+    }
+    mbar_init(&sm.u_ready, 1);
+    mbar_init(&sm.u_free, kEpiThreads / 32);
+    mbar_init(&sm.epi_bar, kEpiThreads / 32);
+    for (int q = 0; q < 4; ++q)
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&sm.x_full[q][i], 1);
+        mbar_init(&sm.x_empty[q][i], 1);
+      }
+    sm.abort_flag = 0;
+    sm.a_issued = sm.s_issued = sm.a_used = sm.s_used = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  {  // P buffers start at zero (padded head rows stay zero)
+    uint4* pz = reinterpret_cast<uint4*>(&sm.p[0][0]);
+    for (int i = tid; i < (int)(sizeof(sm.p) / 16); i += kThreads) pz[i] = make_uint4(0, 0, 0, 0);
+  }
+  if (tid < kD / 2) {
+    const double om = exp2(-2.0 * tid / kD * log2((double)a.theta));
+    sm.om64[tid] = om;
+    sm.om32[tid] = (float)om;
+  }
+  // total tiles and the first sequence of this item (block-wide scan)
+  {
+    int* scan = reinterpret_cast<int*>(sm.x);
+    const int per = (a.B + kThreads - 1) / kThreads;
+    const int b0 = tid * per;
+    int local = 0;
+    for (int b = b0; b < b0 + per && b < a.B; ++b) {
+      local += ntiles_of(a, b);
+      if (blockIdx.x == 0) {
+        const int64_t L = a.seq_len[b], st = a.seq_start[b];
+        if (L < 0 || st < 0 || st + L > a.n_rows) atomicOr(a.err, kErrBadSeq);
+      }
+    }
+    scan[tid] = local;
+    __syncthreads();
+    for (int off = 1; off < kThreads; off <<= 1) {
+      const int v = tid >= off ? scan[tid - off] : 0;
+      __syncthreads();
+      scan[tid] += v;
+      __syncthreads();
+    }
+    const int NT = scan[kThreads - 1];
+    const int x0 = item_begin(blockIdx.x, NT, a.n_items);
+    int run = tid ? scan[tid - 1] : 0;
+    if (tid == 0) {
+      sm.nt_total = NT;
+      sm.b_first = a.B;
+      sm.pre_first = NT;
+    }
+    __syncthreads();
+    for (int b = b0; b < b0 + per && b < a.B; ++b) {
+      const int nt = ntiles_of(a, b);
+      if (nt > 0 && x0 >= run && x0 < run + nt) {
+        sm.b_first = b;
+        sm.pre_first = run;
+      }
+      run += nt;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  const int NT = sm.nt_total;
+  const int x0 = item_begin(blockIdx.x, NT, a.n_items);
+  const int x1 = item_begin(blockIdx.x + 1, NT, a.n_items);
+  Walker walk{sm.b_first, sm.pre_first, x0, x1};
+  Segment seg;
+
+  if (warp == 0) {
+    // ---- TMA producer (one lane) ------------------------------------------
+    if (lane == 0 && x0 < x1) {
+      const uint64_t pol_stream = policy_evict_first();
+      const uint64_t pol_keep = policy_evict_last();
+      int a_cnt = 0, s_cnt = 0;
+      bool ok = true;
+      auto load_v = [&](int64_t yrow) {
+        for (int c = 0; c < ta.n_chunks && ok; ++c)
+          for (int th = 0; th < 2 && ok; ++th) {
+            const int sl = s_cnt % kNS;
+            if (s_cnt >= kNS && !(ok = mbar_wait(&sm.s_empty[sl], ((s_cnt / kNS) - 1) & 1, abort_flag))) break;
+            mbar_expect_tx(&sm.s_full[sl], kSlot);
+            tma_load_2d_hint(sm.s[sl], &maps.vc, &sm.s_full[sl], 128 * c, (int32_t)(yrow + 64 * th), pol_stream);
+            tma_load_2d_hint(sm.s[sl] + kSlot / 2, &maps.vc, &sm.s_full[sl], 128 * c + 64, (int32_t)(yrow + 64 * th),
+                             pol_stream);
+            ++s_cnt;
+          }
+      };
+      while (ok && walk.next(a, seg)) {
+        for (int i = 0; i < seg.ntiles && ok; ++i) {
+          const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
+          for (int g = 0; g < lt.G && ok; ++g) {
+            const int np = ta.pc.n[g];
+            for (int p = 0; p < np; ++p) {
+              const int sl = a_cnt % kNA;
+              if (a_cnt >= kNA && !(ok = mbar_wait(&sm.a_empty[sl], ((a_cnt / kNA) - 1) & 1, abort_flag))) break;
+              const int w = ta.pc.w[g][p];
+              const CUtensorMap* m = w == 64 ? &maps.kc64 : (w == 32 ? &maps.kc32 : &maps.kc16);
+              mbar_expect_tx(&sm.a_full[sl], kTile * w * 2);
+              tma_load_2d_hint(sm.a[sl], m, &sm.a_full[sl], lt.grp_roff[g] + ta.pc.k[g][p], (int32_t)yrow,
+                               pol_stream);
+              ++a_cnt;
+            }
+            const int ng = lt.grp_nh[g];
+            for (int s = 0; s < ng && ok; ++s)
+              for (int p = 0; p < np && ok; ++p) {
+                const int sl = s_cnt % kNS;
+                if (s_cnt >= kNS && !(ok = mbar_wait(&sm.s_empty[sl], ((s_cnt / kNS) - 1) & 1, abort_flag))) break;
+                mbar_expect_tx(&sm.s_full[sl], kSlot);
+                tma_load_2d_hint(sm.s[sl], &maps.bk[g], &sm.s_full[sl], s * kD, ta.pc.k[g][p], pol_keep);
+                tma_load_2d_hint(sm.s[sl] + kSlot / 2, &maps.bk[g], &sm.s_full[sl], s * kD + 64, ta.pc.k[g][p],
+                                 pol_keep);
+                ++s_cnt;
+              }
+            if (g == 0 && i > 0) load_v(yrow - kTile);
+          }
+        }
+        if (ok) load_v(seg.row0 + seg.t_begin + (int64_t)kTile * (seg.ntiles - 1));
+      }
+      sm.a_issued = a_cnt;
+      sm.s_issued = s_cnt;
+    }
+  } else if (warp == 1) {
+    // ---- MMA issuer (whole warp follows, lane 0 issues) ---------------------
+    if (x0 < x1) {
+      const uint32_t idesc_k = idesc_bf16(128, kD, false, true);
+      const uint32_t idesc_v = idesc_bf16(128, hq_pad, true, false);
+      const uint32_t p_atom = hq_pad * 128;
+      int a_cnt = 0, s_cnt = 0, kh = 0, tl = 0, sgc = 0;
+      bool ok = true;
+      // value absorption of one tile: U[:, c-chunk] += C_v^T P
+      auto pv = [&](int tt, bool first_of_seg, int nvalid) {
+        const int pb = tt & 1;
+        if (!(ok = wwait(&sm.p_full[pb], (tt >> 1) & 1, abort_flag))) return;
+        if (first_of_seg && sgc > 0 && !(ok = wwait(&sm.u_free, (sgc - 1) & 1, abort_flag))) return;
+        tc_fence_after();
+        const uint32_t pbase = smem_u32(sm.p[pb]);
+        for (int c = 0; c < ta.n_chunks && ok; ++c)
+          for (int th = 0; th < 2; ++th) {
+            const int sl = s_cnt % kNS;
+            if (!(ok = wwait(&sm.s_full[sl], (s_cnt / kNS) & 1, abort_flag))) break;
+            if (nvalid < 128) {  // rows past the sequence end: make them exact zeros
+              const int r0 = max(0, nvalid - 64 * th);
+              for (int r = r0 + (lane >> 3); r < 64; r += 4) {
+                uint4* row0 = reinterpret_cast<uint4*>(sm.s[sl] + r * 128);
+                uint4* row1 = reinterpret_cast<uint4*>(sm.s[sl] + kSlot / 2 + r * 128);
+                row0[lane & 7] = make_uint4(0, 0, 0, 0);
+                row1[lane & 7] = make_uint4(0, 0, 0, 0);
+              }
+              fence_proxy_async_smem();
+              __syncwarp();
+            }
+            tc_fence_after();
+            if (lane == 0) {
+              const uint32_t vb = smem_u32(sm.s[sl]);
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const uint64_t ad = sdesc(vb + k * 2048, kSlot / 2, 1024, kSw128);
+                const uint64_t bd = sdesc(pbase + th * p_atom + k * 32, 16, 1024, kSw128);
+                umma_f16(tmem + kUCol + c * hq_pad, ad, bd, idesc_v, (first_of_seg && th == 0 && k == 0) ? 0u : 1u);
+              }
+              umma_commit(&sm.s_empty[sl]);
+            }
+            __syncwarp();
+            ++s_cnt;
+          }
+        if (ok && lane == 0) umma_commit(&sm.p_empty[pb]);
+        __syncwarp();
+      };
+      while (ok && walk.next(a, seg)) {
+        const int tl_first = tl;
+        for (int i = 0; i < seg.ntiles && ok; ++i) {
+          for (int g = 0; g < lt.G && ok; ++g) {
+            const int np = ta.pc.n[g];
+            const int a_base = a_cnt;
+            const int ng = lt.grp_nh[g];
+            for (int s = 0; s < ng && ok; ++s) {
+              const int buf = kh & 1;
+              if (kh >= 2 && !(ok = wwait(&sm.k_empty[buf], ((kh >> 1) - 1) & 1, abort_flag))) break;
+              for (int p = 0; p < np && ok; ++p) {
+                const int asl = (a_base + p) % kNA;
+                if (s == 0 && !(ok = wwait(&sm.a_full[asl], ((a_base + p) / kNA) & 1, abort_flag))) break;
+                const int ssl = s_cnt % kNS;
+                if (!(ok = wwait(&sm.s_full[ssl], (s_cnt / kNS) & 1, abort_flag))) break;
+                tc_fence_after();
+                if (lane == 0) {
+                  const int w = ta.pc.w[g][p];
+                  const uint32_t ab = smem_u32(sm.a[asl]);
+                  const uint32_t bb = smem_u32(sm.s[ssl]);
+                  const uint32_t swz = swz_of(w);
+                  for (int k = 0; k < w / 16; ++k) {
+                    const uint64_t ad = sdesc(ab + k * 32, 16, 16 * w, swz);
+                    const uint64_t bd = sdesc(bb + k * 2048, kSlot / 2, 1024, kSw128);
+                    umma_f16(tmem + buf * kD, ad, bd, idesc_k, (p > 0 || k > 0) ? 1u : 0u);
+                  }
+                  umma_commit(&sm.s_empty[ssl]);
+                }
+                __syncwarp();
+                ++s_cnt;
+              }
+              if (ok && lane == 0) umma_commit(&sm.k_full[buf]);
+              __syncwarp();
+              ++kh;
+            }
+            if (ok && lane == 0)
+              for (int p = 0; p < np; ++p) umma_commit(&sm.a_empty[(a_base + p) % kNA]);
+            __syncwarp();
+            a_cnt += np;
+            if (ok && g == 0 && i > 0) pv(tl - 1, tl - 1 == tl_first, 128);
+          }
+          ++tl;
+        }
+        if (ok) {
+          const int nvalid = seg.t_end - (seg.t_begin + kTile * (seg.ntiles - 1));
+          pv(tl - 1, tl - 1 == tl_first, nvalid);
+        }
+        if (ok && lane == 0) umma_commit(&sm.u_ready);
+        __syncwarp();
+        ++sgc;
+      }
+      if (lane == 0) {
+        sm.a_used = a_cnt;
+        sm.s_used = s_cnt;
+      }
+    }
+  } else {
+    // ---- epilogue: RoPE, scores, softmax, P, U readout ----------------------
+    const int e = tid - 64;              // 0 .. 255
+    const int quad = warp & 3;           // TMEM lane quadrant
+    const int hf = (warp - 2) >> 2;      // frequency half, then head half
+    const int tau = quad * 32 + lane;    // token row inside the tile
+    const int hh = hq_pad / 2;           // heads owned after the exchange
+    const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+    int kh = 0, tl = 0, sgc = 0, round = 0;
+    bool ok = true;
+    // bounded barrier over the eight epilogue warps
+    auto epi_sync = [&]() -> bool {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.epi_bar);
+      const bool r = wwait(&sm.epi_bar, round & 1, abort_flag);
+      ++round;
+      return r;
+    };
+    float m_ref[kMaxHqTc / 2];
+    float l_acc[kMaxHqTc / 2];
+    while (ok && walk.next(a, seg)) {
+      // rotated queries of this sequence at position L-1, scaled to log2 units
+      const double P = (double)(seg.L - 1);
+      const float qscale = 1.4426950408889634f * rsqrtf((float)kD);
+      const __nv_bfloat16* qb = static_cast<const __nv_bfloat16*>(a.q) + (int64_t)seg.b * Hq * kD;
+      for (int i = e; i < Hq * (kD / 2); i += kEpiThreads) {
+        const int j = i / (kD / 2), pi = i % (kD / 2);
+        double sn, cs;
+        sincos(P * sm.om64[pi], &sn, &cs);
+        const double x1v = __bfloat162float(qb[j * kD + pi]), x2v = __bfloat162float(qb[j * kD + pi + kD / 2]);
+        sm.qr[j * kD + pi] = (float)(x1v * cs - x2v * sn) * qscale;
+        sm.qr[j * kD + pi + kD / 2] = (float)(x1v * sn + x2v * cs) * qscale;
+      }
+#pragma unroll
+      for (int u = 0; u < kMaxHqTc / 2; ++u) {
+        m_ref[u] = -INFINITY;
+        l_acc[u] = 0.f;
+      }
+      if (!(ok = epi_sync())) break;
+      const int tl_first = tl;
+      for (int i = 0; i < seg.ntiles && ok; ++i) {
+        const int t0 = seg.t_begin + kTile * i;
+        const bool valid = t0 + tau < seg.t_end;
+        // RoPE angle of token t0+tau and pair p: (t0*omega_p mod 2pi, fp64) + tau*omega_p (fp32)
+        if (e < kD / 2) {
+          const double ang = (double)t0 * sm.om64[e];
+          sm.beta[e] = (float)(ang - 6.283185307179586 * floor(ang * 0.15915494309189535));
+        }
+        if (!(ok = epi_sync())) break;
+        float cs[32], sn[32];
+#pragma unroll
+        for (int ip = 0; ip < 32; ++ip) {
+          const int pi = 32 * hf + ip;
+          float ph = fmaf((float)tau, sm.om32[pi], sm.beta[pi]);
+          ph = fmaf(-kTwoPi, rintf(ph * kInvTwoPi), ph);
+          __sincosf(ph, &sn[ip], &cs[ip]);
+        }
+        // reconstructed keys, head by head in MMA order
+        for (int hi = 0; hi < lt.Hkv && ok; ++hi) {
+          const int buf = kh & 1;
+          if (!(ok = wwait(&sm.k_full[buf], (kh >> 1) & 1, abort_flag))) break;
+          tc_fence_after();
+          const int j0 = ta.order[hi] * qpg;
+          float part[kMaxQPerKv];
+#pragma unroll
+          for (int jj = 0; jj < kMaxQPerKv; ++jj) part[jj] = 0.f;
+#pragma unroll
+          for (int ch = 0; ch < 2; ++ch) {
+            float k1[16], k2[16];
+            tmem_ld16(tmem + lane_base + buf * kD + 32 * hf + 16 * ch, k1);
+            tmem_ld16(tmem + lane_base + buf * kD + 64 + 32 * hf + 16 * ch, k2);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i2 = 0; i2 < 16; ++i2) {
+              const int ip = 16 * ch + i2;
+              const float r1 = fmaf(k1[i2], cs[ip], -k2[i2] * sn[ip]);
+              const float r2 = fmaf(k1[i2], sn[ip], k2[i2] * cs[ip]);
+              const float* qrow = sm.qr + j0 * kD + 32 * hf + ip;
+#pragma unroll
+              for (int jj = 0; jj < kMaxQPerKv; ++jj)
+                if (jj < qpg) part[jj] = fmaf(qrow[jj * kD], r1, fmaf(qrow[jj * kD + 64], r2, part[jj]));
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
+          // the frequency-half-1 warp hands its partial scores to its partner
+          const int yb = kh & 1, yn = kh >> 1;
+          if (hf == 1) {
+            if (yn >= 1 && !(ok = wwait(&sm.x_empty[quad][yb], (yn - 1) & 1, abort_flag))) break;
+#pragma unroll
+            for (int jj = 0; jj < kMaxQPerKv; ++jj)
+              if (jj < qpg) sm.y[quad][yb][jj][lane] = part[jj];
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.x_full[quad][yb]);
+          } else {
+            if (!(ok = wwait(&sm.x_full[quad][yb], yn & 1, abort_flag))) break;
+#pragma unroll
+            for (int jj = 0; jj < kMaxQPerKv; ++jj)
+              if (jj < qpg) sm.x[(j0 + jj) * 128 + tau] = valid ? part[jj] + sm.y[quad][yb][jj][lane] : -INFINITY;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.x_empty[quad][yb]);
+          }
+          ++kh;
+        }
+        if (!ok) break;
+        // ---- tile end: reference max, optional rescale of U, P -------------
+        if (!(ok = epi_sync())) break;
+        float sc[kMaxHqTc / 2];
+#pragma unroll
+        for (int u = 0; u < kMaxHqTc / 2; ++u) {
+          const int j = hf * hh + u;
+          sc[u] = (u < hh && j < Hq) ? sm.x[j * 128 + tau] : -INFINITY;
+          const float mx = warp_max(sc[u]);
+          if (lane == 0 && u < hh && j < Hq) sm.redm[quad][j] = mx;
+        }
+        if (!(ok = epi_sync())) break;
+        float al[kMaxHqTc / 2];
+#pragma unroll
+        for (int u = 0; u < kMaxHqTc / 2; ++u) {
+          const int j = hf * hh + u;
+          al[u] = 1.f;
+          if (u < hh && j < Hq) {
+            const float tmax = fmaxf(fmaxf(sm.redm[0][j], sm.redm[1][j]), fmaxf(sm.redm[2][j], sm.redm[3][j]));
+            if (m_ref[u] == -INFINITY || tmax > m_ref[u] + kRescaleThr) {
+              al[u] = exp2f(m_ref[u] - tmax);
+              m_ref[u] = tmax;
+            }
+            if (quad == 0 && lane == 0) sm.alpha[j] = al[u];
+          }
+        }
+        if (!(ok = epi_sync())) break;
+        bool any = false;
+        if (tl != tl_first)
+          for (int j = 0; j < Hq; ++j) any |= sm.alpha[j] != 1.f;
+        if (any) {
+          // rescale U: the previous tile's absorption must have completed
+          const int tp = tl - 1;
+          if (!(ok = wwait(&sm.p_empty[tp & 1], (tp >> 1) & 1, abort_flag))) break;
+          tc_fence_after();
+          for (int c = hf; c < ta.n_chunks; c += 2)
+            for (int cb = 0; cb < hq_pad / 16; ++cb) {
+              float v[16];
+              const uint32_t tad = tmem + lane_base + kUCol + c * hq_pad + 16 * cb;
+              tmem_ld16(tad, v);
+              tmem_wait_ld();
+#pragma unroll
+              for (int i2 = 0; i2 < 16; ++i2) {
+                const int j = 16 * cb + i2;
+                v[i2] *= (j < Hq) ? sm.alpha[j] : 1.f;
+              }
+              tmem_st16(tad, v);
+            }
+          tmem_wait_st();
+          tc_fence_before();
+        }
+        // probabilities -> P (bf16); row sums use the rounded values
+        const int pb = tl & 1;
+        if (tl >= 2 && !(ok = wwait(&sm.p_empty[pb], ((tl - 2) >> 1) & 1, abort_flag))) break;
+        uint8_t* pbuf = sm.p[pb];
+#pragma unroll
+        for (int u = 0; u < kMaxHqTc / 2; ++u) {
+          const int j = hf * hh + u;
+          if (u < hh && j < Hq) {
+            l_acc[u] *= al[u];
+            const __nv_bfloat16 pv = __float2bfloat16_rn(exp2f(sc[u] - m_ref[u]));
+            l_acc[u] += __bfloat162float(pv);
+            *reinterpret_cast<__nv_bfloat16*>(pbuf + p_off(j, tau, hq_pad)) = pv;
+          }
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.p_full[pb]);
+        ++tl;
+      }
+      if (!ok) break;
+      // ---- segment end: U, reference max and row sums -> partial slot c + b ---
+      if (!(ok = wwait(&sm.u_ready, sgc & 1, abort_flag))) break;
+      tc_fence_after();
+      const int64_t slot = (int64_t)blockIdx.x + seg.b;
+      for (int c = hf; c < ta.n_chunks; c += 2)
+        for (int cb = 0; cb < hq_pad / 16; ++cb) {
+          float v[16];
+          tmem_ld16(tmem + lane_base + kUCol + c * hq_pad + 16 * cb, v);
+          tmem_wait_ld();
+          const int r = c * 128 + tau;
+#pragma unroll
+          for (int i2 = 0; i2 < 16; ++i2) {
+            const int j = 16 * cb + i2;
+            if (j < Hq) a.part_u[(slot * Hq + j) * lt.rv + r] = v[i2];
+          }
+        }
+      tc_fence_before();
+#pragma unroll
+      for (int u = 0; u < kMaxHqTc / 2; ++u) {
+        const int j = hf * hh + u;
+        const float ls = warp_sum(l_acc[u]);
+        if (lane == 0 && u < hh && j < Hq) sm.redl[quad][j] = ls;
+      }
+      if (!(ok = epi_sync())) break;
+      if (quad == 0 && lane == 0) {
+#pragma unroll
+        for (int u = 0; u < kMaxHqTc / 2; ++u) {
+          const int j = hf * hh + u;
+          if (u < hh && j < Hq) {
+            a.part_ml[(slot * Hq + j) * 2] = m_ref[u];
+            a.part_ml[(slot * Hq + j) * 2 + 1] = sm.redl[0][j] + sm.redl[1][j] + sm.redl[2][j] + sm.redl[3][j];
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.u_free);
+      ++sgc;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (sm.abort_flag) {
+    // let copies and MMAs already in flight land before the memory is released
+    const uint64_t t0 = global_timer_ns();
+    while (global_timer_ns() - t0 < 2000000ull) {
+    }
+    if (tid == 0) atomicOr(a.err, kErrTimeout);
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace
+
+// Split of a group rank into TMA/UMMA pieces of 64, 32 and 16 columns.
+static int make_pieces(int r, int8_t* w, int16_t* k) {
+  int n = 0, off = 0;
+  for (const int pw : {64, 32, 16})
+    while (r - off >= pw) {
+      if (n == kMaxPieces) return kMaxPieces + 1;
+      w[n] = (int8_t)pw;
+      k[n] = (int16_t)off;
+      off += pw;
+      ++n;
+    }
+  return off == r ? n : kMaxPieces + 1;
+}
+
+static int hq_pad_of(int Hq) { return std::max(16, (Hq + 15) / 16 * 16); }
+
+bool tc_decode_supports(const LayerTable& lt, int dtype) {
+  if (dtype != DCK_BF16 || lt.d != kD) return false;
+  if (lt.Hq > kMaxHqTc || lt.qpg > kMaxQPerKv || lt.G > kMaxGroupsTc) return false;
+  if (lt.rv % 128 || (lt.rv / 128) * hq_pad_of(lt.Hq) > 256) return false;
+  for (int g = 0; g < lt.G; ++g) {
+    int8_t w[kMaxPieces];
+    int16_t k[kMaxPieces];
+    if (lt.grp_rank[g] > 256 || make_pieces(lt.grp_rank[g], w, k) > kMaxPieces) return false;
+  }
+  return true;
+}
+
+// Tensor maps depend only on the buffers and the layer: cache the last few.
+struct MapsKey {
+  const void *kc, *vc, *bk;
+  int64_t n_rows;
+  int Rk, rv, G;
+  int64_t sig;
+  bool operator==(const MapsKey& o) const {
+    return kc == o.kc && vc == o.vc && bk == o.bk && n_rows == o.n_rows && Rk == o.Rk && rv == o.rv && G == o.G &&
+           sig == o.sig;
+  }
+};
+constexpr int kMapsCache = 64;
+std::mutex g_maps_mu;
+MapsKey g_maps_key[kMapsCache];
+Maps g_maps_val[kMapsCache];
+int g_maps_n = 0, g_maps_next = 0;
+
+cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) {
+  TcArgs ta;
+  std::memset(&ta, 0, sizeof(ta));
+  ta.hq_pad = hq_pad_of(lt.Hq);
+  ta.n_chunks = lt.rv / 128;
+  int pos = 0;
+  for (int g = 0; g < lt.G; ++g) {
+    ta.pc.n[g] = (int8_t)make_pieces(lt.grp_rank[g], ta.pc.w[g], ta.pc.k[g]);
+    for (int sl = 0; sl < lt.grp_nh[g]; ++sl)
+      for (int h = 0; h < lt.Hkv; ++h)
+        if (lt.head_group[h] == g && lt.head_slot[h] == sl) ta.order[pos++] = (int16_t)h;
+  }
+  Maps maps;
+  std::memset(&maps, 0, sizeof(maps));
+  int64_t sig = 0;
+  for (int g = 0; g < lt.G; ++g) sig = sig * 1000003 + lt.grp_rank[g] * 131 + lt.grp_nh[g] * 7 + lt.grp_boff[g];
+  const MapsKey key{a.kc, a.vc, a.Bk, a.n_rows, lt.Rk, lt.rv, lt.G, sig};
+  {
+    std::lock_guard<std::mutex> lk(g_maps_mu);
+    for (int i = 0; i < g_maps_n; ++i)
+      if (g_maps_key[i] == key) {
+        maps = g_maps_val[i];
+        goto have_maps;
+      }
+  }
+  {
+  const uint64_t rows = (uint64_t)std::max<int64_t>(1, a.n_rows);
+  bool ok = make_tmap_2d_bf16(&maps.kc64, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 64, kTile, CU_TENSOR_MAP_SWIZZLE_128B) &&
+            make_tmap_2d_bf16(&maps.kc32, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 32, kTile, CU_TENSOR_MAP_SWIZZLE_64B) &&
+            make_tmap_2d_bf16(&maps.kc16, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 16, kTile, CU_TENSOR_MAP_SWIZZLE_32B) &&
+            make_tmap_2d_bf16(&maps.vc, a.vc, lt.rv, rows, (uint64_t)lt.rv * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B);
+  for (int g = 0; g < lt.G && ok; ++g) {
+    const __nv_bfloat16* base = static_cast<const __nv_bfloat16*>(a.Bk) + lt.grp_boff[g];
+    const uint64_t cols = (uint64_t)lt.grp_nh[g] * kD;
+    ok = make_tmap_2d_bf16(&maps.bk[g], base, cols, lt.grp_rank[g], cols * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B);
+  }
+  if (!ok) return cudaErrorInvalidValue;
+  std::lock_guard<std::mutex> lk(g_maps_mu);
+  g_maps_key[g_maps_next] = key;
+  g_maps_val[g_maps_next] = maps;
+  g_maps_next = (g_maps_next + 1) % kMapsCache;
+  g_maps_n = std::min(g_maps_n + 1, kMapsCache);
+  }
+have_maps:
+  const size_t smem = sizeof(Smem) + 1024;
+  static int attr_done[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64 || !attr_done[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) attr_done[dev] = 1;
+  }
+  if (a.ev0 && cudaEventRecordWithFlags(static_cast<cudaEvent_t>(a.ev0), s, cudaEventRecordExternal) != cudaSuccess) return cudaErrorUnknown;
+  decode_tc_kernel<<<a.n_items, kThreads, smem, s>>>(maps, lt, a, ta);
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess && a.ev1) e = cudaEventRecordWithFlags(static_cast<cudaEvent_t>(a.ev1), s, cudaEventRecordExternal);
+  return e;
+}
+
 }  // namespace dck
