@@ -144,6 +144,32 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q,
                                 void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * Decode attention for callers that cannot allocate device memory (the paper
+ * has no counterpart: this is a deployment convenience of the library).
+ * A runtime whose device memory is fully reserved by its own pool, a plug-in
+ * handed only its input and output tensors, or a loop that must not allocate
+ * after start-up cannot provide the workspace of dck_decode_attention.  This
+ * entry point computes exactly what dck_decode_attention computes, with the
+ * same arguments minus the workspace: the split partials go to a fixed
+ * 32 MiB array in the library's own device memory, which every GPU that
+ * loads the library holds until the process exits.
+ *   - Requests whose dck_decode_workspace_size exceeds 32 MiB are rejected
+ *     with DCK_ERR_WORKSPACE before anything is launched.
+ *   - The first call on a device looks up the array's device address (a
+ *     host-side set-up step); make that first call before any stream capture.
+ *   - All calls share the one array and it keeps the last call's contents (it
+ *     needs no clearing: every value read is written first by the same call).
+ *     Calls that overlap on the same GPU (for example on two streams) race on
+ *     it: serialise them.  Each GPU has its own copy of the array.
+ *   - No device memory is allocated or freed by this call.
+ */
+dck_status dck_decode_attention_noalloc(const dck_layer_desc* desc, const void* q,
+                                        const void* kcache, const void* vcache, int64_t n_rows,
+                                        const void* B_k, const void* B_v,
+                                        const int64_t* d_seq_start, const int32_t* d_seq_len,
+                                        int32_t batch, float rope_theta, void* out, void* stream);
+
+/*
  * Synchronises `stream`, then returns and clears the device error word of the
  * current device: DCK_OK, DCK_ERR_INVALID (a length or row was outside the
  * cache) or DCK_ERR_TIMEOUT (a bounded wait inside a kernel gave up).

@@ -27,7 +27,7 @@ DCK_F32 = 1
 EXPORTED = (
     "dck_status_string", "dck_validate_desc", "dck_latent_append_workspace_size", "dck_latent_append",
     "dck_decode_workspace_size", "dck_decode_attention", "dck_last_device_error", "dck_set_decode_kernel",
-    "dck_last_launch_count", "dck_synth_gaussian", "dck_set_timing_events",
+    "dck_last_launch_count", "dck_synth_gaussian", "dck_set_timing_events", "dck_decode_attention_noalloc",
 )
 
 
@@ -78,6 +78,8 @@ def lib() -> ctypes.CDLL:
     L.dck_decode_workspace_size.argtypes = [D, I32]
     L.dck_decode_attention.restype = I32
     L.dck_decode_attention.argtypes = [D, P, P, P, I64, P, P, P, P, I32, F32, P, P, SZ, P]
+    L.dck_decode_attention_noalloc.restype = I32
+    L.dck_decode_attention_noalloc.argtypes = [D, P, P, P, I64, P, P, P, P, I32, F32, P, P]
     L.dck_last_device_error.restype = I32
     L.dck_last_device_error.argtypes = [P]
     L.dck_set_decode_kernel.restype = I32
@@ -160,6 +162,14 @@ def dck_decode_attention(layer: Layer, q, kcache, vcache, n_rows: int, B_k, B_v,
     return lib().dck_decode_attention(layer.ref, _ptr(q), _ptr(kcache), _ptr(vcache), int(n_rows), _ptr(B_k),
                                       _ptr(B_v), _ptr(seq_start), _ptr(seq_len), int(batch), float(rope_theta),
                                       _ptr(out), _ptr(workspace), int(ws_bytes), _stream(stream))
+
+
+def dck_decode_attention_noalloc(layer: Layer, q, kcache, vcache, n_rows: int, B_k, B_v, seq_start, seq_len,
+                                 batch: int, rope_theta: float, out, stream=None) -> int:
+    """dck_decode_attention without a workspace argument (library-owned fixed scratch)."""
+    return lib().dck_decode_attention_noalloc(layer.ref, _ptr(q), _ptr(kcache), _ptr(vcache), int(n_rows),
+                                              _ptr(B_k), _ptr(B_v), _ptr(seq_start), _ptr(seq_len), int(batch),
+                                              float(rope_theta), _ptr(out), _stream(stream))
 
 
 def dck_latent_append(layer: Layer, x, n_tok: int, A_k, A_v, rows, kcache, vcache, n_rows: int,
