@@ -54,6 +54,7 @@ struct DecodeArgs {
   int* err;
   void* ev0;       // optional cudaEvent_t recorded right before / after the main kernel
   void* ev1;
+  void* extra;     // workspace region of the tensor-core path (per-sequence folded factors)
 };
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }

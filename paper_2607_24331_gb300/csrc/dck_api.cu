@@ -10,6 +10,8 @@
 namespace dck {
 bool simt_supports(const LayerTable& lt);
 bool tc_decode_supports(const LayerTable& lt, int dtype);
+size_t tc_decode_extra_ws(const LayerTable& lt, int batch);
+int tc_decode_launches(const LayerTable& lt);
 cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s);
 bool tc_append_supports(int D, int Rk, int rv, int dtype);
 size_t tc_append_workspace(int n_tok, int Rk, int rv);
@@ -108,9 +110,14 @@ LayerTable make_table(const dck_layer_desc* d) {
   return lt;
 }
 
-size_t decode_ws_bytes(const LayerTable& lt, int batch, int n_items) {
+size_t decode_ws_parts(const LayerTable& lt, int batch, int n_items) {
   const size_t slots = (size_t)n_items + (batch > 0 ? batch - 1 : 0);
   return align_up(slots * lt.Hq * lt.rv * sizeof(float), 256) + align_up(slots * lt.Hq * 2 * sizeof(float), 256);
+}
+
+// Workspace: split partials U and (m, l), then the tensor-core path's extra region.
+size_t decode_ws_bytes(const LayerTable& lt, int batch, int n_items, int dtype) {
+  return decode_ws_parts(lt, batch, n_items) + tc_decode_extra_ws(lt, dtype == DCK_BF16 ? batch : 0);
 }
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
@@ -148,7 +155,7 @@ size_t dck_decode_workspace_size(const dck_layer_desc* desc, int32_t batch) {
   if (check_desc(desc) != DCK_OK || batch < 0) return 0;
   int sms = 0;
   if (!device_state(nullptr, &sms)) return 0;
-  return decode_ws_bytes(make_table(desc), batch, sms);
+  return decode_ws_bytes(make_table(desc), batch, sms, desc->dtype);
 }
 
 dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const void* kcache, const void* vcache,
@@ -170,7 +177,7 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const
   int sms = 0;
   if (!device_state(&err, &sms)) return DCK_ERR_CUDA;
   const LayerTable lt = make_table(desc);
-  const size_t need = decode_ws_bytes(lt, batch, sms);
+  const size_t need = decode_ws_bytes(lt, batch, sms, desc->dtype);
   if (!workspace || ws_bytes < need || !aligned(workspace, 256)) return DCK_ERR_WORKSPACE;
   if (!simt_supports(lt)) return DCK_ERR_UNSUPPORTED;
 
@@ -192,6 +199,7 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const
                                        align_up(slots * lt.Hq * lt.rv * sizeof(float), 256));
   a.out = out;
   a.err = err;
+  a.extra = static_cast<char*>(workspace) + decode_ws_parts(lt, batch, sms);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e;
   const bool use_tc = g_decode_kernel.load() == 0 && n_rows < (int64_t(1) << 31) - 256 &&
@@ -203,7 +211,7 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const
   if (e != cudaSuccess) return DCK_ERR_CUDA;
   e = launch_combine(lt, a, desc->dtype, s);
   if (e != cudaSuccess) return DCK_ERR_CUDA;
-  g_last_launches = 2;
+  g_last_launches = (use_tc ? tc_decode_launches(lt) : 1) + 1;
   return DCK_OK;
 }
 

@@ -41,4 +41,20 @@ inline bool make_tmap_2d_bf16(CUtensorMap* m, const void* base, uint64_t inner, 
   return r == CUDA_SUCCESS;
 }
 
+// 3-D bf16 tensor [d2][d1][d0] with pitches p1 (bytes between d1 rows) and p2
+// (bytes between d2 slabs), box {box0, box1, 1}.
+inline bool make_tmap_3d_bf16(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t p1,
+                              uint64_t p2, uint32_t box0, uint32_t box1, CUtensorMapSwizzle sw) {
+  auto enc = tmap_encoder();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {p1, p2};
+  cuuint32_t box[3] = {box0, box1, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 }  // namespace dck
