@@ -160,3 +160,15 @@ __device__ __forceinline__ int seq_of_tile(const int* prefix, int B, int x) {
 }
 
 }  // namespace dck
+
+namespace dck {
+// Records a caller's timing event on `s`; inside stream capture it becomes an
+// external event node, so that it can be timed after each graph replay.
+inline cudaError_t record_timing_event(void* ev, cudaStream_t s) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &st) != cudaSuccess) return cudaErrorUnknown;
+  if (st == cudaStreamCaptureStatusActive)
+    return cudaEventRecordWithFlags(static_cast<cudaEvent_t>(ev), s, cudaEventRecordExternal);
+  return cudaEventRecord(static_cast<cudaEvent_t>(ev), s);
+}
+}  // namespace dck

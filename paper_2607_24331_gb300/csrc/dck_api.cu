@@ -9,6 +9,7 @@
 
 namespace dck {
 bool simt_supports(const LayerTable& lt);
+bool combine_supports(const LayerTable& lt);
 bool tc_decode_supports(const LayerTable& lt, int dtype);
 size_t tc_decode_extra_ws(const LayerTable& lt, int batch);
 int tc_decode_launches(const LayerTable& lt);
@@ -179,7 +180,7 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const
   const LayerTable lt = make_table(desc);
   const size_t need = decode_ws_bytes(lt, batch, sms, desc->dtype);
   if (!workspace || ws_bytes < need || !aligned(workspace, 256)) return DCK_ERR_WORKSPACE;
-  if (!simt_supports(lt)) return DCK_ERR_UNSUPPORTED;
+  if (!simt_supports(lt) || !combine_supports(lt)) return DCK_ERR_UNSUPPORTED;
 
   DecodeArgs a;
   a.q = q;

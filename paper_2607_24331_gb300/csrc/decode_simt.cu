@@ -211,10 +211,10 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid(a.n_items, lt.Hkv);
-  if (a.ev0 && cudaEventRecordWithFlags(static_cast<cudaEvent_t>(a.ev0), s, cudaEventRecordExternal) != cudaSuccess) return cudaErrorUnknown;
+  if (a.ev0 && record_timing_event(a.ev0, s) != cudaSuccess) return cudaErrorUnknown;
   k<<<grid, kThreads, smem, s>>>(lt, a);
   e = cudaGetLastError();
-  if (e == cudaSuccess && a.ev1) e = cudaEventRecordWithFlags(static_cast<cudaEvent_t>(a.ev1), s, cudaEventRecordExternal);
+  if (e == cudaSuccess && a.ev1) e = record_timing_event(a.ev1, s);
   return e;
 }
 

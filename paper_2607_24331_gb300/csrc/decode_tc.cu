@@ -433,6 +433,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (s == 0 && !(ok = wwait(&sm.a_full[asl], ((a_base + p) / kNA) & 1, abort_flag))) break;
                 const int ssl = s_cnt % kNS;
                 if (!(ok = wwait(&sm.s_full[ssl], (s_cnt / kNS) & 1, abort_flag))) break;
+                DCK_TC_TRACE(14);
                 tc_fence_after();
                 if (lane == 0) {
                   const int w = ta.pc.w[g][p];
@@ -572,6 +573,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               }
             }
           }
+          DCK_TC_TRACE(25);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
@@ -593,6 +595,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(&sm.x_empty[quad][yb]);
           }
+          DCK_TC_TRACE(26);
           ++kh;
         }
         if (!ok) break;
@@ -754,14 +757,32 @@ __global__ void __launch_bounds__(256) absorb_prep_kernel(const LayerTable lt, c
   const int g = lt.head_group[h], s = lt.head_slot[h];
   const int r = lt.grp_rank[g];
   const int64_t ld = (int64_t)lt.grp_nh[g] * kD;
-  const __nv_bfloat16* Bs = static_cast<const __nv_bfloat16*>(a.Bk) + lt.grp_boff[g] + s * kD;
-  __nv_bfloat16* Ws = W + (int64_t)b * wtot + lt.grp_boff[g] + s * kD;
-  for (int idx = threadIdx.x; idx < r * (kD / 2); idx += blockDim.x) {
-    const int k = idx / (kD / 2), i = idx % (kD / 2);
-    const float x = __bfloat162float(Bs[k * ld + i]), y = __bfloat162float(Bs[k * ld + kD / 2 + i]);
-    const float w0 = fmaf(qa[i], x, qb[i] * y);
-    const float w1 = fmaf(qb[i], x, -qa[i] * y);
-    *reinterpret_cast<__nv_bfloat162*>(Ws + k * ld + 2 * i) = __floats2bfloat162_rn(w0, w1);
+  const __nv_bfloat16* __restrict__ Bs = static_cast<const __nv_bfloat16*>(a.Bk) + lt.grp_boff[g] + s * kD;
+  __nv_bfloat16* __restrict__ Ws = W + (int64_t)b * wtot + lt.grp_boff[g] + s * kD;
+  const int total = r * (kD / 2);
+  constexpr int kBatch = 8;  // independent loads in flight per thread
+  for (int base = threadIdx.x; base < total; base += blockDim.x * kBatch) {
+    float x[kBatch], y[kBatch];
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      const int idx = base + u * blockDim.x;
+      x[u] = y[u] = 0.f;
+      if (idx < total) {
+        const int k = idx / (kD / 2), i = idx % (kD / 2);
+        x[u] = __bfloat162float(Bs[k * ld + i]);
+        y[u] = __bfloat162float(Bs[k * ld + kD / 2 + i]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      const int idx = base + u * blockDim.x;
+      if (idx < total) {
+        const int k = idx / (kD / 2), i = idx % (kD / 2);
+        const float w0 = fmaf(qa[i], x[u], qb[i] * y[u]);
+        const float w1 = fmaf(qb[i], x[u], -qa[i] * y[u]);
+        *reinterpret_cast<__nv_bfloat162*>(Ws + k * ld + 2 * i) = __floats2bfloat162_rn(w0, w1);
+      }
+    }
   }
 }
 
@@ -896,7 +917,7 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStre
     if (e != cudaSuccess) return e;
     if (dev_ok) attr_done[dev][fold] = 1;
   }
-  if (a.ev0 && cudaEventRecordWithFlags(static_cast<cudaEvent_t>(a.ev0), s, cudaEventRecordExternal) != cudaSuccess)
+  if (a.ev0 && record_timing_event(a.ev0, s) != cudaSuccess)
     return cudaErrorUnknown;
   cudaError_t e;
   if (fold) {
@@ -919,7 +940,7 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStre
     e = cudaGetLastError();
   }
   if (e == cudaSuccess && a.ev1)
-    e = cudaEventRecordWithFlags(static_cast<cudaEvent_t>(a.ev1), s, cudaEventRecordExternal);
+    e = record_timing_event(a.ev1, s);
   return e;
 }
 
