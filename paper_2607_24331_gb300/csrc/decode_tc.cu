@@ -16,37 +16,45 @@
 //    + sin(t w_i) (b_i x_i - a_i y_i) with (a, b) the halves of q' = R_P q and
 //    (x, y) those of k.  With k = c B_g[:, slot] both brackets are linear in the
 //    latent c, so a per-sequence factor W (columns 2i and 2i+1:
-//    a_i B[:, i] + b_i B[:, i+64] and b_i B[:, i] - a_i B[:, i+64]), prepared by
-//    absorb_prep_kernel, gives Y = C_g W on the tensor cores with the same
-//    flops, and the score is sum_i cos(t w_i) Y[2i] + sin(t w_i) Y[2i+1]: two
-//    FMAs per frequency pair in the epilogue instead of RoPE plus a dot.
+//    a_i B[:, i] + b_i B[:, i+64] and b_i B[:, i] - a_i B[:, i+64]) gives
+//    Y = C_g W on the tensor cores with the same flops, and the score is
+//    sum_i cos(t w_i) Y[2i] + sin(t w_i) Y[2i+1]: two FMAs per frequency pair.
+//
+// Factor pieces (w ranks x 128 columns of one head, w in {64, 32, 16}) are
+// prepared once per call by factor_prep_kernel as the exact 128B-swizzled
+// shared-memory image of the UMMA operand (w * 256 bytes each, in consumption
+// order), so each piece arrives with a single 1-D bulk copy.
 //
 // Scores are in log2 units; the online softmax keeps a per-head reference max
 // that moves only when a tile's max exceeds it by 8 (probabilities <= 256).
-// Once per tile the value latents are absorbed in latent space (Sec. III-D,
-// x W^(v) ~ z_v R_v applied after the sum):
-//   U[:, j] += C_v[tile]^T . P[:, j]     tcgen05.mma, M = 128 rv rows,
-//          N = query heads (padded to 16), K = tokens; U stays in TMEM.
+// The value latents are absorbed in latent space (Sec. III-D, x W^(v) ~ z_v R_v
+// applied after the sum):  U[:, j] += C_v[tile]^T . P[:, j]  (tcgen05.mma,
+// M = 128 rv rows, N = query heads padded to 16, K = tokens; U stays in TMEM).
+// The absorption of tile i is spread over the key groups of tile i+1, one r_v
+// chunk after each of its groups, so value pieces stream steadily.
 // At the end of each sequence segment U, the reference max and the row sum
 // are written as a split partial; the combine kernel merges splits and
 // applies B_v.
 //
-// Warp roles (320 threads):
-//   warp 0     TMA producer: latent pieces of C_g (ring A), factor slices
-//              and C_v pieces (ring S), all through mbarrier rings;
-//   warp 1     TMEM owner and tcgen05.mma issuer (one elected lane);
+// Warp roles (384 threads).  Every TMA or bulk-copy instruction costs its
+// issuing thread a long round trip, so loads are issued by three producer warps,
+// each putting several copies (one per lane) into one instruction:
+//   warp 0     latent pieces of C_g (ring A, all pieces of a group at once)
+//   warp 10    value pieces of C_v (ring V, both halves of an r_v chunk at once)
+//   warp 11    factor pieces (ring W, up to kNW pieces at once)
+//   warp 1     TMEM owner and tcgen05.mma issuer (one elected lane)
 //   warps 2-9  epilogue: each TMEM lane quadrant (32 tokens) is served by two
-//              warps that split the 64 RoPE frequency pairs of a head and
-//              add their partial scores through shared memory.
-// Every wait is bounded (2 s); on expiry the CTA stops issuing work, records
-// kErrTimeout, waits for work in flight and still releases TMEM.
+//              warps that split the 64 RoPE frequency pairs of a head and add
+//              their partial scores with shared-memory atomics.
+// Every wait is bounded (about 2 s); on expiry the CTA stops issuing work,
+// records kErrTimeout, waits for work in flight and still releases TMEM.
 //
-// Shared-memory layouts (all 128B-swizzled unless noted):
+// Shared-memory operand layouts (128B swizzle unless noted):
 //   A slot  [128 tokens][w ranks] K-major, w in {64, 32, 16} with 128/64/32B
 //           swizzle: UMMA operand A of the reconstruction;
-//   S slot  two boxes [64 rows][64 cols]: a factor slice (rows = ranks,
-//           cols = head dims; MN-major operand B) or a C_v piece (rows =
-//           tokens, cols = rv; MN-major operand A of the value absorption);
+//   W slot  [2 halves][w ranks][64 columns] MN-major: operand B;
+//   V pair  two slots [128 tokens][64 rv] (r_v chunk halves), MN-major
+//           operand A of the value absorption;
 //   P       [2 token atoms][Hq_pad heads][64 tokens] bf16, K-major operand B.
 #include <algorithm>
 #include <cstring>
@@ -59,6 +67,9 @@
 #ifndef DCK_TC_TRACE
 #define DCK_TC_TRACE(code) ((void)0)
 #endif
+#ifndef DCK_TC_TRACE_FLUSH
+#define DCK_TC_TRACE_FLUSH() ((void)0)
+#endif
 
 namespace dck {
 namespace {
@@ -66,18 +77,13 @@ namespace {
 using namespace sm100;
 
 constexpr int kD = 128;
-#ifndef DCK_TC_NA
-#define DCK_TC_NA 5
-#endif
-#ifndef DCK_TC_NS
-#define DCK_TC_NS 5
-#endif
-constexpr int kNA = DCK_TC_NA;  // latent-piece ring depth (16 KB slots)
-constexpr int kNS = DCK_TC_NS;  // factor-slice / value-piece ring depth (16 KB slots)
 constexpr int kSlot = 16384;
+constexpr int kNW = 4;            // factor-piece ring depth
+constexpr int kNV = 2;            // value ring depth (one r_v chunk: two halves)
 constexpr int kMaxGroupsTc = 16;
 constexpr int kMaxPieces = 5;
-constexpr int kThreads = 320;
+constexpr int kMaxItems = kMaxKvHeads * kMaxPieces;
+constexpr int kThreads = 384;
 constexpr int kEpiThreads = 256;
 constexpr int kMaxHqTc = 32;
 constexpr float kRescaleThr = 8.f;  // log2 units: probabilities stay <= 256
@@ -87,6 +93,11 @@ constexpr float kTwoPi = 6.28318530717958647692f;
 constexpr float kInvTwoPi = 0.15915494309189533577f;
 constexpr float kLog2e = 1.4426950408889634f;
 
+template <bool kFold>
+struct Ring {
+  static constexpr int NA = kFold ? 5 : 4;  // latent-piece ring depth
+};
+
 struct Pieces {
   int8_t n[kMaxGroupsTc];
   int8_t w[kMaxGroupsTc][kMaxPieces];
@@ -95,33 +106,54 @@ struct Pieces {
 
 struct Maps {
   CUtensorMap kc64, kc32, kc16, vc;
-  CUtensorMap bk[kMaxGroupsTc];  // B_g (key mode, 2-D) or the per-sequence W_g (query-folded mode, 3-D)
 };
 
 struct TcArgs {
   int hq_pad;
   int n_chunks;                  // rv / 128
+  int n_items;                   // factor pieces per tile (sum over groups of n_g * pieces_g)
+  int64_t fimg_seq_bytes;        // factor image bytes per sequence (query-folded mode)
+  const uint8_t* fimg;           // factor images (workspace)
   Pieces pc;
+  int32_t item_off[kMaxItems];   // byte offset of factor piece n in the image
+  int8_t item_w[kMaxItems];      // ranks of factor piece n
   int16_t order[kMaxKvHeads];    // KV head at each (group, slot) position, group-major
+  int8_t chunk_after[kMaxGroupsTc];  // r_v chunks of the previous tile absorbed after group g
 };
 
+// Per-group facts the hot loops need, kept in shared memory: indexing the
+// kernel-parameter tables at run time goes through the small constant cache,
+// which several warps thrash.
+struct GroupSm {
+  int32_t roff;          // first key-cache column of the group
+  int8_t np, ng;         // pieces per head, heads
+  int8_t chunk_after;    // r_v chunks of the previous tile absorbed after this group (cumulative)
+  int8_t pad;
+  int8_t w[kMaxPieces];  // piece widths (ranks)
+  int8_t pad2[3];
+  int16_t k[kMaxPieces]; // first rank of each piece
+};
+
+template <bool kFold>
 struct Smem {
-  uint8_t a[kNA][kSlot];
-  uint8_t s[kNS][kSlot];
+  uint8_t a[Ring<kFold>::NA][kSlot];
+  uint8_t w[kNW][kSlot];
+  uint8_t v[kNV][kSlot];
   uint8_t p[2][2 * kMaxHqTc * 128];
-  float qr[kMaxHqTc * kD];        // key mode: rotated queries * log2(e)/sqrt(d)
-  float x[kMaxHqTc * 128];        // scores [head][token]
-  float y[4][2][kMaxQPerKv][32];  // partial-score hand-off of a quadrant's warp pair
+  float x[kMaxHqTc * 128];                  // scores [head][token], accumulated atomically
+  float qr[kFold ? 1 : kMaxHqTc * kD];      // key mode: rotated queries * log2(e)/sqrt(d)
   double om64[kD / 2];
   float om32[kD / 2];
   float beta[kD / 2];
   float redm[4][kMaxHqTc];
   float redl[4][kMaxHqTc];
-  float alpha[kMaxHqTc];
-  uint64_t a_full[kNA], a_empty[kNA], s_full[kNS], s_empty[kNS];
+  uint64_t a_full[Ring<kFold>::NA], a_empty[Ring<kFold>::NA];
+  uint64_t w_full[kNW], w_empty[kNW], v_full[kNV], v_empty[kNV];
   uint64_t k_full[2], k_empty[2], p_full[2], p_empty[2], u_ready, u_free;
   uint64_t epi_bar;
-  uint64_t x_full[4][2], x_empty[4][2];
+  GroupSm grp[kMaxGroupsTc];
+  int16_t order[kMaxKvHeads];
+  uint32_t item[kMaxItems];  // factor piece n: byte offset | (ranks / 16) << 28
   uint32_t tmem_base;
   int abort_flag;
   int b_first, pre_first, nt_total;
@@ -130,10 +162,50 @@ struct Smem {
 __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void griddep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(pol)
+      : "memory");
+}
+
 // Bounded wait whose outcome is the same in every lane of the warp.
 __device__ __forceinline__ bool wwait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
   const bool r = mbar_wait(bar, parity, abort_flag);
   return __all_sync(0xffffffffu, r);
+}
+
+// Lane 0 waits for the `n` ring slots starting at ring position `cnt` (depth
+// `depth`) to be released; the result is shared with the warp.
+__device__ __forceinline__ bool wait_slots(uint64_t* empty, int depth, int cnt, int n, int lane,
+                                           volatile int* abort_flag) {
+  bool ok = true;
+  if (lane == 0)
+    for (int i = 0; i < n && ok; ++i) {
+      const int c = cnt + i;
+      if (c >= depth) ok = mbar_wait(&empty[c % depth], ((c / depth) - 1) & 1, abort_flag);
+    }
+  return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+}
+
+// Lane 0 waits for ring position `cnt` to be free, then counts how many of the
+// following positions (up to `max_n` in all) are free already, without
+// waiting.  Returns that count to the whole warp, 0 if the wait gave up.  (A
+// position is at most one use ahead of its release, so the parity test
+// cannot see a stale phase.)
+__device__ __forceinline__ int claim_slots(uint64_t* empty, int depth, int cnt, int max_n, int lane,
+                                           volatile int* abort_flag) {
+  int n = 0;
+  if (lane == 0 && (cnt < depth || mbar_wait(&empty[cnt % depth], ((cnt / depth) - 1) & 1, abort_flag))) {
+    n = 1;
+    while (n < max_n) {
+      const int c = cnt + n;
+      if (c >= depth && !mbar_try_wait(&empty[c % depth], ((c / depth) - 1) & 1)) break;
+      ++n;
+    }
+  }
+  return __shfl_sync(0xffffffffu, n, 0);
 }
 
 __device__ __forceinline__ int ntiles_of(const DecodeArgs& a, int b) {
@@ -173,17 +245,6 @@ struct Walker {
 
 __device__ __forceinline__ uint32_t swz_of(int w) { return w == 64 ? kSw128 : (w == 32 ? kSw64 : kSw32); }
 
-__device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-
 // Byte offset of P element (head j, token t) inside one P buffer.
 __device__ __forceinline__ uint32_t p_off(int j, int t, int hq_pad) {
   const int atom = t >> 6, col = t & 63;
@@ -191,68 +252,49 @@ __device__ __forceinline__ uint32_t p_off(int j, int t, int hq_pad) {
 }
 
 // ---------------------------------------------------------------------------
-// producer helper: the C_v pieces of one tile
+// MMA helper (whole MMA warp; lane 0 issues): one r_v chunk of the value
+// absorption of tile `tt`, U[:, chunk c] += C_v[tile, chunk c]^T P
 // ---------------------------------------------------------------------------
 
-__device__ __forceinline__ bool produce_v(Smem& sm, const Maps& maps, int n_chunks, int64_t yrow, int& s_cnt,
-                                          uint64_t pol, volatile int* abort_flag) {
-  for (int c = 0; c < n_chunks; ++c)
-    for (int th = 0; th < 2; ++th) {
-      const int sl = s_cnt % kNS;
-      if (s_cnt >= kNS && !mbar_wait(&sm.s_empty[sl], ((s_cnt / kNS) - 1) & 1, abort_flag)) return false;
-      mbar_expect_tx(&sm.s_full[sl], kSlot);
-      tma_load_2d_hint(sm.s[sl], &maps.vc, &sm.s_full[sl], 128 * c, (int32_t)(yrow + 64 * th), pol);
-      tma_load_2d_hint(sm.s[sl] + kSlot / 2, &maps.vc, &sm.s_full[sl], 128 * c + 64, (int32_t)(yrow + 64 * th), pol);
-      DCK_TC_TRACE(3);
-      ++s_cnt;
-    }
-  return true;
-}
-
-// ---------------------------------------------------------------------------
-// MMA helper (whole MMA warp; lane 0 issues): value absorption of one tile,
-// U[:, c-chunk] += C_v^T P
-// ---------------------------------------------------------------------------
-
-__device__ __forceinline__ bool mma_pv(Smem& sm, uint32_t tmem, const TcArgs& ta, int tt, bool first_of_seg,
-                                       int nvalid, int sgc, int& s_cnt, int lane, volatile int* abort_flag) {
+template <bool kFold>
+__device__ __forceinline__ bool mma_pv_chunk(Smem<kFold>& sm, uint32_t tmem, const TcArgs& ta, int tt, int c,
+                                             bool first_of_seg, int nvalid, int sgc, int& v_cnt, int lane,
+                                             volatile int* abort_flag) {
   const int pb = tt & 1;
   const int hq_pad = ta.hq_pad;
-  if (!wwait(&sm.p_full[pb], (tt >> 1) & 1, abort_flag)) return false;
-  if (first_of_seg && sgc > 0 && !wwait(&sm.u_free, (sgc - 1) & 1, abort_flag)) return false;
+  if (c == 0) {
+    if (!wwait(&sm.p_full[pb], (tt >> 1) & 1, abort_flag)) return false;
+    if (first_of_seg && sgc > 0 && !wwait(&sm.u_free, (sgc - 1) & 1, abort_flag)) return false;
+  }
+  // the two halves of chunk c sit in ring slots 0 and 1 (kNV == 2)
+  if (!wwait(&sm.v_full[0], (v_cnt / kNV) & 1, abort_flag)) return false;
+  if (!wwait(&sm.v_full[1], (v_cnt / kNV) & 1, abort_flag)) return false;
+  if (nvalid < 128) {  // rows past the sequence end: make them exact zeros
+    for (int r = nvalid + (lane >> 3); r < 128; r += 4) {
+      reinterpret_cast<uint4*>(sm.v[0] + r * 128)[lane & 7] = make_uint4(0, 0, 0, 0);
+      reinterpret_cast<uint4*>(sm.v[1] + r * 128)[lane & 7] = make_uint4(0, 0, 0, 0);
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+  }
   tc_fence_after();
   DCK_TC_TRACE(12);
-  const uint32_t idesc_v = idesc_bf16(128, hq_pad, true, false);
-  const uint32_t pbase = smem_u32(sm.p[pb]);
-  for (int c = 0; c < ta.n_chunks; ++c)
-    for (int th = 0; th < 2; ++th) {
-      const int sl = s_cnt % kNS;
-      if (!wwait(&sm.s_full[sl], (s_cnt / kNS) & 1, abort_flag)) return false;
-      if (nvalid < 128) {  // rows past the sequence end: make them exact zeros
-        const int r0 = max(0, nvalid - 64 * th);
-        for (int r = r0 + (lane >> 3); r < 64; r += 4) {
-          reinterpret_cast<uint4*>(sm.s[sl] + r * 128)[lane & 7] = make_uint4(0, 0, 0, 0);
-          reinterpret_cast<uint4*>(sm.s[sl] + kSlot / 2 + r * 128)[lane & 7] = make_uint4(0, 0, 0, 0);
-        }
-        fence_proxy_async_smem();
-        __syncwarp();
-      }
-      tc_fence_after();
-      if (lane == 0) {
-        const uint32_t vb = smem_u32(sm.s[sl]);
+  if (lane == 0) {
+    const uint32_t idesc_v = idesc_bf16(128, hq_pad, true, false);
+    const uint32_t pbase = smem_u32(sm.p[pb]);
+    const uint32_t vb = smem_u32(sm.v[0]);
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const uint64_t ad = sdesc(vb + k * 2048, kSlot / 2, 1024, kSw128);
-          const uint64_t bd = sdesc(pbase + th * (hq_pad * 128) + k * 32, 16, 1024, kSw128);
-          umma_f16(tmem + kUCol + c * hq_pad, ad, bd, idesc_v, (first_of_seg && th == 0 && k == 0) ? 0u : 1u);
-        }
-        umma_commit(&sm.s_empty[sl]);
-      }
-      __syncwarp();
-      ++s_cnt;
+    for (int k = 0; k < 8; ++k) {
+      const uint64_t ad = sdesc(vb + k * 2048, kSlot, 1024, kSw128);
+      const uint64_t bd = sdesc(pbase + (k >> 2) * (hq_pad * 128) + (k & 3) * 32, 16, 1024, kSw128);
+      umma_f16(tmem + kUCol + c * hq_pad, ad, bd, idesc_v, (first_of_seg && k == 0) ? 0u : 1u);
     }
-  if (lane == 0) umma_commit(&sm.p_empty[pb]);
+    umma_commit(&sm.v_empty[0]);
+    umma_commit(&sm.v_empty[1]);
+    if (c == ta.n_chunks - 1) umma_commit(&sm.p_empty[pb]);
+  }
   __syncwarp();
+  v_cnt += kNV;
   DCK_TC_TRACE(13);
   return true;
 }
@@ -264,8 +306,10 @@ __device__ __forceinline__ bool mma_pv(Smem& sm, uint32_t tmem, const TcArgs& ta
 template <bool kFold>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tc_kernel(const __grid_constant__ Maps maps, const LayerTable lt, const DecodeArgs a, const TcArgs ta) {
+  constexpr int NA = Ring<kFold>::NA;
   extern __shared__ uint8_t smem_raw[];
-  Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  Smem<kFold>& sm =
+      *reinterpret_cast<Smem<kFold>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   volatile int* abort_flag = &sm.abort_flag;
   const int hq_pad = ta.hq_pad;
@@ -273,13 +317,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // ---- setup -------------------------------------------------------------
   if (tid == 0) {
-    for (int i = 0; i < kNA; ++i) {
+    for (int i = 0; i < NA; ++i) {
       mbar_init(&sm.a_full[i], 1);
       mbar_init(&sm.a_empty[i], 1);
     }
-    for (int i = 0; i < kNS; ++i) {
-      mbar_init(&sm.s_full[i], 1);
-      mbar_init(&sm.s_empty[i], 1);
+    for (int i = 0; i < kNW; ++i) {
+      mbar_init(&sm.w_full[i], 1);
+      mbar_init(&sm.w_empty[i], 1);
+    }
+    for (int i = 0; i < kNV; ++i) {
+      mbar_init(&sm.v_full[i], 1);
+      mbar_init(&sm.v_empty[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sm.k_full[i], 1);
@@ -290,11 +338,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&sm.u_ready, 1);
     mbar_init(&sm.u_free, kEpiThreads / 32);
     mbar_init(&sm.epi_bar, kEpiThreads / 32);
-    for (int q = 0; q < 4; ++q)
-      for (int i = 0; i < 2; ++i) {
-        mbar_init(&sm.x_full[q][i], 1);
-        mbar_init(&sm.x_empty[q][i], 1);
-      }
     sm.abort_flag = 0;
     fence_mbar_init();
   }
@@ -302,10 +345,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(&sm.tmem_base, kTmemCols);
     tmem_relinquish();
   }
-  {  // P buffers start at zero (padded head rows stay zero)
+  {  // P buffers start at zero (padded head rows stay zero); scores start at zero
     uint4* pz = reinterpret_cast<uint4*>(&sm.p[0][0]);
     for (int i = tid; i < (int)(sizeof(sm.p) / 16); i += kThreads) pz[i] = make_uint4(0, 0, 0, 0);
   }
+  if (tid < lt.G) {
+    GroupSm& gs = sm.grp[tid];
+    gs.roff = lt.grp_roff[tid];
+    gs.np = ta.pc.n[tid];
+    gs.ng = (int8_t)lt.grp_nh[tid];
+    gs.chunk_after = ta.chunk_after[tid];
+    for (int p = 0; p < kMaxPieces; ++p) {
+      gs.w[p] = ta.pc.w[tid][p];
+      gs.k[p] = ta.pc.k[tid][p];
+    }
+  }
+  if (tid < lt.Hkv) sm.order[tid] = ta.order[tid];
+  for (int n = tid; n < ta.n_items; n += kThreads)
+    sm.item[n] = (uint32_t)ta.item_off[n] | ((uint32_t)(ta.item_w[n] / 16) << 28);
   if (tid < kD / 2) {
     const double om = exp2(-2.0 * tid / kD * log2((double)a.theta));
     sm.om64[tid] = om;
@@ -349,6 +406,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       run += nt;
     }
+    __syncthreads();
+    for (int i = tid; i < kMaxHqTc * 128; i += kThreads) sm.x[i] = 0.f;
   }
   tc_fence_before();
   __syncthreads();
@@ -359,132 +418,172 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int x1 = item_begin(blockIdx.x + 1, NT, a.n_items);
   Walker walk{sm.b_first, sm.pre_first, x0, x1};
   Segment seg;
+  DCK_TC_TRACE(0);
 
   if (warp == 0) {
-    // ---- TMA producer (one lane) ------------------------------------------
-    if (lane == 0 && x0 < x1) {
-      const uint64_t pol_stream = policy_evict_first();
-      const uint64_t pol_keep = policy_evict_last();
-      if (kFold) griddep_wait();  // W is written by the preparation kernel
-      int a_cnt = 0, s_cnt = 0;
+    // ---- latent pieces: all pieces of a group in one instruction -----------
+    if (x0 < x1) {
+      const uint64_t pol = policy_evict_first();
+      int a_cnt = 0;
       bool ok = true;
       while (ok && walk.next(a, seg)) {
         for (int i = 0; i < seg.ntiles && ok; ++i) {
           const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
           for (int g = 0; g < lt.G && ok; ++g) {
-            const int np = ta.pc.n[g];
-            for (int p = 0; p < np && ok; ++p) {
-              const int sl = a_cnt % kNA;
-              if (a_cnt >= kNA && !(ok = mbar_wait(&sm.a_empty[sl], ((a_cnt / kNA) - 1) & 1, abort_flag))) break;
-              const int w = ta.pc.w[g][p];
-              const CUtensorMap* m = w == 64 ? &maps.kc64 : (w == 32 ? &maps.kc32 : &maps.kc16);
-              mbar_expect_tx(&sm.a_full[sl], kTile * w * 2);
-              tma_load_2d_hint(sm.a[sl], m, &sm.a_full[sl], lt.grp_roff[g] + ta.pc.k[g][p], (int32_t)yrow,
-                               pol_stream);
-              DCK_TC_TRACE(1);
-              ++a_cnt;
-            }
-            const int ng = lt.grp_nh[g];
-            for (int s = 0; s < ng && ok; ++s)
-              for (int p = 0; p < np && ok; ++p) {
-                const int sl = s_cnt % kNS;
-                if (s_cnt >= kNS && !(ok = mbar_wait(&sm.s_empty[sl], ((s_cnt / kNS) - 1) & 1, abort_flag))) break;
-                mbar_expect_tx(&sm.s_full[sl], kSlot);
-                if (kFold) {
-                  tma_load_3d_hint(sm.s[sl], &maps.bk[g], &sm.s_full[sl], s * kD, ta.pc.k[g][p], seg.b, pol_keep);
-                  tma_load_3d_hint(sm.s[sl] + kSlot / 2, &maps.bk[g], &sm.s_full[sl], s * kD + 64, ta.pc.k[g][p],
-                                   seg.b, pol_keep);
-                } else {
-                  tma_load_2d_hint(sm.s[sl], &maps.bk[g], &sm.s_full[sl], s * kD, ta.pc.k[g][p], pol_keep);
-                  tma_load_2d_hint(sm.s[sl] + kSlot / 2, &maps.bk[g], &sm.s_full[sl], s * kD + 64, ta.pc.k[g][p],
-                                   pol_keep);
-                }
-                DCK_TC_TRACE(2);
-                ++s_cnt;
+            const GroupSm& gs = sm.grp[g];
+            const int np = gs.np;
+            for (int p0 = 0; p0 < np && ok;) {
+              const int nb = claim_slots(sm.a_empty, NA, a_cnt, np - p0, lane, abort_flag);
+              ok = nb > 0;
+              if (!ok) break;
+              if (lane < nb) {
+                const int sl = (a_cnt + lane) % NA;
+                const int w = gs.w[p0 + lane];
+                const CUtensorMap* m = w == 64 ? &maps.kc64 : (w == 32 ? &maps.kc32 : &maps.kc16);
+                mbar_expect_tx(&sm.a_full[sl], kTile * w * 2);
+                tma_load_2d_hint(sm.a[sl], m, &sm.a_full[sl], gs.roff + gs.k[p0 + lane], (int32_t)yrow, pol);
               }
-            if (ok && g == 0 && i > 0)
-              ok = produce_v(sm, maps, ta.n_chunks, yrow - kTile, s_cnt, pol_stream, abort_flag);
+              __syncwarp();
+              DCK_TC_TRACE(300 + nb);
+              a_cnt += nb;
+              p0 += nb;
+            }
           }
         }
-        if (ok)
-          ok = produce_v(sm, maps, ta.n_chunks, seg.row0 + seg.t_begin + (int64_t)kTile * (seg.ntiles - 1), s_cnt,
-                         pol_stream, abort_flag);
+      }
+    }
+  } else if (warp == 10) {
+    // ---- value pieces: both halves of an r_v chunk in one instruction -------
+    if (x0 < x1) {
+      const uint64_t pol = policy_evict_first();
+      int v_cnt = 0;
+      bool ok = true;
+      while (ok && walk.next(a, seg)) {
+        for (int i = 0; i < seg.ntiles && ok; ++i) {
+          const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
+          for (int c = 0; c < ta.n_chunks && ok; ++c) {
+            if (!(ok = wait_slots(sm.v_empty, kNV, v_cnt, kNV, lane, abort_flag))) break;
+            if (lane < kNV) {
+              mbar_expect_tx(&sm.v_full[lane], kSlot);
+              tma_load_2d_hint(sm.v[lane], &maps.vc, &sm.v_full[lane], 128 * c + 64 * lane, (int32_t)yrow, pol);
+            }
+            __syncwarp();
+            DCK_TC_TRACE(3);
+            v_cnt += kNV;
+          }
+        }
+      }
+    }
+  } else if (warp == 11) {
+    // ---- factor pieces: up to kNW 16 KB images per instruction -------------
+    if (x0 < x1) {
+      const uint64_t pol = policy_evict_last();
+      griddep_wait();  // the images are written by the preparation kernel
+      int w_cnt = 0;
+      bool ok = true;
+      while (ok && walk.next(a, seg)) {
+        const uint8_t* img = ta.fimg + (kFold ? (int64_t)seg.b * ta.fimg_seq_bytes : 0);
+        for (int i = 0; i < seg.ntiles && ok; ++i) {
+          for (int n0 = 0; n0 < ta.n_items && ok;) {
+            const int nb = claim_slots(sm.w_empty, kNW, w_cnt, min(kNW, ta.n_items - n0), lane, abort_flag);
+            ok = nb > 0;
+            if (!ok) break;
+            if (lane < nb) {
+              const int sl = (w_cnt + lane) % kNW;
+              const uint32_t it = sm.item[n0 + lane];
+              const uint32_t bytes = (it >> 28) << 12;
+              mbar_expect_tx(&sm.w_full[sl], bytes);
+              bulk_load(sm.w[sl], img + (it & 0x0FFFFFFFu), bytes, &sm.w_full[sl], pol);
+            }
+            __syncwarp();
+            DCK_TC_TRACE(200 + nb);
+            w_cnt += nb;
+            n0 += nb;
+          }
+        }
       }
     }
   } else if (warp == 1) {
     // ---- MMA issuer (whole warp follows, lane 0 issues) ---------------------
     if (x0 < x1) {
       const uint32_t idesc_k = idesc_bf16(128, kD, false, true);
-      int a_cnt = 0, s_cnt = 0, kh = 0, tl = 0, sgc = 0;
+      int a_cnt = 0, w_cnt = 0, v_cnt = 0, kh = 0, tl = 0, sgc = 0;
       bool ok = true;
       while (ok && walk.next(a, seg)) {
         const int tl_first = tl;
         for (int i = 0; i < seg.ntiles && ok; ++i) {
+          int c_next = 0;  // next r_v chunk of the previous tile to absorb
           for (int g = 0; g < lt.G && ok; ++g) {
-            const int np = ta.pc.n[g];
+            const GroupSm& gs = sm.grp[g];
+            const int np = gs.np;
             const int a_base = a_cnt;
-            const int ng = lt.grp_nh[g];
+            const int ng = gs.ng;
             for (int s = 0; s < ng && ok; ++s) {
               const int buf = kh & 1;
               if (kh >= 2 && !(ok = wwait(&sm.k_empty[buf], ((kh >> 1) - 1) & 1, abort_flag))) break;
               DCK_TC_TRACE(10);
               for (int p = 0; p < np && ok; ++p) {
-                const int asl = (a_base + p) % kNA;
-                if (s == 0 && !(ok = wwait(&sm.a_full[asl], ((a_base + p) / kNA) & 1, abort_flag))) break;
-                const int ssl = s_cnt % kNS;
-                if (!(ok = wwait(&sm.s_full[ssl], (s_cnt / kNS) & 1, abort_flag))) break;
+                const int asl = (a_base + p) % NA;
+                if (s == 0 && !(ok = wwait(&sm.a_full[asl], ((a_base + p) / NA) & 1, abort_flag))) break;
+                DCK_TC_TRACE(15);
+                const int wsl = w_cnt % kNW;
+                if (!(ok = wwait(&sm.w_full[wsl], (w_cnt / kNW) & 1, abort_flag))) break;
                 DCK_TC_TRACE(14);
                 tc_fence_after();
                 if (lane == 0) {
-                  const int w = ta.pc.w[g][p];
+                  DCK_TC_TRACE(17);
+                  const int w = gs.w[p];
                   const uint32_t ab = smem_u32(sm.a[asl]);
-                  const uint32_t bb = smem_u32(sm.s[ssl]);
+                  const uint32_t bb = smem_u32(sm.w[wsl]);
                   const uint32_t swz = swz_of(w);
                   for (int k = 0; k < w / 16; ++k) {
                     const uint64_t ad = sdesc(ab + k * 32, 16, 16 * w, swz);
-                    const uint64_t bd = sdesc(bb + k * 2048, kSlot / 2, 1024, kSw128);
+                    const uint64_t bd = sdesc(bb + k * 2048, 128 * w, 1024, kSw128);
                     umma_f16(tmem + buf * kD, ad, bd, idesc_k, (p > 0 || k > 0) ? 1u : 0u);
                   }
-                  umma_commit(&sm.s_empty[ssl]);
+                  DCK_TC_TRACE(18);
+                  umma_commit(&sm.w_empty[wsl]);
+                  if (s == ng - 1) umma_commit(&sm.a_empty[asl]);  // last head: piece done
+                  DCK_TC_TRACE(16);
                 }
                 __syncwarp();
-                ++s_cnt;
+                ++w_cnt;
               }
               if (ok && lane == 0) umma_commit(&sm.k_full[buf]);
               __syncwarp();
               DCK_TC_TRACE(11);
               ++kh;
             }
-            if (ok && lane == 0)
-              for (int p = 0; p < np; ++p) umma_commit(&sm.a_empty[(a_base + p) % kNA]);
-            __syncwarp();
             a_cnt += np;
-            if (ok && g == 0 && i > 0)
-              ok = mma_pv(sm, tmem, ta, tl - 1, tl - 1 == tl_first, 128, sgc, s_cnt, lane, abort_flag);
+            if (i > 0)  // absorb the previous tile's chunks scheduled after this group
+              for (; ok && c_next < gs.chunk_after; ++c_next)
+                ok = mma_pv_chunk<kFold>(sm, tmem, ta, tl - 1, c_next, tl - 1 == tl_first, 128, sgc, v_cnt, lane,
+                                          abort_flag);
           }
           ++tl;
         }
         if (ok) {
           const int nvalid = seg.t_end - (seg.t_begin + kTile * (seg.ntiles - 1));
-          ok = mma_pv(sm, tmem, ta, tl - 1, tl - 1 == tl_first, nvalid, sgc, s_cnt, lane, abort_flag);
+          for (int c = 0; ok && c < ta.n_chunks; ++c)
+            ok = mma_pv_chunk<kFold>(sm, tmem, ta, tl - 1, c, tl - 1 == tl_first, nvalid, sgc, v_cnt, lane,
+                                      abort_flag);
         }
         if (ok && lane == 0) umma_commit(&sm.u_ready);
         __syncwarp();
         ++sgc;
       }
     }
-  } else {
+  } else if (warp >= 2 && warp <= 9) {
     // ---- epilogue: RoPE, scores, softmax, P, U readout ----------------------
     const int e = tid - 64;              // 0 .. 255
     const int quad = warp & 3;           // TMEM lane quadrant
     const int hf = (warp - 2) >> 2;      // frequency half, then head half
     const int tau = quad * 32 + lane;    // token row inside the tile
-    const int hh = hq_pad / 2;           // heads owned after the hand-off
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     int kh = 0, tl = 0, sgc = 0, round = 0;
     bool ok = true;
-    float m_ref[kMaxHqTc / 2];
-    float l_acc[kMaxHqTc / 2];
+    float m_ref[16];  // reference max of heads 16 hf + u (log2 units)
+    const int jb0 = 16 * hf;  // heads owned at tile and segment ends
 #define EPI_SYNC()                                  \
   do {                                              \
     __syncwarp();                                   \
@@ -508,23 +607,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
 #pragma unroll
-      for (int u = 0; u < kMaxHqTc / 2; ++u) {
-        m_ref[u] = -INFINITY;
-        l_acc[u] = 0.f;
+      for (int u = 0; u < 16; ++u) m_ref[u] = -INFINITY;
+      // RoPE angle of token t0+tau and pair p: (t0*w_p mod 2pi, fp64) + tau*w_p (fp32);
+      // the offsets beta of later tiles are written at the previous tile's end
+      if (e < kD / 2) {
+        const double ang = (double)seg.t_begin * sm.om64[e];
+        sm.beta[e] = (float)(ang - 6.283185307179586 * floor(ang * 0.15915494309189535));
       }
       EPI_SYNC();
       if (!ok) break;
+      // running row sums: one per (quadrant, head), kept by the warp owning both
+      if (lane < 16 && 16 * hf + lane < Hq) sm.redl[quad][16 * hf + lane] = 0.f;
       const int tl_first = tl;
       for (int i = 0; i < seg.ntiles && ok; ++i) {
         const int t0 = seg.t_begin + kTile * i;
         const bool valid = t0 + tau < seg.t_end;
-        // RoPE angle of token t0+tau and pair p: (t0*w_p mod 2pi, fp64) + tau*w_p (fp32)
-        if (e < kD / 2) {
-          const double ang = (double)t0 * sm.om64[e];
-          sm.beta[e] = (float)(ang - 6.283185307179586 * floor(ang * 0.15915494309189535));
-        }
-        EPI_SYNC();
-        if (!ok) break;
         float cs[32], sn[32];
 #pragma unroll
         for (int ip = 0; ip < 32; ++ip) {
@@ -533,139 +630,158 @@ __global__ void __launch_bounds__(kThreads, 1)
           ph = fmaf(-kTwoPi, rintf(ph * kInvTwoPi), ph);
           __sincosf(ph, &sn[ip], &cs[ip]);
         }
-        // per KV head, in MMA order
+        // per KV head, in MMA order: partial scores of this frequency half
         for (int hi = 0; hi < lt.Hkv; ++hi) {
           const int buf = kh & 1;
           if (!(ok = wwait(&sm.k_full[buf], (kh >> 1) & 1, abort_flag))) break;
           tc_fence_after();
           DCK_TC_TRACE(20);
-          const int j0 = ta.order[hi] * qpg;
-          float part[kMaxQPerKv];
-#pragma unroll
-          for (int jj = 0; jj < kMaxQPerKv; ++jj) part[jj] = 0.f;
+          const int j0 = sm.order[hi] * qpg;
           if (kFold) {
             // Y columns [64 hf, 64 hf + 64): pairs (2i, 2i+1) of my 32 frequencies
+            float y0[32], y1[32];
+            tmem_ld32(tmem + lane_base + buf * kD + 64 * hf, y0);
+            tmem_ld32(tmem + lane_base + buf * kD + 64 * hf + 32, y1);
+            tmem_wait_ld();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
+            float part0 = 0.f, part1 = 0.f;
 #pragma unroll
-            for (int ch = 0; ch < 2; ++ch) {
-              float yv[32];
-              tmem_ld32(tmem + lane_base + buf * kD + 64 * hf + 32 * ch, yv);
-              tmem_wait_ld();
-#pragma unroll
-              for (int i2 = 0; i2 < 16; ++i2)
-                part[0] = fmaf(cs[16 * ch + i2], yv[2 * i2], fmaf(sn[16 * ch + i2], yv[2 * i2 + 1], part[0]));
+            for (int i2 = 0; i2 < 16; ++i2) {
+              part0 = fmaf(cs[i2], y0[2 * i2], fmaf(sn[i2], y0[2 * i2 + 1], part0));
+              part1 = fmaf(cs[16 + i2], y1[2 * i2], fmaf(sn[16 + i2], y1[2 * i2 + 1], part1));
             }
+            atomicAdd(&sm.x[j0 * 128 + tau], part0 + part1);
           } else {
+            // two passes of 16 frequency pairs keep the register footprint small
+            float part[kMaxQPerKv];
 #pragma unroll
-            for (int ch = 0; ch < 2; ++ch) {
-              float k1[16], k2[16];
-              tmem_ld16(tmem + lane_base + buf * kD + 32 * hf + 16 * ch, k1);
-              tmem_ld16(tmem + lane_base + buf * kD + 64 + 32 * hf + 16 * ch, k2);
+            for (int jj = 0; jj < kMaxQPerKv; ++jj) part[jj] = 0.f;
+#pragma unroll
+            for (int ps = 0; ps < 2; ++ps) {
+              float k1v[16], k2v[16];
+              tmem_ld16(tmem + lane_base + buf * kD + 32 * hf + 16 * ps, k1v);
+              tmem_ld16(tmem + lane_base + buf * kD + 64 + 32 * hf + 16 * ps, k2v);
               tmem_wait_ld();
+              if (ps == 1) {
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
+              }
 #pragma unroll
               for (int i2 = 0; i2 < 16; ++i2) {
-                const int ip = 16 * ch + i2;
-                const float r1 = fmaf(k1[i2], cs[ip], -k2[i2] * sn[ip]);
-                const float r2 = fmaf(k1[i2], sn[ip], k2[i2] * cs[ip]);
+                const int ip = 16 * ps + i2;
+                const float r1 = fmaf(k1v[i2], cs[ip], -k2v[i2] * sn[ip]);
+                const float r2 = fmaf(k1v[i2], sn[ip], k2v[i2] * cs[ip]);
                 const float* qrow = sm.qr + j0 * kD + 32 * hf + ip;
 #pragma unroll
                 for (int jj = 0; jj < kMaxQPerKv; ++jj)
                   if (jj < qpg) part[jj] = fmaf(qrow[jj * kD], r1, fmaf(qrow[jj * kD + 64], r2, part[jj]));
               }
             }
+#pragma unroll
+            for (int jj = 0; jj < kMaxQPerKv; ++jj)
+              if (jj < qpg) atomicAdd(&sm.x[(j0 + jj) * 128 + tau], part[jj]);
           }
-          DCK_TC_TRACE(25);
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
           DCK_TC_TRACE(21);
-          // the frequency-half-1 warp hands its partial scores to its partner
-          const int yb = kh & 1, yn = kh >> 1;
-          if (hf == 1) {
-            if (yn >= 1 && !(ok = wwait(&sm.x_empty[quad][yb], (yn - 1) & 1, abort_flag))) break;
-#pragma unroll
-            for (int jj = 0; jj < kMaxQPerKv; ++jj)
-              if (jj < qpg) sm.y[quad][yb][jj][lane] = part[jj];
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sm.x_full[quad][yb]);
-          } else {
-            if (!(ok = wwait(&sm.x_full[quad][yb], yn & 1, abort_flag))) break;
-#pragma unroll
-            for (int jj = 0; jj < kMaxQPerKv; ++jj)
-              if (jj < qpg) sm.x[(j0 + jj) * 128 + tau] = valid ? part[jj] + sm.y[quad][yb][jj][lane] : -INFINITY;
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sm.x_empty[quad][yb]);
-          }
-          DCK_TC_TRACE(26);
           ++kh;
         }
         if (!ok) break;
         // ---- tile end: reference max, optional rescale of U, P -------------
+        // Heads [jb, jb + 16) belong to this warp here (none for hf = 1 when
+        // Hq <= 16); every per-head step runs over all 16 at once so that the
+        // shared-memory and shuffle latencies overlap.
         DCK_TC_TRACE(22);
-        EPI_SYNC();
+        EPI_SYNC();  // every partial score of the tile is in x
         if (!ok) break;
-        float sc[kMaxHqTc / 2];
+        const int jb = jb0;
+        const int nh = max(0, min(16, Hq - jb));
+        float sc[16], mx[16];
 #pragma unroll
-        for (int u = 0; u < kMaxHqTc / 2; ++u) {
-          const int j = hf * hh + u;
-          sc[u] = (u < hh && j < Hq) ? sm.x[j * 128 + tau] : -INFINITY;
-          const float mx = warp_max(sc[u]);
-          if (lane == 0 && u < hh && j < Hq) sm.redm[quad][j] = mx;
+        for (int u = 0; u < 16; ++u) sc[u] = (u < nh && valid) ? sm.x[(jb + u) * 128 + tau] : -INFINITY;
+#pragma unroll
+        for (int u = 0; u < 16; ++u)
+          if (u < nh) sm.x[(jb + u) * 128 + tau] = 0.f;  // ready for the next tile
+#pragma unroll
+        for (int u = 0; u < 16; ++u) mx[u] = sc[u];
+#pragma unroll
+        for (int o = 16; o; o >>= 1)
+#pragma unroll
+          for (int u = 0; u < 16; ++u) mx[u] = fmaxf(mx[u], __shfl_xor_sync(0xffffffffu, mx[u], o));
+        {
+          float v = mx[0];
+#pragma unroll
+          for (int u = 1; u < 16; ++u) v = lane == u ? mx[u] : v;
+          if (lane < nh) sm.redm[quad][jb + lane] = v;
         }
-        EPI_SYNC();
+        if (e < kD / 2 && i + 1 < seg.ntiles) {  // RoPE phase offsets of the next tile
+          const double ang = (double)(t0 + kTile) * sm.om64[e];
+          sm.beta[e] = (float)(ang - 6.283185307179586 * floor(ang * 0.15915494309189535));
+        }
+        EPI_SYNC();  // per-quadrant maxima are in redm
+        DCK_TC_TRACE(28);
         if (!ok) break;
-        float al[kMaxHqTc / 2];
+        float al[16];
+        bool resc = false;
+        {
+          float tm[16];
 #pragma unroll
-        for (int u = 0; u < kMaxHqTc / 2; ++u) {
-          const int j = hf * hh + u;
-          al[u] = 1.f;
-          if (u < hh && j < Hq) {
-            const float tmax = fmaxf(fmaxf(sm.redm[0][j], sm.redm[1][j]), fmaxf(sm.redm[2][j], sm.redm[3][j]));
-            if (m_ref[u] == -INFINITY || tmax > m_ref[u] + kRescaleThr) {
-              al[u] = exp2f(m_ref[u] - tmax);
-              m_ref[u] = tmax;
+          for (int u = 0; u < 16; ++u)
+            tm[u] = u < nh ? fmaxf(fmaxf(sm.redm[0][jb + u], sm.redm[1][jb + u]),
+                                   fmaxf(sm.redm[2][jb + u], sm.redm[3][jb + u]))
+                           : -INFINITY;
+#pragma unroll
+          for (int u = 0; u < 16; ++u) {
+            al[u] = 1.f;
+            if (u < nh && (m_ref[u] == -INFINITY || tm[u] > m_ref[u] + kRescaleThr)) {
+              al[u] = exp2f(m_ref[u] - tm[u]);
+              m_ref[u] = tm[u];
+              resc = true;
             }
-            if (quad == 0 && lane == 0) sm.alpha[j] = al[u];
           }
         }
-        EPI_SYNC();
-        if (!ok) break;
-        bool any = false;
-        if (tl != tl_first)
-          for (int j = 0; j < Hq; ++j) any |= sm.alpha[j] != 1.f;
-        if (any) {
-          // rescale U: the previous tile's absorption must have completed
+        if (resc && tl != tl_first) {
+          // rescale this warp's heads of U; the previous tile's absorption must be complete
           const int tp = tl - 1;
           if (!(ok = wwait(&sm.p_empty[tp & 1], (tp >> 1) & 1, abort_flag))) break;
           tc_fence_after();
-          for (int c = hf; c < ta.n_chunks; c += 2)
-            for (int cb = 0; cb < hq_pad / 16; ++cb) {
-              float v[16];
-              const uint32_t tad = tmem + lane_base + kUCol + c * hq_pad + 16 * cb;
-              tmem_ld16(tad, v);
-              tmem_wait_ld();
+          for (int c = 0; c < ta.n_chunks; ++c) {
+            float v[16];
+            const uint32_t tad = tmem + lane_base + kUCol + c * hq_pad + jb;
+            tmem_ld16(tad, v);
+            tmem_wait_ld();
 #pragma unroll
-              for (int i2 = 0; i2 < 16; ++i2) {
-                const int j = 16 * cb + i2;
-                v[i2] *= (j < Hq) ? sm.alpha[j] : 1.f;
-              }
-              tmem_st16(tad, v);
-            }
+            for (int i2 = 0; i2 < 16; ++i2) v[i2] *= al[i2];
+            tmem_st16(tad, v);
+          }
           tmem_wait_st();
           tc_fence_before();
         }
         // probabilities -> P (bf16); row sums use the rounded values
         const int pb = tl & 1;
         if (tl >= 2 && !(ok = wwait(&sm.p_empty[pb], ((tl - 2) >> 1) & 1, abort_flag))) break;
+        DCK_TC_TRACE(30);
         uint8_t* pbuf = sm.p[pb];
+        float ps[16];
 #pragma unroll
-        for (int u = 0; u < kMaxHqTc / 2; ++u) {
-          const int j = hf * hh + u;
-          if (u < hh && j < Hq) {
-            l_acc[u] *= al[u];
-            const __nv_bfloat16 pv = __float2bfloat16_rn(exp2f(sc[u] - m_ref[u]));
-            l_acc[u] += __bfloat162float(pv);
-            *reinterpret_cast<__nv_bfloat16*>(pbuf + p_off(j, tau, hq_pad)) = pv;
+        for (int u = 0; u < 16; ++u) {
+          const __nv_bfloat16 pv = __float2bfloat16_rn(exp2f(sc[u] - m_ref[u]));
+          if (u < nh) *reinterpret_cast<__nv_bfloat16*>(pbuf + p_off(jb + u, tau, hq_pad)) = pv;
+          ps[u] = u < nh ? __bfloat162float(pv) : 0.f;
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1)
+#pragma unroll
+          for (int u = 0; u < 16; ++u) ps[u] += __shfl_xor_sync(0xffffffffu, ps[u], o);
+        {
+          float v = ps[0], a1 = al[0];
+#pragma unroll
+          for (int u = 1; u < 16; ++u) {
+            v = lane == u ? ps[u] : v;
+            a1 = lane == u ? al[u] : a1;
           }
+          if (lane < nh) sm.redl[quad][jb + lane] = fmaf(sm.redl[quad][jb + lane], a1, v);
         }
         fence_proxy_async_smem();
         __syncwarp();
@@ -678,35 +794,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!(ok = wwait(&sm.u_ready, sgc & 1, abort_flag))) break;
       tc_fence_after();
       const int64_t slot = (int64_t)blockIdx.x + seg.b;
-      for (int c = hf; c < ta.n_chunks; c += 2)
-        for (int cb = 0; cb < hq_pad / 16; ++cb) {
-          float v[16];
-          tmem_ld16(tmem + lane_base + kUCol + c * hq_pad + 16 * cb, v);
-          tmem_wait_ld();
-          const int r = c * 128 + tau;
+      for (int c = hf; c < ta.n_chunks; c += 2) {
+        float v0[16], v1[16];
+        tmem_ld16(tmem + lane_base + kUCol + c * hq_pad, v0);
+        if (hq_pad > 16) tmem_ld16(tmem + lane_base + kUCol + c * hq_pad + 16, v1);
+        tmem_wait_ld();
+        float* dst = a.part_u + slot * Hq * lt.rv + c * 128 + tau;
 #pragma unroll
-          for (int i2 = 0; i2 < 16; ++i2) {
-            const int j = 16 * cb + i2;
-            if (j < Hq) a.part_u[(slot * Hq + j) * lt.rv + r] = v[i2];
-          }
+        for (int i2 = 0; i2 < 16; ++i2) {
+          if (i2 < Hq) dst[(int64_t)i2 * lt.rv] = v0[i2];
+          if (16 + i2 < Hq) dst[(int64_t)(16 + i2) * lt.rv] = v1[i2];
         }
-      tc_fence_before();
-#pragma unroll
-      for (int u = 0; u < kMaxHqTc / 2; ++u) {
-        const int j = hf * hh + u;
-        const float ls = warp_sum(l_acc[u]);
-        if (lane == 0 && u < hh && j < Hq) sm.redl[quad][j] = ls;
       }
+      tc_fence_before();
       EPI_SYNC();
       if (!ok) break;
-      if (quad == 0 && lane == 0) {
+      if (quad == 0) {
+        float m = m_ref[0];
 #pragma unroll
-        for (int u = 0; u < kMaxHqTc / 2; ++u) {
-          const int j = hf * hh + u;
-          if (u < hh && j < Hq) {
-            a.part_ml[(slot * Hq + j) * 2] = m_ref[u];
-            a.part_ml[(slot * Hq + j) * 2 + 1] = sm.redl[0][j] + sm.redl[1][j] + sm.redl[2][j] + sm.redl[3][j];
-          }
+        for (int u = 1; u < 16; ++u) m = lane == u ? m_ref[u] : m;
+        const int j = jb0 + lane;
+        if (lane < 16 && j < Hq) {
+          a.part_ml[(slot * Hq + j) * 2] = m;
+          a.part_ml[(slot * Hq + j) * 2 + 1] = sm.redl[0][j] + sm.redl[1][j] + sm.redl[2][j] + sm.redl[3][j];
         }
       }
       __syncwarp();
@@ -717,10 +827,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   tc_fence_before();
   __syncthreads();
+  DCK_TC_TRACE_FLUSH();
   if (sm.abort_flag) {
     // let copies and MMAs already in flight land before the memory is released
-    const uint64_t t0 = global_timer_ns();
-    while (global_timer_ns() - t0 < 2000000ull) {
+    const long long c0 = clock64();
+    while (clock64() - c0 < 4000000ll) {
     }
     if (tid == 0) atomicOr(a.err, kErrTimeout);
   }
@@ -731,58 +842,85 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// Per-sequence query-folded factor of every head (one query head per KV head):
-// W_b[g][k][s*128 + 2i]     = a_i B_g[k][s*128 + i] + b_i B_g[k][s*128 + 64 + i]
-// W_b[g][k][s*128 + 2i + 1] = b_i B_g[k][s*128 + i] - a_i B_g[k][s*128 + 64 + i]
-// with (a, b) the halves of RoPE(q_h, L_b - 1) * log2(e)/sqrt(d) (fp64 angles).
-__global__ void __launch_bounds__(256) absorb_prep_kernel(const LayerTable lt, const DecodeArgs a,
-                                                          __nv_bfloat16* __restrict__ W, int64_t wtot) {
+// ---------------------------------------------------------------------------
+// factor images
+// ---------------------------------------------------------------------------
+
+struct PrepArgs {
+  int n_items;
+  int16_t item_g[kMaxItems];   // group of factor piece n
+  int16_t item_s[kMaxItems];   // head slot of piece n in its group
+  int16_t item_k[kMaxItems];   // first rank of piece n
+  int8_t item_w[kMaxItems];    // ranks of piece n
+  int32_t item_off[kMaxItems];  // byte offset of piece n in a sequence's image
+  int64_t seq_bytes;
+};
+
+// One block writes one piece image of w * 256 bytes: [2 halves][w rank rows]
+// [64 columns] bf16, 128B-swizzled (16-byte chunk c of row r stored at chunk
+// c ^ (r % 8); w * 128 is a multiple of the 1024-byte swizzle atom).
+// Key mode: columns of B_g[:, slot].
+// Query-folded mode (one block row per sequence b): columns 2i and 2i+1 are
+//   a_i B[:, i] + b_i B[:, i+64]  and  b_i B[:, i] - a_i B[:, i+64]
+// with (a, b) the halves of RoPE(q_{b,h}, L_b - 1) * log2(e)/sqrt(d).
+template <bool kFold>
+__global__ void __launch_bounds__(256) factor_prep_kernel(const LayerTable lt, const DecodeArgs a, const PrepArgs pa,
+                                                          uint8_t* __restrict__ img) {
   griddep_launch();
-  const int h = blockIdx.x, b = blockIdx.y;
-  const int L = valid_len(a.seq_len, a.seq_start, b, a.n_rows);
-  if (L == 0) return;  // no tile of this sequence is ever processed
+  const int n = blockIdx.x, b = blockIdx.y;
+  const int g = pa.item_g[n], s = pa.item_s[n], k0 = pa.item_k[n], wr = pa.item_w[n];
   __shared__ float qa[kD / 2], qb[kD / 2];
-  if (threadIdx.x < kD / 2) {
-    const int i = threadIdx.x;
-    const double om = exp2(-2.0 * i / kD * log2((double)a.theta));
-    double sn, cs;
-    sincos((double)(L - 1) * om, &sn, &cs);
-    const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(a.q) + ((int64_t)b * lt.Hq + h) * kD;
-    const double x1 = __bfloat162float(q[i]), x2 = __bfloat162float(q[i + kD / 2]);
-    const float sc = kLog2e * rsqrtf((float)kD);
-    qa[i] = (float)(x1 * cs - x2 * sn) * sc;
-    qb[i] = (float)(x1 * sn + x2 * cs) * sc;
+  if (kFold) {
+    int kv = 0;
+    for (int hh = 0; hh < lt.Hkv; ++hh)
+      if (lt.head_group[hh] == g && lt.head_slot[hh] == s) kv = hh;
+    const int L = valid_len(a.seq_len, a.seq_start, b, a.n_rows);
+    if (L == 0) return;  // no tile of this sequence is ever processed
+    if (threadIdx.x < kD / 2) {
+      const int i = threadIdx.x;
+      const double om = exp2(-2.0 * i / kD * log2((double)a.theta));
+      double sn, cs;
+      sincos((double)(L - 1) * om, &sn, &cs);
+      const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(a.q) + ((int64_t)b * lt.Hq + kv) * kD;
+      const double x1 = __bfloat162float(q[i]), x2 = __bfloat162float(q[i + kD / 2]);
+      const float sc = kLog2e * rsqrtf((float)kD);
+      qa[i] = (float)(x1 * cs - x2 * sn) * sc;
+      qb[i] = (float)(x1 * sn + x2 * cs) * sc;
+    }
+    __syncthreads();
   }
-  __syncthreads();
-  const int g = lt.head_group[h], s = lt.head_slot[h];
-  const int r = lt.grp_rank[g];
   const int64_t ld = (int64_t)lt.grp_nh[g] * kD;
   const __nv_bfloat16* __restrict__ Bs = static_cast<const __nv_bfloat16*>(a.Bk) + lt.grp_boff[g] + s * kD;
-  __nv_bfloat16* __restrict__ Ws = W + (int64_t)b * wtot + lt.grp_boff[g] + s * kD;
-  const int total = r * (kD / 2);
-  constexpr int kBatch = 8;  // independent loads in flight per thread
-  for (int base = threadIdx.x; base < total; base += blockDim.x * kBatch) {
-    float x[kBatch], y[kBatch];
+  uint8_t* dst = img + (kFold ? (int64_t)b * pa.seq_bytes : 0) + pa.item_off[n];
+  // thread -> (row, 8-column chunk): w rows x 16 chunks (2 halves x 8)
+  for (int idx = threadIdx.x; idx < wr * 16; idx += blockDim.x) {
+    const int r = idx >> 4, ch = idx & 15;
+    const int half = ch >> 3, c8 = ch & 7;
+    float v[8];
+    {
+      const int k = k0 + r;
+      if (kFold) {
+        // output columns col = 64*half + 8*c8 + t, t even/odd -> pair i = col/2
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
-      const int idx = base + u * blockDim.x;
-      x[u] = y[u] = 0.f;
-      if (idx < total) {
-        const int k = idx / (kD / 2), i = idx % (kD / 2);
-        x[u] = __bfloat162float(Bs[k * ld + i]);
-        y[u] = __bfloat162float(Bs[k * ld + kD / 2 + i]);
+        for (int t = 0; t < 8; t += 2) {
+          const int i = (64 * half + 8 * c8 + t) >> 1;
+          const float x = __bfloat162float(Bs[k * ld + i]);
+          const float y = __bfloat162float(Bs[k * ld + kD / 2 + i]);
+          v[t] = fmaf(qa[i], x, qb[i] * y);
+          v[t + 1] = fmaf(qb[i], x, -qa[i] * y);
+        }
+      } else {
+        const uint4 raw = *reinterpret_cast<const uint4*>(Bs + k * ld + 64 * half + 8 * c8);
+        const __nv_bfloat16* h8 = reinterpret_cast<const __nv_bfloat16*>(&raw);
+#pragma unroll
+        for (int t = 0; t < 8; ++t) v[t] = __bfloat162float(h8[t]);
       }
     }
+    uint4 out;
+    __nv_bfloat162* o2 = reinterpret_cast<__nv_bfloat162*>(&out);
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
-      const int idx = base + u * blockDim.x;
-      if (idx < total) {
-        const int k = idx / (kD / 2), i = idx % (kD / 2);
-        const float w0 = fmaf(qa[i], x[u], qb[i] * y[u]);
-        const float w1 = fmaf(qb[i], x[u], -qa[i] * y[u]);
-        *reinterpret_cast<__nv_bfloat162*>(Ws + k * ld + 2 * i) = __floats2bfloat162_rn(w0, w1);
-      }
-    }
+    for (int t = 0; t < 4; ++t) o2[t] = __floats2bfloat162_rn(v[2 * t], v[2 * t + 1]);
+    *reinterpret_cast<uint4*>(dst + half * (wr * 128) + r * 128 + ((c8 ^ (r & 7)) << 4)) = out;
   }
 }
 
@@ -802,21 +940,30 @@ int make_pieces(int r, int8_t* w, int16_t* k) {
 
 int hq_pad_of(int Hq) { return std::max(16, (Hq + 15) / 16 * 16); }
 
-int64_t bk_elems(const LayerTable& lt) {
-  int64_t n = 0;
-  for (int g = 0; g < lt.G; ++g) n += (int64_t)lt.grp_rank[g] * lt.grp_nh[g] * kD;
+int n_items_of(const LayerTable& lt) {
+  int n = 0;
+  for (int g = 0; g < lt.G; ++g) {
+    int8_t w[kMaxPieces];
+    int16_t k[kMaxPieces];
+    n += lt.grp_nh[g] * make_pieces(lt.grp_rank[g], w, k);
+  }
+  return n;
+}
+
+// Bytes of one copy of all factor images: sum over heads of r_g * 128 columns * 2.
+size_t image_bytes_of(const LayerTable& lt) {
+  size_t n = 0;
+  for (int g = 0; g < lt.G; ++g) n += (size_t)lt.grp_nh[g] * lt.grp_rank[g] * 256;
   return n;
 }
 
 // Tensor maps depend only on the buffers and the layer: cache the last few.
 struct MapsKey {
-  const void *kc, *vc, *bk;
+  const void *kc, *vc;
   int64_t n_rows;
-  int Rk, rv, G, B;
-  int64_t sig;
+  int Rk, rv;
   bool operator==(const MapsKey& o) const {
-    return kc == o.kc && vc == o.vc && bk == o.bk && n_rows == o.n_rows && Rk == o.Rk && rv == o.rv && G == o.G &&
-           B == o.B && sig == o.sig;
+    return kc == o.kc && vc == o.vc && n_rows == o.n_rows && Rk == o.Rk && rv == o.rv;
   }
 };
 constexpr int kMapsCache = 64;
@@ -825,26 +972,50 @@ MapsKey g_maps_key[kMapsCache];
 Maps g_maps_val[kMapsCache];
 int g_maps_n = 0, g_maps_next = 0;
 
-bool build_maps(const LayerTable& lt, const DecodeArgs& a, bool fold, Maps& maps) {
+bool build_maps(const LayerTable& lt, const DecodeArgs& a, Maps& maps) {
   std::memset(&maps, 0, sizeof(maps));
   const uint64_t rows = (uint64_t)std::max<int64_t>(1, a.n_rows);
-  bool ok = make_tmap_2d_bf16(&maps.kc64, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 64, kTile, CU_TENSOR_MAP_SWIZZLE_128B) &&
-            make_tmap_2d_bf16(&maps.kc32, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 32, kTile, CU_TENSOR_MAP_SWIZZLE_64B) &&
-            make_tmap_2d_bf16(&maps.kc16, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 16, kTile, CU_TENSOR_MAP_SWIZZLE_32B) &&
-            make_tmap_2d_bf16(&maps.vc, a.vc, lt.rv, rows, (uint64_t)lt.rv * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B);
-  const int64_t wtot = bk_elems(lt);
-  for (int g = 0; g < lt.G && ok; ++g) {
-    const uint64_t cols = (uint64_t)lt.grp_nh[g] * kD;
-    if (fold) {
-      const __nv_bfloat16* base = static_cast<const __nv_bfloat16*>(a.extra) + lt.grp_boff[g];
-      ok = make_tmap_3d_bf16(&maps.bk[g], base, cols, lt.grp_rank[g], a.B, cols * 2, (uint64_t)wtot * 2, 64, 64,
-                             CU_TENSOR_MAP_SWIZZLE_128B);
-    } else {
-      const __nv_bfloat16* base = static_cast<const __nv_bfloat16*>(a.Bk) + lt.grp_boff[g];
-      ok = make_tmap_2d_bf16(&maps.bk[g], base, cols, lt.grp_rank[g], cols * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B);
-    }
+  return make_tmap_2d_bf16(&maps.kc64, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 64, kTile, CU_TENSOR_MAP_SWIZZLE_128B) &&
+         make_tmap_2d_bf16(&maps.kc32, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 32, kTile, CU_TENSOR_MAP_SWIZZLE_64B) &&
+         make_tmap_2d_bf16(&maps.kc16, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 16, kTile, CU_TENSOR_MAP_SWIZZLE_32B) &&
+         make_tmap_2d_bf16(&maps.vc, a.vc, lt.rv, rows, (uint64_t)lt.rv * 2, 64, kTile, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+static_assert(sizeof(Smem<true>) + 1024 <= 232448, "shared memory of the query-folded kernel");
+static_assert(sizeof(Smem<false>) + 1024 <= 232448, "shared memory of the key-mode kernel");
+
+template <bool kFold>
+cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& maps, const TcArgs& ta,
+                        const PrepArgs& pa, cudaStream_t s) {
+  const size_t smem = sizeof(Smem<kFold>) + 1024;
+  static int attr_done[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const bool dev_ok = dev >= 0 && dev < 64;
+  if (!dev_ok || !attr_done[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kFold>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    if (dev_ok) attr_done[dev] = 1;
   }
-  return ok;
+  if (a.ev0 && record_timing_event(a.ev0, s) != cudaSuccess) return cudaErrorUnknown;
+  factor_prep_kernel<kFold><<<dim3(pa.n_items, kFold ? a.B : 1), 256, 0, s>>>(lt, a, pa,
+                                                                                static_cast<uint8_t*>(a.extra));
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.n_items);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, decode_tc_kernel<kFold>, maps, lt, a, ta);
+  if (e == cudaSuccess && a.ev1) e = record_timing_event(a.ev1, s);
+  return e;
 }
 
 }  // namespace
@@ -856,36 +1027,57 @@ bool tc_decode_supports(const LayerTable& lt, int dtype) {
   for (int g = 0; g < lt.G; ++g) {
     int8_t w[kMaxPieces];
     int16_t k[kMaxPieces];
-    if (lt.grp_rank[g] > 256 || make_pieces(lt.grp_rank[g], w, k) > kMaxPieces) return false;
+    const int np = make_pieces(lt.grp_rank[g], w, k);
+    if (lt.grp_rank[g] > 256 || np > kMaxPieces || np > (lt.qpg == 1 ? Ring<true>::NA : Ring<false>::NA))
+      return false;
   }
-  return true;
+  return n_items_of(lt) <= kMaxItems;
 }
 
-// Extra workspace of the tensor-core path: the per-sequence folded factors.
+// Extra workspace of the tensor-core path: the factor piece images.
 size_t tc_decode_extra_ws(const LayerTable& lt, int batch) {
-  if (lt.qpg != 1 || !tc_decode_supports(lt, DCK_BF16)) return 0;
-  return align_up((size_t)batch * bk_elems(lt) * 2, 256);
+  if (!tc_decode_supports(lt, DCK_BF16)) return 0;
+  const size_t per = image_bytes_of(lt);
+  return align_up(lt.qpg == 1 ? per * std::max(batch, 1) : per, 256);
 }
 
-int tc_decode_launches(const LayerTable& lt) { return lt.qpg == 1 ? 2 : 1; }
+int tc_decode_launches(const LayerTable&) { return 2; }
 
 cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) {
   const bool fold = lt.qpg == 1;
-  if (fold && !a.extra) return cudaErrorInvalidValue;
+  if (!a.extra) return cudaErrorInvalidValue;
   TcArgs ta;
   std::memset(&ta, 0, sizeof(ta));
+  PrepArgs pa;
+  std::memset(&pa, 0, sizeof(pa));
   ta.hq_pad = hq_pad_of(lt.Hq);
   ta.n_chunks = lt.rv / 128;
-  int pos = 0;
+  int pos = 0, item = 0, off = 0;
   for (int g = 0; g < lt.G; ++g) {
     ta.pc.n[g] = (int8_t)make_pieces(lt.grp_rank[g], ta.pc.w[g], ta.pc.k[g]);
-    for (int sl = 0; sl < lt.grp_nh[g]; ++sl)
+    for (int sl = 0; sl < lt.grp_nh[g]; ++sl) {
       for (int h = 0; h < lt.Hkv; ++h)
         if (lt.head_group[h] == g && lt.head_slot[h] == sl) ta.order[pos++] = (int16_t)h;
+      for (int p = 0; p < ta.pc.n[g]; ++p, ++item) {
+        pa.item_g[item] = (int16_t)g;
+        pa.item_s[item] = (int16_t)sl;
+        pa.item_k[item] = ta.pc.k[g][p];
+        pa.item_w[item] = ta.pc.w[g][p];
+        pa.item_off[item] = off;
+        ta.item_w[item] = ta.pc.w[g][p];
+        ta.item_off[item] = off;
+        off += ta.pc.w[g][p] * 256;
+      }
+    }
+    // r_v chunks of the previous tile absorbed after group g (cumulative count)
+    ta.chunk_after[g] = (int8_t)(((int64_t)(g + 1) * ta.n_chunks) / lt.G);
   }
-  int64_t sig = fold ? 1 : 0;
-  for (int g = 0; g < lt.G; ++g) sig = sig * 1000003 + lt.grp_rank[g] * 131 + lt.grp_nh[g] * 7 + lt.grp_boff[g];
-  const MapsKey key{a.kc, a.vc, fold ? a.extra : a.Bk, a.n_rows, lt.Rk, lt.rv, lt.G, fold ? a.B : 0, sig};
+  ta.n_items = item;
+  pa.n_items = item;
+  pa.seq_bytes = off;
+  ta.fimg_seq_bytes = pa.seq_bytes;
+  ta.fimg = static_cast<const uint8_t*>(a.extra);
+  const MapsKey key{a.kc, a.vc, a.n_rows, lt.Rk, lt.rv};
   Maps maps;
   bool have = false;
   {
@@ -897,51 +1089,14 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStre
       }
   }
   if (!have) {
-    if (!build_maps(lt, a, fold, maps)) return cudaErrorInvalidValue;
+    if (!build_maps(lt, a, maps)) return cudaErrorInvalidValue;
     std::lock_guard<std::mutex> lk(g_maps_mu);
     g_maps_key[g_maps_next] = key;
     g_maps_val[g_maps_next] = maps;
     g_maps_next = (g_maps_next + 1) % kMapsCache;
     g_maps_n = std::min(g_maps_n + 1, kMapsCache);
   }
-  const size_t smem = sizeof(Smem) + 1024;
-  static int attr_done[64][2] = {};
-  int dev = 0;
-  cudaGetDevice(&dev);
-  const bool dev_ok = dev >= 0 && dev < 64;
-  if (!dev_ok || !attr_done[dev][fold]) {
-    cudaError_t e = fold ? cudaFuncSetAttribute(decode_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                (int)smem)
-                         : cudaFuncSetAttribute(decode_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                (int)smem);
-    if (e != cudaSuccess) return e;
-    if (dev_ok) attr_done[dev][fold] = 1;
-  }
-  if (a.ev0 && record_timing_event(a.ev0, s) != cudaSuccess)
-    return cudaErrorUnknown;
-  cudaError_t e;
-  if (fold) {
-    absorb_prep_kernel<<<dim3(lt.Hq, a.B), 256, 0, s>>>(lt, a, static_cast<__nv_bfloat16*>(a.extra), bk_elems(lt));
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(a.n_items);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, decode_tc_kernel<true>, maps, lt, a, ta);
-  } else {
-    decode_tc_kernel<false><<<a.n_items, kThreads, smem, s>>>(maps, lt, a, ta);
-    e = cudaGetLastError();
-  }
-  if (e == cudaSuccess && a.ev1)
-    e = record_timing_event(a.ev1, s);
-  return e;
+  return fold ? launch_mode<true>(lt, a, maps, ta, pa, s) : launch_mode<false>(lt, a, maps, ta, pa, s);
 }
 
 }  // namespace dck

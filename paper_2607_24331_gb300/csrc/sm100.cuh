@@ -51,18 +51,20 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Wait for phase `parity` of `bar` to complete, for at most `limit_ns`.  On
-// expiry sets *abort (shared, visible to the CTA) and returns false; a CTA
-// that sees *abort set stops issuing work.
+// Wait for phase `parity` of `bar` to complete, for at most `limit_cycles` SM
+// clock cycles (about 2 s at the GB300's clocks).  On expiry sets *abort
+// (shared, visible to the CTA) and returns false; a CTA that sees *abort set
+// stops issuing work.  The budget is kept with the SM-local clock: reading the
+// global timer costs a long round trip, which would sit on every hand-off.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                          uint64_t limit_ns = 2000000000ull) {
+                                          long long limit_cycles = 4000000000ll) {
   if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = global_timer_ns();
+  const long long c0 = clock64();
   while (true) {
     for (int i = 0; i < 64; ++i)
       if (mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
-    if (global_timer_ns() - t0 > limit_ns) {
+    if (clock64() - c0 > limit_cycles) {
       *abort = 1;
       return false;
     }
