@@ -2,9 +2,12 @@
 //
 // One persistent CTA per SM walks its share of 128-token tiles (see
 // DecodeArgs).  For every tile and every key group g (Sec. III-C) the group's
-// latent tile C_g [128 tokens x r_g] meets, on the tensor cores, one 128-column
-// factor per KV head h of the group (tcgen05.mma, M = 128 tokens, N = 128,
-// K = r_g, fp32 accumulator in TMEM):
+// latent tile C_g [128 tokens x r_g] meets, on the tensor cores, the factor
+// columns of the group's KV heads, two heads per MMA where the group has them
+// (tcgen05.mma, M = 128 tokens, N = 256 or 128, K = r_g, fp32 accumulator in
+// TMEM).  A pair shares every read of the latent operand: one-head MMAs that
+// read fresh shared-memory operands run the tensor pipe at about half rate.
+// Per head:
 //
 //  * key mode (several query heads per KV head): the factor is B_g[:, slot(h)],
 //    the product is the reconstructed key K^_h = C_g B_g[:, slot(h)]
@@ -20,29 +23,32 @@
 //    Y = C_g W on the tensor cores with the same flops, and the score is
 //    sum_i cos(t w_i) Y[2i] + sin(t w_i) Y[2i+1]: two FMAs per frequency pair.
 //
-// Factor pieces (w ranks x 128 columns of one head, w in {64, 32, 16}) are
-// prepared once per call by factor_prep_kernel as the exact 128B-swizzled
-// shared-memory image of the UMMA operand (w * 256 bytes each, in consumption
-// order), so each piece arrives with a single 1-D bulk copy.
+// Factor items (one latent piece's ranks x 128 columns of each head of a
+// unit) are prepared once per call by factor_prep_kernel as the exact
+// 128B-swizzled shared-memory image of the UMMA B operand (heads * ranks * 256
+// bytes each, in consumption order), so each item arrives with one 1-D bulk copy.
 //
 // Scores are in log2 units; the online softmax keeps a per-head reference max
 // that moves only when a tile's max exceeds it by 8 (probabilities <= 256).
 // The value latents are absorbed in latent space (Sec. III-D, x W^(v) ~ z_v R_v
 // applied after the sum):  U[:, j] += C_v[tile]^T . P[:, j]  (tcgen05.mma,
 // M = 128 rv rows, N = query heads padded to 16, K = tokens; U stays in TMEM).
-// The absorption of tile i is spread over the key groups of tile i+1, one r_v
-// chunk after each of its groups, so value pieces stream steadily.
-// At the end of each sequence segment U, the reference max and the row sum
-// are written as a split partial; the combine kernel merges splits and
-// applies B_v.
+// The key accumulator has one 256-column TMEM buffer (U takes the other half),
+// so while the epilogue reads a unit the MMA thread issues a pending r_v chunk
+// of the previous tile's absorption if its inputs are ready.  At the end of each
+// sequence segment U, the reference max and the row sum are written as a split
+// partial; the combine kernel merges splits and applies B_v.
 //
 // Warp roles (384 threads).  Every TMA or bulk-copy instruction costs its
 // issuing thread a long round trip, so loads are issued by three producer warps,
 // each putting several copies (one per lane) into one instruction:
-//   warp 0     latent pieces of C_g (ring A, all pieces of a group at once)
+//   warp 0     latent pieces of C_g (ring A)
 //   warp 10    value pieces of C_v (ring V, both halves of an r_v chunk at once)
-//   warp 11    factor pieces (ring W, up to kNW pieces at once)
-//   warp 1     TMEM owner and tcgen05.mma issuer (one elected lane)
+//   warp 11    factor items (ring W)
+//   warp 1     TMEM owner; its lane 0 alone runs the MMA schedule (on this GPU
+//              every barrier test, commit or fence costs a dependent round trip
+//              of 100-200 cycles, so the issuing path is kept to one thread and
+//              the fewest such operations per MMA)
 //   warps 2-9  epilogue: each TMEM lane quadrant (32 tokens) is served by two
 //              warps that split the 64 RoPE frequency pairs of a head and add
 //              their partial scores with shared-memory atomics.
@@ -52,7 +58,8 @@
 // Shared-memory operand layouts (128B swizzle unless noted):
 //   A slot  [128 tokens][w ranks] K-major, w in {64, 32, 16} with 128/64/32B
 //           swizzle: UMMA operand A of the reconstruction;
-//   W slot  [2 halves][w ranks][64 columns] MN-major: operand B;
+//   W slot  [nh heads][2 halves][w ranks][64 columns] MN-major: operand B
+//           (N = 128 nh, the 64-column atoms w * 128 bytes apart);
 //   V pair  two slots [128 tokens][64 rv] (r_v chunk halves), MN-major
 //           operand A of the value absorption;
 //   P       [2 token atoms][Hq_pad heads][64 tokens] bf16, K-major operand B.
@@ -77,15 +84,16 @@ namespace {
 using namespace sm100;
 
 constexpr int kD = 128;
-constexpr int kSlot = 16384;
-constexpr int kNW = 4;            // factor-piece ring depth
+constexpr int kSlot = 16384;     // latent and value slots
+constexpr int kSlotW = 32768;    // factor slots: up to 2 heads x 64 ranks x 128 columns
+constexpr int kNA = 4;            // latent-piece ring depth
 constexpr int kNV = 2;            // value ring depth (one r_v chunk: two halves)
 constexpr int kMaxGroupsTc = 16;
 constexpr int kMaxPieces = 5;
-constexpr int kMaxItems = kMaxKvHeads * kMaxPieces;
+constexpr int kMaxHqTc = 32;
+constexpr int kMaxItems = 256;
 constexpr int kThreads = 384;
 constexpr int kEpiThreads = 256;
-constexpr int kMaxHqTc = 32;
 constexpr float kRescaleThr = 8.f;  // log2 units: probabilities stay <= 256
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kUCol = 256;     // first TMEM column of the U accumulators
@@ -95,51 +103,44 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 template <bool kFold>
 struct Ring {
-  static constexpr int NA = kFold ? 5 : 4;  // latent-piece ring depth
-};
-
-struct Pieces {
-  int8_t n[kMaxGroupsTc];
-  int8_t w[kMaxGroupsTc][kMaxPieces];
-  int16_t k[kMaxGroupsTc][kMaxPieces];
+  static constexpr int NW = kFold ? 3 : 2;  // factor-item ring depth (key mode keeps 16 KB for queries)
 };
 
 struct Maps {
   CUtensorMap kc64, kc32, kc16, vc;
 };
 
-struct TcArgs {
-  int hq_pad;
-  int n_chunks;                  // rv / 128
-  int n_items;                   // factor pieces per tile (sum over groups of n_g * pieces_g)
-  int64_t fimg_seq_bytes;        // factor image bytes per sequence (query-folded mode)
-  const uint8_t* fimg;           // factor images (workspace)
-  Pieces pc;
-  int32_t item_off[kMaxItems];   // byte offset of factor piece n in the image
-  int8_t item_w[kMaxItems];      // ranks of factor piece n
-  int16_t order[kMaxKvHeads];    // KV head at each (group, slot) position, group-major
-  int8_t chunk_after[kMaxGroupsTc];  // r_v chunks of the previous tile absorbed after group g
-};
-
-// Per-group facts the hot loops need, kept in shared memory: indexing the
-// kernel-parameter tables at run time goes through the small constant cache,
-// which several warps thrash.
+// Per-group facts the hot loops need; copied to shared memory at kernel start
+// (indexing kernel-parameter tables at run time goes through the small constant
+// cache, which several warps would share).
 struct GroupSm {
   int32_t roff;          // first key-cache column of the group
-  int8_t np, ng;         // pieces per head, heads
-  int8_t chunk_after;    // r_v chunks of the previous tile absorbed after this group (cumulative)
-  int8_t pad;
+  int8_t np;             // latent pieces
+  int8_t h0, nh;         // MMA position of the group's first head, heads
+  int8_t nu;             // units (pairs of heads, the last one single when nh is odd)
   int8_t w[kMaxPieces];  // piece widths (ranks)
   int8_t pad2[3];
   int16_t k[kMaxPieces]; // first rank of each piece
+  int16_t pad3;
+};
+
+struct TcArgs {
+  int hq_pad;
+  int n_chunks;                  // rv / 128
+  int n_items;                   // factor items per tile
+  int64_t fimg_seq_bytes;        // factor image bytes per sequence (query-folded mode)
+  const uint8_t* fimg;           // factor images (workspace)
+  GroupSm grp[kMaxGroupsTc];
+  int16_t order[kMaxHqTc];       // KV head at each MMA position (group-major, slot order)
+  uint32_t item[kMaxItems];      // factor item n: byte offset | (bytes / 4096) << 26
 };
 
 template <bool kFold>
 struct Smem {
-  uint8_t a[Ring<kFold>::NA][kSlot];
-  uint8_t w[kNW][kSlot];
+  uint8_t a[kNA][kSlot];
+  uint8_t w[Ring<kFold>::NW][kSlotW];
   uint8_t v[kNV][kSlot];
-  uint8_t p[2][2 * kMaxHqTc * 128];
+  uint8_t p[2 * kMaxHqTc * 128];
   float x[kMaxHqTc * 128];                  // scores [head][token], accumulated atomically
   float qr[kFold ? 1 : kMaxHqTc * kD];      // key mode: rotated queries * log2(e)/sqrt(d)
   double om64[kD / 2];
@@ -147,13 +148,14 @@ struct Smem {
   float beta[kD / 2];
   float redm[4][kMaxHqTc];
   float redl[4][kMaxHqTc];
-  uint64_t a_full[Ring<kFold>::NA], a_empty[Ring<kFold>::NA];
-  uint64_t w_full[kNW], w_empty[kNW], v_full[kNV], v_empty[kNV];
-  uint64_t k_full[2], k_empty[2], p_full[2], p_empty[2], u_ready, u_free;
+  float mref[2][kMaxHqTc];  // reference max per head (log2 units), double-buffered by tile parity
+  uint64_t a_full[kNA], a_empty[kNA];
+  uint64_t w_full[Ring<kFold>::NW], w_empty[Ring<kFold>::NW], v_full[kNV], v_empty[kNV];
+  uint64_t k_full, k_empty, p_full, p_empty, u_ready, u_free;
   uint64_t epi_bar;
   GroupSm grp[kMaxGroupsTc];
-  int16_t order[kMaxKvHeads];
-  uint32_t item[kMaxItems];  // factor piece n: byte offset | (ranks / 16) << 28
+  int16_t order[kMaxHqTc];
+  uint32_t item[kMaxItems];
   uint32_t tmem_base;
   int abort_flag;
   int b_first, pre_first, nt_total;
@@ -170,10 +172,20 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
       : "memory");
 }
 
+// Moves [src, src + bytes) toward L2 ahead of its TMA loads (16-byte multiples).
+__device__ __forceinline__ void prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 // Bounded wait whose outcome is the same in every lane of the warp.
 __device__ __forceinline__ bool wwait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
   const bool r = mbar_wait(bar, parity, abort_flag);
   return __all_sync(0xffffffffu, r);
+}
+
+// Single non-blocking test, same outcome in every lane.
+__device__ __forceinline__ bool wtest(uint64_t* bar, uint32_t parity) {
+  return __all_sync(0xffffffffu, mbar_test(bar, parity));
 }
 
 // Lane 0 waits for the `n` ring slots starting at ring position `cnt` (depth
@@ -201,7 +213,7 @@ __device__ __forceinline__ int claim_slots(uint64_t* empty, int depth, int cnt, 
     n = 1;
     while (n < max_n) {
       const int c = cnt + n;
-      if (c >= depth && !mbar_try_wait(&empty[c % depth], ((c / depth) - 1) & 1)) break;
+      if (c >= depth && !mbar_test(&empty[c % depth], ((c / depth) - 1) & 1)) break;
       ++n;
     }
   }
@@ -252,50 +264,73 @@ __device__ __forceinline__ uint32_t p_off(int j, int t, int hq_pad) {
 }
 
 // ---------------------------------------------------------------------------
-// MMA helper (whole MMA warp; lane 0 issues): one r_v chunk of the value
-// absorption of tile `tt`, U[:, chunk c] += C_v[tile, chunk c]^T P
+// Value absorption bookkeeping of the MMA warp: chunks are issued in
+// (tile, chunk) order; `pt`, `pc` name the next one.
 // ---------------------------------------------------------------------------
 
+struct Absorb {
+  int pt, pc;      // next tile (CTA-local tile counter) and r_v chunk to absorb
+  int v_cnt;       // value ring position
+  int seg_first;   // first tile of the current segment
+  int sgc;         // segment counter
+  bool p_seen;     // P of tile pt (and, first tile of a segment, U free) already observed
+};
+
+// Issues chunk (ab.pt, ab.pc) from the single MMA thread.  Non-blocking mode
+// returns false without issuing when its inputs are not ready; blocking mode
+// waits (bounded).  `nvalid`: valid tokens of the tile (rows past it are zeroed).
 template <bool kFold>
-__device__ __forceinline__ bool mma_pv_chunk(Smem<kFold>& sm, uint32_t tmem, const TcArgs& ta, int tt, int c,
-                                             bool first_of_seg, int nvalid, int sgc, int& v_cnt, int lane,
-                                             volatile int* abort_flag) {
-  const int pb = tt & 1;
-  const int hq_pad = ta.hq_pad;
-  if (c == 0) {
-    if (!wwait(&sm.p_full[pb], (tt >> 1) & 1, abort_flag)) return false;
-    if (first_of_seg && sgc > 0 && !wwait(&sm.u_free, (sgc - 1) & 1, abort_flag)) return false;
+__device__ __forceinline__ bool absorb_chunk(Smem<kFold>& sm, uint32_t tmem, const TcArgs& ta, Absorb& ab,
+                                             int nvalid, bool blocking, volatile int* abort_flag, bool& ok) {
+  const int tt = ab.pt, c = ab.pc;
+  const bool first = tt == ab.seg_first;
+  const uint32_t vpar = (ab.v_cnt / kNV) & 1;
+  if (!ab.p_seen) {
+    if (blocking) {
+      if (!(ok = mbar_wait(&sm.p_full, tt & 1, abort_flag))) return false;
+      if (first && ab.sgc > 0 && !(ok = mbar_wait(&sm.u_free, (ab.sgc - 1) & 1, abort_flag))) return false;
+    } else {
+      if (!mbar_test(&sm.p_full, tt & 1)) return false;
+      if (first && ab.sgc > 0 && !mbar_test(&sm.u_free, (ab.sgc - 1) & 1)) return false;
+    }
+    ab.p_seen = true;
+    tc_fence_after();  // the epilogue's TMEM accesses of U precede the next absorption
   }
-  // the two halves of chunk c sit in ring slots 0 and 1 (kNV == 2)
-  if (!wwait(&sm.v_full[0], (v_cnt / kNV) & 1, abort_flag)) return false;
-  if (!wwait(&sm.v_full[1], (v_cnt / kNV) & 1, abort_flag)) return false;
+  if (blocking) {
+    if (!(ok = mbar_wait(&sm.v_full[0], vpar, abort_flag))) return false;
+    if (!(ok = mbar_wait(&sm.v_full[1], vpar, abort_flag))) return false;
+  } else if (!mbar_test(&sm.v_full[1], vpar) || !mbar_test(&sm.v_full[0], vpar)) {
+    return false;
+  }
   if (nvalid < 128) {  // rows past the sequence end: make them exact zeros
-    for (int r = nvalid + (lane >> 3); r < 128; r += 4) {
-      reinterpret_cast<uint4*>(sm.v[0] + r * 128)[lane & 7] = make_uint4(0, 0, 0, 0);
-      reinterpret_cast<uint4*>(sm.v[1] + r * 128)[lane & 7] = make_uint4(0, 0, 0, 0);
-    }
-    fence_proxy_async_smem();
-    __syncwarp();
-  }
-  tc_fence_after();
-  DCK_TC_TRACE(12);
-  if (lane == 0) {
-    const uint32_t idesc_v = idesc_bf16(128, hq_pad, true, false);
-    const uint32_t pbase = smem_u32(sm.p[pb]);
-    const uint32_t vb = smem_u32(sm.v[0]);
+    for (int r = nvalid; r < 128; ++r)
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      const uint64_t ad = sdesc(vb + k * 2048, kSlot, 1024, kSw128);
-      const uint64_t bd = sdesc(pbase + (k >> 2) * (hq_pad * 128) + (k & 3) * 32, 16, 1024, kSw128);
-      umma_f16(tmem + kUCol + c * hq_pad, ad, bd, idesc_v, (first_of_seg && k == 0) ? 0u : 1u);
-    }
-    umma_commit(&sm.v_empty[0]);
-    umma_commit(&sm.v_empty[1]);
-    if (c == ta.n_chunks - 1) umma_commit(&sm.p_empty[pb]);
+      for (int q = 0; q < 8; ++q) {
+        reinterpret_cast<uint4*>(sm.v[0] + r * 128)[q] = make_uint4(0, 0, 0, 0);
+        reinterpret_cast<uint4*>(sm.v[1] + r * 128)[q] = make_uint4(0, 0, 0, 0);
+      }
+    fence_proxy_async_smem();
   }
-  __syncwarp();
-  v_cnt += kNV;
-  DCK_TC_TRACE(13);
+  DCK_TC_TRACE(12);
+  const int hq_pad = ta.hq_pad;
+  const uint32_t idesc_v = idesc_bf16(128, hq_pad, true, false);
+  const uint32_t pbase = smem_u32(sm.p);
+  const uint32_t vb = smem_u32(sm.v[0]);
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const uint64_t ad = sdesc(vb + k * 2048, kSlot, 1024, kSw128);
+    const uint64_t bd = sdesc(pbase + (k >> 2) * (hq_pad * 128) + (k & 3) * 32, 16, 1024, kSw128);
+    umma_f16(tmem + kUCol + c * hq_pad, ad, bd, idesc_v, (first && k == 0) ? 0u : 1u);
+  }
+  umma_commit(&sm.v_empty[0]);
+  umma_commit(&sm.v_empty[1]);
+  if (c == ta.n_chunks - 1) umma_commit(&sm.p_empty);
+  ab.v_cnt += kNV;
+  if (++ab.pc == ta.n_chunks) {
+    ab.pc = 0;
+    ++ab.pt;
+    ab.p_seen = false;
+  }
   return true;
 }
 
@@ -306,7 +341,7 @@ __device__ __forceinline__ bool mma_pv_chunk(Smem<kFold>& sm, uint32_t tmem, con
 template <bool kFold>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tc_kernel(const __grid_constant__ Maps maps, const LayerTable lt, const DecodeArgs a, const TcArgs ta) {
-  constexpr int NA = Ring<kFold>::NA;
+  constexpr int NW = Ring<kFold>::NW;
   extern __shared__ uint8_t smem_raw[];
   Smem<kFold>& sm =
       *reinterpret_cast<Smem<kFold>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -317,11 +352,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // ---- setup -------------------------------------------------------------
   if (tid == 0) {
-    for (int i = 0; i < NA; ++i) {
+    for (int i = 0; i < kNA; ++i) {
       mbar_init(&sm.a_full[i], 1);
       mbar_init(&sm.a_empty[i], 1);
     }
-    for (int i = 0; i < kNW; ++i) {
+    for (int i = 0; i < NW; ++i) {
       mbar_init(&sm.w_full[i], 1);
       mbar_init(&sm.w_empty[i], 1);
     }
@@ -329,12 +364,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&sm.v_full[i], 1);
       mbar_init(&sm.v_empty[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&sm.k_full[i], 1);
-      mbar_init(&sm.k_empty[i], kEpiThreads / 32);
-      mbar_init(&sm.p_full[i], kEpiThreads / 32);
-      mbar_init(&sm.p_empty[i], 1);
-    }
+    mbar_init(&sm.k_full, 1);
+    mbar_init(&sm.k_empty, kEpiThreads / 32);
+    mbar_init(&sm.p_full, kEpiThreads / 32);
+    mbar_init(&sm.p_empty, 1);
     mbar_init(&sm.u_ready, 1);
     mbar_init(&sm.u_free, kEpiThreads / 32);
     mbar_init(&sm.epi_bar, kEpiThreads / 32);
@@ -345,24 +378,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(&sm.tmem_base, kTmemCols);
     tmem_relinquish();
   }
-  {  // P buffers start at zero (padded head rows stay zero); scores start at zero
-    uint4* pz = reinterpret_cast<uint4*>(&sm.p[0][0]);
+  {  // P starts at zero (padded head rows stay zero)
+    uint4* pz = reinterpret_cast<uint4*>(&sm.p[0]);
     for (int i = tid; i < (int)(sizeof(sm.p) / 16); i += kThreads) pz[i] = make_uint4(0, 0, 0, 0);
   }
-  if (tid < lt.G) {
-    GroupSm& gs = sm.grp[tid];
-    gs.roff = lt.grp_roff[tid];
-    gs.np = ta.pc.n[tid];
-    gs.ng = (int8_t)lt.grp_nh[tid];
-    gs.chunk_after = ta.chunk_after[tid];
-    for (int p = 0; p < kMaxPieces; ++p) {
-      gs.w[p] = ta.pc.w[tid][p];
-      gs.k[p] = ta.pc.k[tid][p];
-    }
-  }
+  if (tid < lt.G) sm.grp[tid] = ta.grp[tid];
   if (tid < lt.Hkv) sm.order[tid] = ta.order[tid];
-  for (int n = tid; n < ta.n_items; n += kThreads)
-    sm.item[n] = (uint32_t)ta.item_off[n] | ((uint32_t)(ta.item_w[n] / 16) << 28);
+  for (int n = tid; n < ta.n_items; n += kThreads) sm.item[n] = ta.item[n];
   if (tid < kD / 2) {
     const double om = exp2(-2.0 * tid / kD * log2((double)a.theta));
     sm.om64[tid] = om;
@@ -421,7 +443,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   DCK_TC_TRACE(0);
 
   if (warp == 0) {
-    // ---- latent pieces: all pieces of a group in one instruction -----------
+    // ---- latent pieces, issued as soon as their slots are free --------------
     if (x0 < x1) {
       const uint64_t pol = policy_evict_first();
       int a_cnt = 0;
@@ -429,15 +451,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       while (ok && walk.next(a, seg)) {
         for (int i = 0; i < seg.ntiles && ok; ++i) {
           const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
+          if (lane == 0 && i + 1 < seg.ntiles) {  // next tile's latent rows toward L2
+            const int64_t r0 = yrow + kTile, nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
+            if (nr > 0)
+              prefetch_l2(static_cast<const __nv_bfloat16*>(a.kc) + r0 * lt.Rk, (uint32_t)(nr * lt.Rk * 2));
+          }
           for (int g = 0; g < lt.G && ok; ++g) {
             const GroupSm& gs = sm.grp[g];
             const int np = gs.np;
             for (int p0 = 0; p0 < np && ok;) {
-              const int nb = claim_slots(sm.a_empty, NA, a_cnt, np - p0, lane, abort_flag);
+              const int nb = claim_slots(sm.a_empty, kNA, a_cnt, np - p0, lane, abort_flag);
               ok = nb > 0;
               if (!ok) break;
               if (lane < nb) {
-                const int sl = (a_cnt + lane) % NA;
+                const int sl = (a_cnt + lane) % kNA;
                 const int w = gs.w[p0 + lane];
                 const CUtensorMap* m = w == 64 ? &maps.kc64 : (w == 32 ? &maps.kc32 : &maps.kc16);
                 mbar_expect_tx(&sm.a_full[sl], kTile * w * 2);
@@ -461,6 +488,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       while (ok && walk.next(a, seg)) {
         for (int i = 0; i < seg.ntiles && ok; ++i) {
           const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
+          if (lane == 0) {  // this tile's value rows toward L2 (absorbed during the next tile)
+            const int64_t nr = a.n_rows - yrow < kTile ? a.n_rows - yrow : (int64_t)kTile;
+            if (nr > 0)
+              prefetch_l2(static_cast<const __nv_bfloat16*>(a.vc) + yrow * lt.rv, (uint32_t)(nr * lt.rv * 2));
+          }
           for (int c = 0; c < ta.n_chunks && ok; ++c) {
             if (!(ok = wait_slots(sm.v_empty, kNV, v_cnt, kNV, lane, abort_flag))) break;
             if (lane < kNV) {
@@ -475,7 +507,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else if (warp == 11) {
-    // ---- factor pieces: up to kNW 16 KB images per instruction -------------
+    // ---- factor items: several bulk copies per instruction ------------------
     if (x0 < x1) {
       const uint64_t pol = policy_evict_last();
       griddep_wait();  // the images are written by the preparation kernel
@@ -485,18 +517,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint8_t* img = ta.fimg + (kFold ? (int64_t)seg.b * ta.fimg_seq_bytes : 0);
         for (int i = 0; i < seg.ntiles && ok; ++i) {
           for (int n0 = 0; n0 < ta.n_items && ok;) {
-            const int nb = claim_slots(sm.w_empty, kNW, w_cnt, min(kNW, ta.n_items - n0), lane, abort_flag);
+            const int nb = claim_slots(sm.w_empty, NW, w_cnt, min(NW, ta.n_items - n0), lane, abort_flag);
             ok = nb > 0;
             if (!ok) break;
             if (lane < nb) {
-              const int sl = (w_cnt + lane) % kNW;
+              const int sl = (w_cnt + lane) % NW;
               const uint32_t it = sm.item[n0 + lane];
-              const uint32_t bytes = (it >> 28) << 12;
+              const uint32_t bytes = (it >> 26) << 12;
               mbar_expect_tx(&sm.w_full[sl], bytes);
-              bulk_load(sm.w[sl], img + (it & 0x0FFFFFFFu), bytes, &sm.w_full[sl], pol);
+              bulk_load(sm.w[sl], img + (it & 0x03FFFFFFu), bytes, &sm.w_full[sl], pol);
             }
             __syncwarp();
-            DCK_TC_TRACE(200 + nb);
+            DCK_TC_TRACE(100000 + w_cnt * 10 + nb);
             w_cnt += nb;
             n0 += nb;
           }
@@ -504,75 +536,88 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else if (warp == 1) {
-    // ---- MMA issuer (whole warp follows, lane 0 issues) ---------------------
-    if (x0 < x1) {
-      const uint32_t idesc_k = idesc_bf16(128, kD, false, true);
-      int a_cnt = 0, w_cnt = 0, v_cnt = 0, kh = 0, tl = 0, sgc = 0;
+    // ---- MMA issuer: one thread runs the whole schedule (warp-wide
+    // bookkeeping would only lengthen the path between MMAs) ----------------
+    if (lane == 0 && x0 < x1) {
+      int a_cnt = 0, w_cnt = 0, kc = 0, tl = 0;
+      Absorb ab{0, 0, 0, 0, 0, false};
       bool ok = true;
       while (ok && walk.next(a, seg)) {
-        const int tl_first = tl;
+        ab.seg_first = tl;
         for (int i = 0; i < seg.ntiles && ok; ++i) {
-          int c_next = 0;  // next r_v chunk of the previous tile to absorb
+          // the absorption of two tiles back must be complete before this tile's
+          // units: the epilogue's softmax step of the previous tile waits for it
+          while (ok && ab.pt < tl - 1) absorb_chunk<kFold>(sm, tmem, ta, ab, 128, true, abort_flag, ok);
           for (int g = 0; g < lt.G && ok; ++g) {
             const GroupSm& gs = sm.grp[g];
-            const int np = gs.np;
+            const int np = gs.np, nu = gs.nu;
             const int a_base = a_cnt;
-            const int ng = gs.ng;
-            for (int s = 0; s < ng && ok; ++s) {
-              const int buf = kh & 1;
-              if (kh >= 2 && !(ok = wwait(&sm.k_empty[buf], ((kh >> 1) - 1) & 1, abort_flag))) break;
-              DCK_TC_TRACE(10);
-              for (int p = 0; p < np && ok; ++p) {
-                const int asl = (a_base + p) % NA;
-                if (s == 0 && !(ok = wwait(&sm.a_full[asl], ((a_base + p) / NA) & 1, abort_flag))) break;
-                DCK_TC_TRACE(15);
-                const int wsl = w_cnt % kNW;
-                if (!(ok = wwait(&sm.w_full[wsl], (w_cnt / kNW) & 1, abort_flag))) break;
-                DCK_TC_TRACE(14);
+            for (int u = 0; u < nu && ok; ++u) {
+              const int nh = min(2, gs.nh - 2 * u);
+              const uint32_t idesc_k = idesc_bf16(128, kD * nh, false, true);
+              // one key buffer: the epilogue has read the previous unit
+              if (kc >= 1) {
+                if (!(ok = mbar_wait(&sm.k_empty, (kc - 1) & 1, abort_flag))) break;
                 tc_fence_after();
-                if (lane == 0) {
-                  DCK_TC_TRACE(17);
-                  const int w = gs.w[p];
-                  const uint32_t ab = smem_u32(sm.a[asl]);
-                  const uint32_t bb = smem_u32(sm.w[wsl]);
-                  const uint32_t swz = swz_of(w);
-                  for (int k = 0; k < w / 16; ++k) {
-                    const uint64_t ad = sdesc(ab + k * 32, 16, 16 * w, swz);
-                    const uint64_t bd = sdesc(bb + k * 2048, 128 * w, 1024, kSw128);
-                    umma_f16(tmem + buf * kD, ad, bd, idesc_k, (p > 0 || k > 0) ? 1u : 0u);
-                  }
-                  DCK_TC_TRACE(18);
-                  umma_commit(&sm.w_empty[wsl]);
-                  if (s == ng - 1) umma_commit(&sm.a_empty[asl]);  // last head: piece done
-                  DCK_TC_TRACE(16);
+              }
+              DCK_TC_TRACE(10);
+              // readiness of this unit's factor items (and, first unit of the group,
+              // latent pieces): independent tests whose latencies overlap; blocking
+              // waits, in ring order, only for what is not there yet.  Only items
+              // within one turn of the ring are tested: the previous use of their
+              // slot has been consumed, so the parity test cannot see a stale phase
+              // (an item a full turn ahead shares its slot with one still in flight).
+              uint32_t miss = 0;
+#pragma unroll
+              for (int p = 0; p < kMaxPieces; ++p)
+                if (p < np) {
+                  const int c = w_cnt + p;
+                  if (p >= NW || !mbar_test(&sm.w_full[c % NW], (c / NW) & 1)) miss |= 1u << p;
+                  if (u == 0 && !mbar_test(&sm.a_full[(a_base + p) % kNA], ((a_base + p) / kNA) & 1))
+                    miss |= 0x100u << p;
                 }
-                __syncwarp();
+              for (int p = 0; p < np; ++p) {
+                const int asl = (a_base + p) % kNA;
+                const int wsl = w_cnt % NW;
+                // an item not ready at the test is waited for here, in ring order (the
+                // factor ring may be shallower than a unit's item count)
+                if (((miss >> (8 + p)) & 1) && !(ok = mbar_wait(&sm.a_full[asl], ((a_base + p) / kNA) & 1, abort_flag)))
+                  break;
+                if (((miss >> p) & 1) && !(ok = mbar_wait(&sm.w_full[wsl], (w_cnt / NW) & 1, abort_flag))) break;
+                const int w = gs.w[p];
+                const uint32_t ab0 = smem_u32(sm.a[asl]);
+                const uint32_t bb = smem_u32(sm.w[wsl]);
+                const uint32_t swz = swz_of(w);
+                for (int k = 0; k < w / 16; ++k) {
+                  const uint64_t ad = sdesc(ab0 + k * 32, 16, 16 * w, swz);
+                  const uint64_t bd = sdesc(bb + k * 2048, 128 * w, 1024, kSw128);
+                  umma_f16(tmem, ad, bd, idesc_k, (p > 0 || k > 0) ? 1u : 0u);
+                }
+                umma_commit(&sm.w_empty[wsl]);
+                if (u == nu - 1) umma_commit(&sm.a_empty[asl]);  // last unit of the group: piece done
                 ++w_cnt;
               }
-              if (ok && lane == 0) umma_commit(&sm.k_full[buf]);
-              __syncwarp();
+              if (!ok) break;
+              umma_commit(&sm.k_full);
               DCK_TC_TRACE(11);
-              ++kh;
+              ++kc;
+              // while the epilogue drains the unit: one pending absorption chunk, if ready
+              if (ab.pt < tl) absorb_chunk<kFold>(sm, tmem, ta, ab, 128, false, abort_flag, ok);
             }
             a_cnt += np;
-            if (i > 0)  // absorb the previous tile's chunks scheduled after this group
-              for (; ok && c_next < gs.chunk_after; ++c_next)
-                ok = mma_pv_chunk<kFold>(sm, tmem, ta, tl - 1, c_next, tl - 1 == tl_first, 128, sgc, v_cnt, lane,
-                                          abort_flag);
           }
           ++tl;
         }
-        if (ok) {
-          const int nvalid = seg.t_end - (seg.t_begin + kTile * (seg.ntiles - 1));
-          for (int c = 0; ok && c < ta.n_chunks; ++c)
-            ok = mma_pv_chunk<kFold>(sm, tmem, ta, tl - 1, c, tl - 1 == tl_first, nvalid, sgc, v_cnt, lane,
-                                      abort_flag);
+        // segment end: the rest of the absorption, the last tile with its valid rows
+        while (ok && ab.pt < tl) {
+          const int nvalid = ab.pt == tl - 1 ? seg.t_end - (seg.t_begin + kTile * (seg.ntiles - 1)) : 128;
+          absorb_chunk<kFold>(sm, tmem, ta, ab, nvalid, true, abort_flag, ok);
         }
-        if (ok && lane == 0) umma_commit(&sm.u_ready);
-        __syncwarp();
-        ++sgc;
+        if (ok) umma_commit(&sm.u_ready);
+        ++ab.sgc;
       }
     }
+    __syncwarp();
   } else if (warp >= 2 && warp <= 9) {
     // ---- epilogue: RoPE, scores, softmax, P, U readout ----------------------
     const int e = tid - 64;              // 0 .. 255
@@ -580,9 +625,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int hf = (warp - 2) >> 2;      // frequency half, then head half
     const int tau = quad * 32 + lane;    // token row inside the tile
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
-    int kh = 0, tl = 0, sgc = 0, round = 0;
+    int kc = 0, tl = 0, sgc = 0, round = 0;
     bool ok = true;
-    float m_ref[16];  // reference max of heads 16 hf + u (log2 units)
     const int jb0 = 16 * hf;  // heads owned at tile and segment ends
 #define EPI_SYNC()                                  \
   do {                                              \
@@ -606,8 +650,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           sm.qr[j * kD + pi + kD / 2] = (float)(x1v * sn + x2v * cs) * qscale;
         }
       }
-#pragma unroll
-      for (int u = 0; u < 16; ++u) m_ref[u] = -INFINITY;
+      // reference maxima start at -inf: the buffer a tile end reads is that of tile tl - 1
+      if (quad == 0 && lane < 16 && jb0 + lane < Hq) sm.mref[(tl - 1) & 1][jb0 + lane] = -INFINITY;
       // RoPE angle of token t0+tau and pair p: (t0*w_p mod 2pi, fp64) + tau*w_p (fp32);
       // the offsets beta of later tiles are written at the previous tile's end
       if (e < kD / 2) {
@@ -617,7 +661,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       EPI_SYNC();
       if (!ok) break;
       // running row sums: one per (quadrant, head), kept by the warp owning both
-      if (lane < 16 && 16 * hf + lane < Hq) sm.redl[quad][16 * hf + lane] = 0.f;
+      if (lane < 16 && jb0 + lane < Hq) sm.redl[quad][jb0 + lane] = 0.f;
       const int tl_first = tl;
       for (int i = 0; i < seg.ntiles && ok; ++i) {
         const int t0 = seg.t_begin + kTile * i;
@@ -630,62 +674,72 @@ __global__ void __launch_bounds__(kThreads, 1)
           ph = fmaf(-kTwoPi, rintf(ph * kInvTwoPi), ph);
           __sincosf(ph, &sn[ip], &cs[ip]);
         }
-        // per KV head, in MMA order: partial scores of this frequency half
-        for (int hi = 0; hi < lt.Hkv; ++hi) {
-          const int buf = kh & 1;
-          if (!(ok = wwait(&sm.k_full[buf], (kh >> 1) & 1, abort_flag))) break;
-          tc_fence_after();
-          DCK_TC_TRACE(20);
-          const int j0 = sm.order[hi] * qpg;
-          if (kFold) {
-            // Y columns [64 hf, 64 hf + 64): pairs (2i, 2i+1) of my 32 frequencies
-            float y0[32], y1[32];
-            tmem_ld32(tmem + lane_base + buf * kD + 64 * hf, y0);
-            tmem_ld32(tmem + lane_base + buf * kD + 64 * hf + 32, y1);
-            tmem_wait_ld();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
-            float part0 = 0.f, part1 = 0.f;
+        // per unit (one or two KV heads), in MMA order: partial scores of this frequency half
+        for (int g = 0; g < lt.G && ok; ++g) {
+          const GroupSm& gs = sm.grp[g];
+          for (int u = 0; u < gs.nu; ++u) {
+            const int nh = min(2, gs.nh - 2 * u);
+            if (!(ok = wwait(&sm.k_full, kc & 1, abort_flag))) break;
+            tc_fence_after();
+            DCK_TC_TRACE(20);
+            for (int hh = 0; hh < nh; ++hh) {
+              const int j0 = sm.order[gs.h0 + 2 * u + hh] * qpg;
+              const uint32_t cb = tmem + lane_base + hh * kD;
+              const bool last = hh == nh - 1;
+              if (kFold) {
+                // Y columns [64 hf, 64 hf + 64): pairs (2i, 2i+1) of my 32 frequencies,
+                // read in two passes of 16 pairs to keep the register footprint small
+                float pa[4] = {0.f, 0.f, 0.f, 0.f};  // independent chains
 #pragma unroll
-            for (int i2 = 0; i2 < 16; ++i2) {
-              part0 = fmaf(cs[i2], y0[2 * i2], fmaf(sn[i2], y0[2 * i2 + 1], part0));
-              part1 = fmaf(cs[16 + i2], y1[2 * i2], fmaf(sn[16 + i2], y1[2 * i2 + 1], part1));
-            }
-            atomicAdd(&sm.x[j0 * 128 + tau], part0 + part1);
-          } else {
-            // two passes of 16 frequency pairs keep the register footprint small
-            float part[kMaxQPerKv];
+                for (int ps = 0; ps < 2; ++ps) {
+                  float y[32];
+                  tmem_ld32(cb + 64 * hf + 32 * ps, y);
+                  tmem_wait_ld();
+                  if (last && ps == 1) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sm.k_empty);
+                  }
 #pragma unroll
-            for (int jj = 0; jj < kMaxQPerKv; ++jj) part[jj] = 0.f;
+                  for (int i2 = 0; i2 < 16; ++i2)
+                    pa[i2 & 3] = fmaf(cs[16 * ps + i2], y[2 * i2], fmaf(sn[16 * ps + i2], y[2 * i2 + 1], pa[i2 & 3]));
+                }
+                atomicAdd(&sm.x[j0 * 128 + tau], (pa[0] + pa[1]) + (pa[2] + pa[3]));
+              } else {
+                // two passes of 16 frequency pairs keep the register footprint small
+                float part[kMaxQPerKv];
 #pragma unroll
-            for (int ps = 0; ps < 2; ++ps) {
-              float k1v[16], k2v[16];
-              tmem_ld16(tmem + lane_base + buf * kD + 32 * hf + 16 * ps, k1v);
-              tmem_ld16(tmem + lane_base + buf * kD + 64 + 32 * hf + 16 * ps, k2v);
-              tmem_wait_ld();
-              if (ps == 1) {
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
-              }
+                for (int jj = 0; jj < kMaxQPerKv; ++jj) part[jj] = 0.f;
 #pragma unroll
-              for (int i2 = 0; i2 < 16; ++i2) {
-                const int ip = 16 * ps + i2;
-                const float r1 = fmaf(k1v[i2], cs[ip], -k2v[i2] * sn[ip]);
-                const float r2 = fmaf(k1v[i2], sn[ip], k2v[i2] * cs[ip]);
-                const float* qrow = sm.qr + j0 * kD + 32 * hf + ip;
+                for (int ps = 0; ps < 2; ++ps) {
+                  float k1v[16], k2v[16];
+                  tmem_ld16(cb + 32 * hf + 16 * ps, k1v);
+                  tmem_ld16(cb + 64 + 32 * hf + 16 * ps, k2v);
+                  tmem_wait_ld();
+                  if (last && ps == 1) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sm.k_empty);
+                  }
+#pragma unroll
+                  for (int i2 = 0; i2 < 16; ++i2) {
+                    const int ip = 16 * ps + i2;
+                    const float r1 = fmaf(k1v[i2], cs[ip], -k2v[i2] * sn[ip]);
+                    const float r2 = fmaf(k1v[i2], sn[ip], k2v[i2] * cs[ip]);
+                    const float* qrow = sm.qr + j0 * kD + 32 * hf + ip;
+#pragma unroll
+                    for (int jj = 0; jj < kMaxQPerKv; ++jj)
+                      if (jj < qpg) part[jj] = fmaf(qrow[jj * kD], r1, fmaf(qrow[jj * kD + 64], r2, part[jj]));
+                  }
+                }
 #pragma unroll
                 for (int jj = 0; jj < kMaxQPerKv; ++jj)
-                  if (jj < qpg) part[jj] = fmaf(qrow[jj * kD], r1, fmaf(qrow[jj * kD + 64], r2, part[jj]));
+                  if (jj < qpg) atomicAdd(&sm.x[(j0 + jj) * 128 + tau], part[jj]);
               }
             }
-#pragma unroll
-            for (int jj = 0; jj < kMaxQPerKv; ++jj)
-              if (jj < qpg) atomicAdd(&sm.x[(j0 + jj) * 128 + tau], part[jj]);
+            DCK_TC_TRACE(21);
+            ++kc;
           }
-          DCK_TC_TRACE(21);
-          ++kh;
         }
         if (!ok) break;
         // ---- tile end: reference max, optional rescale of U, P -------------
@@ -722,29 +776,37 @@ __global__ void __launch_bounds__(kThreads, 1)
         EPI_SYNC();  // per-quadrant maxima are in redm
         DCK_TC_TRACE(28);
         if (!ok) break;
-        float al[16];
+        float al[16], mr[16];  // rescale factors, reference maxima after this tile
         bool resc = false;
         {
           float tm[16];
 #pragma unroll
-          for (int u = 0; u < 16; ++u)
+          for (int u = 0; u < 16; ++u) {
             tm[u] = u < nh ? fmaxf(fmaxf(sm.redm[0][jb + u], sm.redm[1][jb + u]),
                                    fmaxf(sm.redm[2][jb + u], sm.redm[3][jb + u]))
                            : -INFINITY;
+            mr[u] = u < nh ? sm.mref[(tl - 1) & 1][jb + u] : 0.f;
+          }
 #pragma unroll
           for (int u = 0; u < 16; ++u) {
             al[u] = 1.f;
-            if (u < nh && (m_ref[u] == -INFINITY || tm[u] > m_ref[u] + kRescaleThr)) {
-              al[u] = exp2f(m_ref[u] - tm[u]);
-              m_ref[u] = tm[u];
+            if (u < nh && (mr[u] == -INFINITY || tm[u] > mr[u] + kRescaleThr)) {
+              al[u] = exp2f(mr[u] - tm[u]);
+              mr[u] = tm[u];
               resc = true;
             }
           }
+          float v = mr[0];
+#pragma unroll
+          for (int u = 1; u < 16; ++u) v = lane == u ? mr[u] : v;
+          if (quad == 0 && lane < nh) sm.mref[tl & 1][jb + lane] = v;
         }
+        // the previous tile's absorption must be complete before U is rescaled
+        // or P is overwritten
+        if (tl >= 1 && !(ok = wwait(&sm.p_empty, (tl - 1) & 1, abort_flag))) break;
+        DCK_TC_TRACE(30);
         if (resc && tl != tl_first) {
-          // rescale this warp's heads of U; the previous tile's absorption must be complete
-          const int tp = tl - 1;
-          if (!(ok = wwait(&sm.p_empty[tp & 1], (tp >> 1) & 1, abort_flag))) break;
+          // rescale this warp's heads of U
           tc_fence_after();
           for (int c = 0; c < ta.n_chunks; ++c) {
             float v[16];
@@ -759,14 +821,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_before();
         }
         // probabilities -> P (bf16); row sums use the rounded values
-        const int pb = tl & 1;
-        if (tl >= 2 && !(ok = wwait(&sm.p_empty[pb], ((tl - 2) >> 1) & 1, abort_flag))) break;
-        DCK_TC_TRACE(30);
-        uint8_t* pbuf = sm.p[pb];
+        uint8_t* pbuf = sm.p;
         float ps[16];
 #pragma unroll
         for (int u = 0; u < 16; ++u) {
-          const __nv_bfloat16 pv = __float2bfloat16_rn(exp2f(sc[u] - m_ref[u]));
+          const __nv_bfloat16 pv = __float2bfloat16_rn(exp2f(sc[u] - mr[u]));
           if (u < nh) *reinterpret_cast<__nv_bfloat16*>(pbuf + p_off(jb + u, tau, hq_pad)) = pv;
           ps[u] = u < nh ? __bfloat162float(pv) : 0.f;
         }
@@ -785,7 +844,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.p_full[pb]);
+        if (lane == 0) mbar_arrive(&sm.p_full);
         DCK_TC_TRACE(23);
         ++tl;
       }
@@ -810,12 +869,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       EPI_SYNC();
       if (!ok) break;
       if (quad == 0) {
-        float m = m_ref[0];
-#pragma unroll
-        for (int u = 1; u < 16; ++u) m = lane == u ? m_ref[u] : m;
         const int j = jb0 + lane;
         if (lane < 16 && j < Hq) {
-          a.part_ml[(slot * Hq + j) * 2] = m;
+          a.part_ml[(slot * Hq + j) * 2] = sm.mref[(tl - 1) & 1][j];
           a.part_ml[(slot * Hq + j) * 2 + 1] = sm.redl[0][j] + sm.redl[1][j] + sm.redl[2][j] + sm.redl[3][j];
         }
       }
@@ -846,21 +902,24 @@ __global__ void __launch_bounds__(kThreads, 1)
 // factor images
 // ---------------------------------------------------------------------------
 
-struct PrepArgs {
-  int n_items;
-  int16_t item_g[kMaxItems];   // group of factor piece n
-  int16_t item_s[kMaxItems];   // head slot of piece n in its group
-  int16_t item_k[kMaxItems];   // first rank of piece n
-  int8_t item_w[kMaxItems];    // ranks of piece n
-  int32_t item_off[kMaxItems];  // byte offset of piece n in a sequence's image
-  int64_t seq_bytes;
+struct PrepItem {
+  int8_t g, s0, nh, ws;  // group, first head slot, heads, ranks
+  int16_t k0;            // first rank
+  int16_t pad;
+  int32_t off;           // byte offset in a sequence's image
 };
 
-// One block writes one piece image of w * 256 bytes: [2 halves][w rank rows]
+struct PrepArgs {
+  int n_items;
+  int64_t seq_bytes;
+  PrepItem item[kMaxItems];
+};
+
+// One block writes one factor item: [nh heads][2 halves][ws rank rows]
 // [64 columns] bf16, 128B-swizzled (16-byte chunk c of row r stored at chunk
-// c ^ (r % 8); w * 128 is a multiple of the 1024-byte swizzle atom).
-// Key mode: columns of B_g[:, slot].
-// Query-folded mode (one block row per sequence b): columns 2i and 2i+1 are
+// c ^ (r % 8); every half starts on a 1024-byte swizzle atom).
+// Key mode: columns of B_g[:, slot].  Query-folded mode (one block row per
+// sequence b): columns 2i and 2i+1 are
 //   a_i B[:, i] + b_i B[:, i+64]  and  b_i B[:, i] - a_i B[:, i+64]
 // with (a, b) the halves of RoPE(q_{b,h}, L_b - 1) * log2(e)/sqrt(d).
 template <bool kFold>
@@ -868,59 +927,59 @@ __global__ void __launch_bounds__(256) factor_prep_kernel(const LayerTable lt, c
                                                           uint8_t* __restrict__ img) {
   griddep_launch();
   const int n = blockIdx.x, b = blockIdx.y;
-  const int g = pa.item_g[n], s = pa.item_s[n], k0 = pa.item_k[n], wr = pa.item_w[n];
-  __shared__ float qa[kD / 2], qb[kD / 2];
+  const PrepItem it = pa.item[n];
+  const int g = it.g, ws = it.ws, nh = it.nh;
+  __shared__ float qa[2][kD / 2], qb[2][kD / 2];
   if (kFold) {
-    int kv = 0;
-    for (int hh = 0; hh < lt.Hkv; ++hh)
-      if (lt.head_group[hh] == g && lt.head_slot[hh] == s) kv = hh;
     const int L = valid_len(a.seq_len, a.seq_start, b, a.n_rows);
     if (L == 0) return;  // no tile of this sequence is ever processed
-    if (threadIdx.x < kD / 2) {
-      const int i = threadIdx.x;
+    if (threadIdx.x < nh * (kD / 2)) {
+      const int hh = threadIdx.x / (kD / 2), i = threadIdx.x % (kD / 2);
+      int kv = 0;
+      for (int h = 0; h < lt.Hkv; ++h)
+        if (lt.head_group[h] == g && lt.head_slot[h] == it.s0 + hh) kv = h;
       const double om = exp2(-2.0 * i / kD * log2((double)a.theta));
       double sn, cs;
       sincos((double)(L - 1) * om, &sn, &cs);
       const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(a.q) + ((int64_t)b * lt.Hq + kv) * kD;
       const double x1 = __bfloat162float(q[i]), x2 = __bfloat162float(q[i + kD / 2]);
       const float sc = kLog2e * rsqrtf((float)kD);
-      qa[i] = (float)(x1 * cs - x2 * sn) * sc;
-      qb[i] = (float)(x1 * sn + x2 * cs) * sc;
+      qa[hh][i] = (float)(x1 * cs - x2 * sn) * sc;
+      qb[hh][i] = (float)(x1 * sn + x2 * cs) * sc;
     }
     __syncthreads();
   }
   const int64_t ld = (int64_t)lt.grp_nh[g] * kD;
-  const __nv_bfloat16* __restrict__ Bs = static_cast<const __nv_bfloat16*>(a.Bk) + lt.grp_boff[g] + s * kD;
-  uint8_t* dst = img + (kFold ? (int64_t)b * pa.seq_bytes : 0) + pa.item_off[n];
-  // thread -> (row, 8-column chunk): w rows x 16 chunks (2 halves x 8)
-  for (int idx = threadIdx.x; idx < wr * 16; idx += blockDim.x) {
-    const int r = idx >> 4, ch = idx & 15;
+  uint8_t* dst = img + (kFold ? (int64_t)b * pa.seq_bytes : 0) + it.off;
+  // thread -> (head, row, 8-column chunk): nh x ws rows x 16 chunks (2 halves x 8)
+  for (int idx = threadIdx.x; idx < nh * ws * 16; idx += blockDim.x) {
+    const int hh = idx / (ws * 16), r = (idx >> 4) % ws, ch = idx & 15;
     const int half = ch >> 3, c8 = ch & 7;
+    const __nv_bfloat16* __restrict__ Bs =
+        static_cast<const __nv_bfloat16*>(a.Bk) + lt.grp_boff[g] + (it.s0 + hh) * kD;
+    const int k = it.k0 + r;
     float v[8];
-    {
-      const int k = k0 + r;
-      if (kFold) {
-        // output columns col = 64*half + 8*c8 + t, t even/odd -> pair i = col/2
+    if (kFold) {
+      // output columns col = 64*half + 8*c8 + t, t even/odd -> pair i = col/2
 #pragma unroll
-        for (int t = 0; t < 8; t += 2) {
-          const int i = (64 * half + 8 * c8 + t) >> 1;
-          const float x = __bfloat162float(Bs[k * ld + i]);
-          const float y = __bfloat162float(Bs[k * ld + kD / 2 + i]);
-          v[t] = fmaf(qa[i], x, qb[i] * y);
-          v[t + 1] = fmaf(qb[i], x, -qa[i] * y);
-        }
-      } else {
-        const uint4 raw = *reinterpret_cast<const uint4*>(Bs + k * ld + 64 * half + 8 * c8);
-        const __nv_bfloat16* h8 = reinterpret_cast<const __nv_bfloat16*>(&raw);
-#pragma unroll
-        for (int t = 0; t < 8; ++t) v[t] = __bfloat162float(h8[t]);
+      for (int t = 0; t < 8; t += 2) {
+        const int i = (64 * half + 8 * c8 + t) >> 1;
+        const float x = __bfloat162float(Bs[k * ld + i]);
+        const float y = __bfloat162float(Bs[k * ld + kD / 2 + i]);
+        v[t] = fmaf(qa[hh][i], x, qb[hh][i] * y);
+        v[t + 1] = fmaf(qb[hh][i], x, -qa[hh][i] * y);
       }
+    } else {
+      const uint4 raw = *reinterpret_cast<const uint4*>(Bs + k * ld + 64 * half + 8 * c8);
+      const __nv_bfloat16* h8 = reinterpret_cast<const __nv_bfloat16*>(&raw);
+#pragma unroll
+      for (int t = 0; t < 8; ++t) v[t] = __bfloat162float(h8[t]);
     }
     uint4 out;
     __nv_bfloat162* o2 = reinterpret_cast<__nv_bfloat162*>(&out);
 #pragma unroll
     for (int t = 0; t < 4; ++t) o2[t] = __floats2bfloat162_rn(v[2 * t], v[2 * t + 1]);
-    *reinterpret_cast<uint4*>(dst + half * (wr * 128) + r * 128 + ((c8 ^ (r & 7)) << 4)) = out;
+    *reinterpret_cast<uint4*>(dst + (hh * 2 + half) * (ws * 128) + r * 128 + ((c8 ^ (r & 7)) << 4)) = out;
   }
 }
 
@@ -939,16 +998,6 @@ int make_pieces(int r, int8_t* w, int16_t* k) {
 }
 
 int hq_pad_of(int Hq) { return std::max(16, (Hq + 15) / 16 * 16); }
-
-int n_items_of(const LayerTable& lt) {
-  int n = 0;
-  for (int g = 0; g < lt.G; ++g) {
-    int8_t w[kMaxPieces];
-    int16_t k[kMaxPieces];
-    n += lt.grp_nh[g] * make_pieces(lt.grp_rank[g], w, k);
-  }
-  return n;
-}
 
 // Bytes of one copy of all factor images: sum over heads of r_g * 128 columns * 2.
 size_t image_bytes_of(const LayerTable& lt) {
@@ -1018,23 +1067,69 @@ cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& m
   return e;
 }
 
+// Units, items and per-group tables of a layer.  Returns false when the layer
+// does not fit the tables.
+bool build_tables(const LayerTable& lt, TcArgs& ta, PrepArgs& pa) {
+  std::memset(&ta, 0, sizeof(ta));
+  std::memset(&pa, 0, sizeof(pa));
+  ta.hq_pad = hq_pad_of(lt.Hq);
+  ta.n_chunks = lt.rv / 128;
+  int pos = 0, item = 0, off = 0;
+  for (int g = 0; g < lt.G; ++g) {
+    GroupSm& gs = ta.grp[g];
+    gs.roff = lt.grp_roff[g];
+    int16_t kk[kMaxPieces];
+    gs.np = (int8_t)make_pieces(lt.grp_rank[g], gs.w, kk);
+    if (gs.np > kMaxPieces || gs.np > kNA) return false;
+    for (int p = 0; p < gs.np; ++p) gs.k[p] = kk[p];
+    gs.h0 = (int8_t)pos;
+    gs.nh = (int8_t)lt.grp_nh[g];
+    gs.nu = (int8_t)((lt.grp_nh[g] + 1) / 2);
+    for (int sl = 0; sl < lt.grp_nh[g]; ++sl)
+      for (int h = 0; h < lt.Hkv; ++h)
+        if (lt.head_group[h] == g && lt.head_slot[h] == sl) {
+          if (pos >= kMaxHqTc) return false;
+          ta.order[pos++] = (int16_t)h;
+        }
+    for (int s0 = 0; s0 < lt.grp_nh[g]; s0 += 2) {
+      const int nh = std::min(2, lt.grp_nh[g] - s0);
+      for (int p = 0; p < gs.np; ++p) {
+        if (item >= kMaxItems) return false;
+        const int w = gs.w[p], bytes = nh * w * 256;
+        PrepItem& pi = pa.item[item];
+        pi.g = (int8_t)g;
+        pi.s0 = (int8_t)s0;
+        pi.nh = (int8_t)nh;
+        pi.ws = (int8_t)w;
+        pi.k0 = gs.k[p];
+        pi.off = off;
+        ta.item[item] = (uint32_t)off | ((uint32_t)(bytes >> 12) << 26);
+        off += bytes;
+        ++item;
+      }
+    }
+  }
+  ta.n_items = item;
+  pa.n_items = item;
+  pa.seq_bytes = off;
+  ta.fimg_seq_bytes = off;
+  return true;
+}
+
 }  // namespace
 
 bool tc_decode_supports(const LayerTable& lt, int dtype) {
   if (dtype != DCK_BF16 || lt.d != kD) return false;
   if (lt.Hq > kMaxHqTc || lt.qpg > kMaxQPerKv || lt.G > kMaxGroupsTc) return false;
   if (lt.rv % 128 || (lt.rv / 128) * hq_pad_of(lt.Hq) > 256) return false;
-  for (int g = 0; g < lt.G; ++g) {
-    int8_t w[kMaxPieces];
-    int16_t k[kMaxPieces];
-    const int np = make_pieces(lt.grp_rank[g], w, k);
-    if (lt.grp_rank[g] > 256 || np > kMaxPieces || np > (lt.qpg == 1 ? Ring<true>::NA : Ring<false>::NA))
-      return false;
-  }
-  return n_items_of(lt) <= kMaxItems;
+  for (int g = 0; g < lt.G; ++g)
+    if (lt.grp_rank[g] > 256 || lt.grp_rank[g] % 16) return false;
+  static thread_local TcArgs ta;
+  static thread_local PrepArgs pa;
+  return build_tables(lt, ta, pa);
 }
 
-// Extra workspace of the tensor-core path: the factor piece images.
+// Extra workspace of the tensor-core path: the factor images.
 size_t tc_decode_extra_ws(const LayerTable& lt, int batch) {
   if (!tc_decode_supports(lt, DCK_BF16)) return 0;
   const size_t per = image_bytes_of(lt);
@@ -1046,36 +1141,9 @@ int tc_decode_launches(const LayerTable&) { return 2; }
 cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) {
   const bool fold = lt.qpg == 1;
   if (!a.extra) return cudaErrorInvalidValue;
-  TcArgs ta;
-  std::memset(&ta, 0, sizeof(ta));
-  PrepArgs pa;
-  std::memset(&pa, 0, sizeof(pa));
-  ta.hq_pad = hq_pad_of(lt.Hq);
-  ta.n_chunks = lt.rv / 128;
-  int pos = 0, item = 0, off = 0;
-  for (int g = 0; g < lt.G; ++g) {
-    ta.pc.n[g] = (int8_t)make_pieces(lt.grp_rank[g], ta.pc.w[g], ta.pc.k[g]);
-    for (int sl = 0; sl < lt.grp_nh[g]; ++sl) {
-      for (int h = 0; h < lt.Hkv; ++h)
-        if (lt.head_group[h] == g && lt.head_slot[h] == sl) ta.order[pos++] = (int16_t)h;
-      for (int p = 0; p < ta.pc.n[g]; ++p, ++item) {
-        pa.item_g[item] = (int16_t)g;
-        pa.item_s[item] = (int16_t)sl;
-        pa.item_k[item] = ta.pc.k[g][p];
-        pa.item_w[item] = ta.pc.w[g][p];
-        pa.item_off[item] = off;
-        ta.item_w[item] = ta.pc.w[g][p];
-        ta.item_off[item] = off;
-        off += ta.pc.w[g][p] * 256;
-      }
-    }
-    // r_v chunks of the previous tile absorbed after group g (cumulative count)
-    ta.chunk_after[g] = (int8_t)(((int64_t)(g + 1) * ta.n_chunks) / lt.G);
-  }
-  ta.n_items = item;
-  pa.n_items = item;
-  pa.seq_bytes = off;
-  ta.fimg_seq_bytes = pa.seq_bytes;
+  static thread_local TcArgs ta;
+  static thread_local PrepArgs pa;
+  if (!build_tables(lt, ta, pa)) return cudaErrorInvalidValue;
   ta.fimg = static_cast<const uint8_t*>(a.extra);
   const MapsKey key{a.kc, a.vc, a.n_rows, lt.Rk, lt.rv};
   Maps maps;
