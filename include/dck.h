@@ -129,13 +129,19 @@ dck_status dck_latent_append(const dck_layer_desc* desc, const void* x, int32_t 
  *               zero output row.
  *   rope_theta  RoPE base theta > 0
  *   out         [B, Hq, d]
- *   workspace   scratch of at least dck_decode_workspace_size(desc, B) bytes,
- *               256-byte aligned; its contents need no initialisation
+ *   workspace   scratch of at least dck_decode_workspace_size(desc, B, n_rows)
+ *               bytes, 256-byte aligned; its contents need no initialisation
  * Work is balanced over the device's SMs by 128-token tiles; the split
- * partials live in the workspace and are merged by a second kernel on the
- * same stream.
+ * partials live in the workspace and are merged by a last kernel on the same
+ * stream.  The bf16 tensor-core path also keeps per-tile softmax
+ * probabilities there, sized for sequences that do not share cache rows:
+ * more than ceil(n_rows / 128) + B tiles in all is reported as DCK_ERR_INVALID
+ * by dck_last_device_error and leaves `out` undefined.
  */
-size_t dck_decode_workspace_size(const dck_layer_desc* desc, int32_t batch);
+/* Workspace bytes for a decode call over `batch` sequences in caches of
+ * `n_rows` rows (0 for an invalid descriptor or when the device cannot be
+ * queried). */
+size_t dck_decode_workspace_size(const dck_layer_desc* desc, int32_t batch, int64_t n_rows);
 dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q,
                                 const void* kcache, const void* vcache, int64_t n_rows,
                                 const void* B_k, const void* B_v,
@@ -153,7 +159,7 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q,
  * same arguments minus the workspace: the split partials go to a fixed
  * 32 MiB array in the library's own device memory, which every GPU that
  * loads the library holds until the process exits.
- *   - Requests whose dck_decode_workspace_size exceeds 32 MiB are rejected
+ *   - Requests whose dck_decode_workspace_size(desc, B, n_rows) exceeds 32 MiB are rejected
  *     with DCK_ERR_WORKSPACE before anything is launched.
  *   - The first call on a device looks up the array's device address (a
  *     host-side set-up step); make that first call before any stream capture.

@@ -1,0 +1,356 @@
+// Value absorption in latent space on the tensor cores (Sec. III-D: the value
+// up-projection x W^(v) ~ z_v R_v is applied once, after the attention sum):
+//   U_seg[:, j] = sum over the tiles of a sequence segment of C_v[tile]^T P_tile[:, j]
+// with P_tile the bf16 probabilities the scores kernel wrote (already the
+// 128B-swizzled image of the UMMA B operand) and C_v[tile] the tile's value
+// latents [128 tokens x r_v].  The segments and their partial slots are those
+// of the scores kernel (the same flattened tile split over the same number of
+// CTAs), which has already written each segment's reference max and row sum.
+//
+// The scores kernel's reference max of a head can rise from one tile to the
+// next (it moves only when a tile's max exceeds it by 8); before such a tile
+// the epilogue warps rescale U by exp2(m_old - m_new) in TMEM, after the MMAs
+// of the earlier tiles have completed.  The MMA thread and the epilogue both
+// read from the stored maxima which tiles need this and hand off only there
+// (drain, then tile_ok), so each hand-off phase follows the MMA thread's own
+// commit.  U = [r_v / 128 chunks][Hq_pad heads] fp32 accumulators, one TMEM
+// lane per r_v row of a chunk.
+//
+// Warps: 0 producer (P images by bulk copy, value chunks by TMA, next tile's
+// values prefetched toward L2), 1 TMEM owner whose lane 0 issues the MMAs
+// (M = 128 r_v rows, N = Hq_pad, K = 16 tokens; 8 per chunk and tile),
+// 2-5 epilogue (one TMEM lane quadrant each: rescales and the U readout).
+// Every wait is bounded; on expiry the CTA records kErrTimeout and releases
+// TMEM after the work in flight has landed.
+#include <algorithm>
+#include <cstring>
+#include <mutex>
+
+#include "tc_common.cuh"
+#include "tc_host.h"
+#include "tmap.h"
+
+#ifndef DCK_AB_TRACE
+#define DCK_AB_TRACE(code) ((void)0)
+#endif
+#ifndef DCK_AB_TRACE_FLUSH
+#define DCK_AB_TRACE_FLUSH() ((void)0)
+#endif
+
+namespace dck {
+namespace {
+
+using namespace sm100;
+using namespace tc;
+
+constexpr int kAThreads = 192;
+constexpr int kVSlot = 16384;  // [128 tokens][64 rv] bf16, 128B-swizzled: one half of an r_v chunk
+constexpr int kNVs = 8;        // value slots: four chunks in flight
+constexpr int kPSlot = 8192;   // P image of one tile (Hq_pad <= 32)
+constexpr int kNP = 2;
+constexpr uint32_t kTmemCols = 512;
+
+struct AMaps {
+  CUtensorMap vc;
+};
+
+struct AbsArgs {
+  int hq_pad;
+  int n_chunks;        // r_v / 128
+  const uint8_t* pglob;
+  const float* mglob;
+  int64_t max_tiles;
+};
+
+struct ASmem {
+  uint8_t v[kNVs][kVSlot];
+  uint8_t p[kNP][kPSlot];
+  uint64_t v_full[kNVs], v_empty[kNVs], p_full[kNP], p_empty[kNP];
+  uint64_t drain, tile_ok, u_ready, u_free;
+  int scan[kAThreads];
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+__global__ void __launch_bounds__(kAThreads, 1)
+    absorb_tc_kernel(const __grid_constant__ AMaps maps, const LayerTable lt, const DecodeArgs a, const AbsArgs aa) {
+  extern __shared__ uint8_t smem_raw[];
+  ASmem& sm = *reinterpret_cast<ASmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  volatile int* abort_flag = &sm.abort_flag;
+  const int Hq = lt.Hq, hq_pad = aa.hq_pad, n_chunks = aa.n_chunks;
+  const uint32_t pbytes = (uint32_t)hq_pad * 256;
+
+  if (tid == 0) {
+    for (int i = 0; i < kNVs; ++i) {
+      mbar_init(&sm.v_full[i], 1);
+      mbar_init(&sm.v_empty[i], 1);
+    }
+    for (int i = 0; i < kNP; ++i) {
+      mbar_init(&sm.p_full[i], 1);
+      mbar_init(&sm.p_empty[i], 1);
+    }
+    mbar_init(&sm.drain, 1);
+    mbar_init(&sm.tile_ok, 4);
+    mbar_init(&sm.u_ready, 1);
+    mbar_init(&sm.u_free, 4);
+    sm.abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  int NT, b_first, pre_first;
+  tile_scan(a, sm.scan, a.n_items, NT, b_first, pre_first);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  const bool fits = NT <= aa.max_tiles;  // else the scores kernel has reported the input
+  const int x0 = fits ? item_begin(blockIdx.x, NT, a.n_items) : 0;
+  const int x1 = fits ? item_begin(blockIdx.x + 1, NT, a.n_items) : 0;
+  Walker walk{b_first, pre_first, x0, x1};
+  Segment seg;
+  DCK_AB_TRACE(0);
+
+  if (warp == 0) {
+    // ---- producer ------------------------------------------------------------
+    if (x0 < x1) {
+      const uint64_t pol = policy_evict_first();
+      int v_cnt = 0, p_cnt = 0;
+      bool ok = true;
+      while (ok && walk.next(a, seg)) {
+        for (int i = 0; i < seg.ntiles && ok; ++i) {
+          const int64_t x = seg.x0 + i;
+          const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
+          if (lane == 0 && i + 1 < seg.ntiles) {  // next tile's value rows toward L2
+            const int64_t r0 = yrow + kTile, nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
+            if (nr > 0)
+              prefetch_l2(static_cast<const __nv_bfloat16*>(a.vc) + r0 * lt.rv, (uint32_t)(nr * lt.rv * 2));
+          }
+          if (!(ok = wait_slots(sm.p_empty, kNP, p_cnt, 1, lane, abort_flag))) break;
+          if (lane == 0) {
+            const int sl = p_cnt % kNP;
+            mbar_expect_tx(&sm.p_full[sl], pbytes);
+            bulk_load(sm.p[sl], aa.pglob + x * pbytes, pbytes, &sm.p_full[sl], pol);
+          }
+          __syncwarp();
+          DCK_AB_TRACE(1);
+          ++p_cnt;
+          for (int c = 0; c < n_chunks && ok; ++c) {
+            if (!(ok = wait_slots(sm.v_empty, kNVs, v_cnt, 2, lane, abort_flag))) break;
+            if (lane < 2) {
+              const int sl = (v_cnt + lane) % kNVs;
+              mbar_expect_tx(&sm.v_full[sl], kVSlot);
+              tma_load_2d_hint(sm.v[sl], &maps.vc, &sm.v_full[sl], 128 * c + 64 * lane, (int32_t)yrow, pol);
+            }
+            __syncwarp();
+            DCK_AB_TRACE(2);
+            v_cnt += 2;
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---- MMA issuer (lane 0) ---------------------------------------------------
+    if (lane == 0 && x0 < x1) {
+      const uint32_t idesc_v = idesc_bf16(128, hq_pad, true, false);
+      int v_cnt = 0, p_cnt = 0, rc = 0, sgc = 0;
+      bool ok = true;
+      while (ok && walk.next(a, seg)) {
+        for (int i = 0; i < seg.ntiles && ok; ++i) {
+          if (i > 0) {
+            // did any head's reference max rise at this tile?  Then the epilogue
+            // rescales U once the earlier tiles' MMAs are done (drain) and
+            // releases this tile (tile_ok).
+            const int64_t x = seg.x0 + i;
+            bool need = false;
+            for (int j = 0; j < Hq; ++j) need |= aa.mglob[x * Hq + j] > aa.mglob[(x - 1) * Hq + j];
+            if (need) {
+              umma_commit(&sm.drain);
+              if (!(ok = mbar_wait(&sm.tile_ok, rc & 1, abort_flag))) break;
+              tc_fence_after();
+              DCK_AB_TRACE(10);
+              ++rc;
+            }
+          } else if (sgc > 0) {  // the epilogue has read the previous segment's U
+            if (!(ok = mbar_wait(&sm.u_free, (sgc - 1) & 1, abort_flag))) break;
+            tc_fence_after();
+          }
+          const int psl = p_cnt % kNP;
+          if (!(ok = mbar_wait(&sm.p_full[psl], (p_cnt / kNP) & 1, abort_flag))) break;
+          DCK_AB_TRACE(11);
+          const int nvalid = i == seg.ntiles - 1 ? seg.t_end - (seg.t_begin + kTile * i) : kTile;
+          const uint32_t pbase = smem_u32(sm.p[psl]);
+          for (int c = 0; c < n_chunks && ok; ++c) {
+            const int sl = v_cnt % kNVs;  // even: the chunk's halves are adjacent slots
+            const uint32_t vpar = (v_cnt / kNVs) & 1;
+            if (!(ok = mbar_wait(&sm.v_full[sl], vpar, abort_flag))) break;
+            if (!(ok = mbar_wait(&sm.v_full[sl + 1], vpar, abort_flag))) break;
+            if (nvalid < kTile) {  // rows past the sequence end: exact zeros
+              for (int r = nvalid; r < kTile; ++r)
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                  reinterpret_cast<uint4*>(sm.v[sl] + r * 128)[q] = make_uint4(0, 0, 0, 0);
+                  reinterpret_cast<uint4*>(sm.v[sl + 1] + r * 128)[q] = make_uint4(0, 0, 0, 0);
+                }
+              fence_proxy_async_smem();
+            }
+            const uint32_t vb = smem_u32(sm.v[sl]);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const uint64_t ad = sdesc(vb + k * 2048, kVSlot, 1024, kSw128);
+              const uint64_t bd = sdesc(pbase + (k >> 2) * (hq_pad * 128) + (k & 3) * 32, 16, 1024, kSw128);
+              umma_f16(tmem + c * hq_pad, ad, bd, idesc_v, (i == 0 && k == 0) ? 0u : 1u);
+            }
+            umma_commit(&sm.v_empty[sl]);
+            umma_commit(&sm.v_empty[sl + 1]);
+            DCK_AB_TRACE(12);
+            v_cnt += 2;
+          }
+          if (!ok) break;
+          umma_commit(&sm.p_empty[psl]);
+          ++p_cnt;
+        }
+        if (!ok) break;
+        umma_commit(&sm.u_ready);
+        DCK_AB_TRACE(13);
+        ++sgc;
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---- epilogue (warps 2-5): rescales between tiles, U readout -------------
+    const int quad = warp & 3;
+    const int tau = quad * 32 + lane;  // r_v row inside a chunk
+    const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+    int rc = 0, sgc = 0;
+    bool ok = true;
+    while (ok && walk.next(a, seg)) {
+      for (int i = 1; i < seg.ntiles && ok; ++i) {
+        const int64_t x = seg.x0 + i;
+        // reference maxima of this tile and the previous one, head = lane
+        const float mn = lane < Hq ? aa.mglob[x * Hq + lane] : 0.f;
+        const float mo = lane < Hq ? aa.mglob[(x - 1) * Hq + lane] : 0.f;
+        if (__any_sync(0xffffffffu, mn > mo)) {
+          if (!(ok = wwait(&sm.drain, rc & 1, abort_flag))) break;
+          tc_fence_after();
+          const float al = lane < Hq ? exp2f(mo - mn) : 1.f;  // this lane's head
+          for (int c = 0; c < n_chunks; ++c)
+            for (int cb = 0; cb < hq_pad / 16; ++cb) {
+              float v[16];
+              const uint32_t tad = tmem + lane_base + c * hq_pad + 16 * cb;
+              tmem_ld16(tad, v);
+              tmem_wait_ld();
+#pragma unroll
+              for (int i2 = 0; i2 < 16; ++i2) v[i2] *= __shfl_sync(0xffffffffu, al, 16 * cb + i2);
+              tmem_st16(tad, v);
+            }
+          tmem_wait_st();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.tile_ok);
+          DCK_AB_TRACE(20);
+          ++rc;
+        }
+      }
+      if (!ok) break;
+      // segment end: U -> partial slot c + b
+      if (!(ok = wwait(&sm.u_ready, sgc & 1, abort_flag))) break;
+      tc_fence_after();
+      DCK_AB_TRACE(22);
+      const int64_t slot = (int64_t)blockIdx.x + seg.b;
+      float* dst = a.part_u + slot * Hq * lt.rv + tau;
+      for (int c = 0; c < n_chunks; ++c) {
+        float v0[16], v1[16];
+        tmem_ld16(tmem + lane_base + c * hq_pad, v0);
+        if (hq_pad > 16) tmem_ld16(tmem + lane_base + c * hq_pad + 16, v1);
+        tmem_wait_ld();
+#pragma unroll
+        for (int i2 = 0; i2 < 16; ++i2) {
+          if (i2 < Hq) dst[(int64_t)i2 * lt.rv + c * 128] = v0[i2];
+          if (16 + i2 < Hq) dst[(int64_t)(16 + i2) * lt.rv + c * 128] = v1[i2];
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.u_free);
+      ++sgc;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  DCK_AB_TRACE_FLUSH();
+  if (sm.abort_flag) {
+    const long long c0 = clock64();
+    while (clock64() - c0 < 4000000ll) {
+    }
+    if (tid == 0) atomicOr(a.err, kErrTimeout);
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+struct VKey {
+  const void* vc;
+  int64_t n_rows;
+  int rv;
+  bool operator==(const VKey& o) const { return vc == o.vc && n_rows == o.n_rows && rv == o.rv; }
+};
+constexpr int kVMaps = 64;
+std::mutex g_vmaps_mu;
+VKey g_vkey[kVMaps];
+AMaps g_vval[kVMaps];
+int g_vn = 0, g_vnext = 0;
+
+}  // namespace
+
+cudaError_t launch_absorb_tc(const LayerTable& lt, const DecodeArgs& a, const TcRegions& r, cudaStream_t s) {
+  if (r.hq_pad * 256 > kPSlot || (lt.rv / 128) * r.hq_pad > (int)kTmemCols) return cudaErrorInvalidValue;
+  const VKey key{a.vc, a.n_rows, lt.rv};
+  AMaps maps;
+  bool have = false;
+  {
+    std::lock_guard<std::mutex> lk(g_vmaps_mu);
+    for (int i = 0; i < g_vn && !have; ++i)
+      if (g_vkey[i] == key) {
+        maps = g_vval[i];
+        have = true;
+      }
+  }
+  if (!have) {
+    std::memset(&maps, 0, sizeof(maps));
+    const uint64_t rows = (uint64_t)std::max<int64_t>(1, a.n_rows);
+    if (!make_tmap_2d_bf16(&maps.vc, a.vc, lt.rv, rows, (uint64_t)lt.rv * 2, 64, kTile, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+    std::lock_guard<std::mutex> lk(g_vmaps_mu);
+    g_vkey[g_vnext] = key;
+    g_vval[g_vnext] = maps;
+    g_vnext = (g_vnext + 1) % kVMaps;
+    g_vn = std::min(g_vn + 1, kVMaps);
+  }
+  AbsArgs aa;
+  aa.hq_pad = r.hq_pad;
+  aa.n_chunks = lt.rv / 128;
+  aa.pglob = r.pglob;
+  aa.mglob = r.mglob;
+  aa.max_tiles = r.max_tiles;
+  const size_t smem = sizeof(ASmem) + 1024;
+  static int attr_done[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const bool dev_ok = dev >= 0 && dev < 64;
+  if (!dev_ok || !attr_done[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(absorb_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    if (dev_ok) attr_done[dev] = 1;
+  }
+  absorb_tc_kernel<<<a.n_items, kAThreads, smem, s>>>(maps, lt, a, aa);
+  return cudaGetLastError();
+}
+
+}  // namespace dck

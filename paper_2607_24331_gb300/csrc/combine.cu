@@ -8,13 +8,15 @@
 // and applies the value up-factor once per head (Sec. III-D, x W^(v) ~ z_v R_v):
 //   o_j = (u / l) B_v[:, h d : (h+1) d],  h = KV head of j.
 //
-// Grid: (KV head h, chunk of sequences) x cluster of kSplit CTAs along r_v.
-// CTA `rank` of a cluster owns rows [rank*rv/kSplit, (rank+1)*rv/kSplit) of u
+// Grid: (KV head h, chunk of sequences) x cluster of `split` CTAs along r_v
+// (8 where r_v allows, else 4); a chunk holds as many (sequence, query head)
+// rows as fit kMaxRows, so each head's B_v block is staged about once.
+// CTA `rank` of a cluster owns rows [rank*rv/split, (rank+1)*rv/split) of u
 // and of B_v's column block: it merges those rows of every (sequence, query
-// head) row of its chunk, stages its B_v rows in shared memory with cp.async
-// (all issued up front), and forms the partial product over its rows.  The
-// cluster adds the kSplit partial outputs through distributed shared memory
-// and rank 0 writes o.
+// head) row of its chunk (eight items' loads in flight at a time), stages its
+// B_v rows in shared memory with cp.async (all issued up front), and forms the
+// partial product over its rows.  The cluster adds the partial outputs through
+// distributed shared memory and rank 0 writes o.
 #include <algorithm>
 
 #include <cooperative_groups.h>
@@ -27,8 +29,9 @@ namespace dck {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kSplit = 4;       // CTAs per cluster (r_v split)
+constexpr int kMaxSplit = 8;    // CTAs per cluster (r_v split), portable cluster size
 constexpr int kMaxRows = 16;    // (sequence, query head) rows per cluster
+constexpr int kItemBatch = 8;   // partial items whose loads are in flight together
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)),
@@ -39,17 +42,18 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
 template <typename T, int D>
-__global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, const DecodeArgs a, int bchunk) {
+__global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, const DecodeArgs a, int bchunk,
+                                                          int split) {
   extern __shared__ __align__(16) uint8_t smem_c[];
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank();
   const int B = a.B;
   const int qpg = lt.qpg, rv = lt.rv, Hq = lt.Hq;
-  const int h = blockIdx.x / kSplit;
+  const int h = blockIdx.x / split;
   const int b0 = blockIdx.y * bchunk;
   const int nb = min(bchunk, B - b0);
   const int nrow = nb * qpg;
-  const int rr = rv / kSplit;           // rows of u / B_v owned by this CTA (rv % 64 == 0)
+  const int rr = rv / split;            // rows of u / B_v owned by this CTA (a multiple of 4)
   const int r0 = rank * rr;
 
   // shared layout: B_v rows [rr][D] T | u rows [kMaxRows][rr] | partial o [kMaxRows][D] | m, 1/l | scan | prefix
@@ -113,11 +117,11 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, 
       const int c0 = item_of_tile(prefix[b], NT, a.n_items);
       const int c1 = item_of_tile(prefix[b + 1] - 1, NT, a.n_items);
       const float Mi = sM[i];
-      for (int cc = c0; cc <= c1; cc += 4) {
-        float w[4];
-        float4 v[4];
+      for (int cc = c0; cc <= c1; cc += kItemBatch) {
+        float w[kItemBatch];
+        float4 v[kItemBatch];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < kItemBatch; ++u) {
           const int c = cc + u;
           const bool live = c <= c1 && item_begin(c, NT, a.n_items) != item_begin(c + 1, NT, a.n_items);
           const int64_t sl = ((int64_t)(live ? c : c0) + b) * Hq + j;
@@ -125,7 +129,7 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, 
           v[u] = reinterpret_cast<const float4*>(a.part_u + sl * rv + r0)[r4];
         }
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < kItemBatch; ++u) {
           acc.x = fmaf(w[u], v[u].x, acc.x);
           acc.y = fmaf(w[u], v[u].y, acc.y);
           acc.z = fmaf(w[u], v[u].z, acc.z);
@@ -169,7 +173,7 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, 
     T* out = static_cast<T*>(a.out);
     for (int idx = threadIdx.x; idx < nrow * D; idx += kThreads) {
       float v = 0.f;
-      for (int q = 0; q < kSplit; ++q) v += cluster.map_shared_rank(so, q)[idx];
+      for (int q = 0; q < split; ++q) v += cluster.map_shared_rank(so, q)[idx];
       const int i = idx / D, e = idx % D;
       const int b = b0 + i / qpg, j = h * qpg + i % qpg;
       out[((int64_t)b * Hq + j) * D + e] = from_f32<T>(v * sinv[i]);
@@ -183,11 +187,10 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int maxb = std::max(1, kMaxRows / lt.qpg);
-  // about one cluster per kSplit SMs
-  int bchunk = (a.B * lt.Hkv * kSplit + sms - 1) / std::max(1, sms);
-  bchunk = std::max(1, std::min(bchunk, maxb));
-  const int rr = lt.rv / kSplit;
+  const int split = lt.rv % (4 * kMaxSplit) == 0 ? kMaxSplit : kMaxSplit / 2;
+  // as many sequences per cluster as its rows allow: each head's B_v block is staged once per chunk
+  const int bchunk = std::max(1, std::min(a.B, kMaxRows / lt.qpg));
+  const int rr = lt.rv / split;
   const size_t smem = (size_t)rr * D * sizeof(T) +
                       sizeof(float) * ((size_t)kMaxRows * rr + kMaxRows * D + 2 * kMaxRows) +
                       sizeof(int) * (kThreads + a.B + 1);
@@ -195,24 +198,24 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(lt.Hkv * kSplit, (a.B + bchunk - 1) / bchunk);
+  cfg.gridDim = dim3(lt.Hkv * split, (a.B + bchunk - 1) / bchunk);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kSplit;
+  attr[0].val.clusterDim.x = split;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k, lt, a, bchunk);
+  return cudaLaunchKernelEx(&cfg, k, lt, a, bchunk, split);
 }
 
 }  // namespace
 
-// r_v must split into kSplit parts of whole float4 and 16-byte rows.
-bool combine_supports(const LayerTable& lt) { return lt.rv % (4 * kSplit) == 0 && lt.rv <= kMaxRankV; }
+// r_v must split into at least four parts of whole float4 and 16-byte rows.
+bool combine_supports(const LayerTable& lt) { return lt.rv % (4 * kMaxSplit / 2) == 0 && lt.rv <= kMaxRankV; }
 
 cudaError_t launch_combine(const LayerTable& lt, const DecodeArgs& a, int dtype, cudaStream_t s) {
   if (dtype == DCK_F32) return lt.d == 64 ? launch_t<float, 64>(lt, a, s) : launch_t<float, 128>(lt, a, s);

@@ -11,7 +11,7 @@ namespace dck {
 bool simt_supports(const LayerTable& lt);
 bool combine_supports(const LayerTable& lt);
 bool tc_decode_supports(const LayerTable& lt, int dtype);
-size_t tc_decode_extra_ws(const LayerTable& lt, int batch);
+size_t tc_decode_extra_ws(const LayerTable& lt, int batch, int64_t n_rows);
 int tc_decode_launches(const LayerTable& lt);
 cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s);
 bool tc_append_supports(int D, int Rk, int rv, int dtype);
@@ -117,8 +117,8 @@ size_t decode_ws_parts(const LayerTable& lt, int batch, int n_items) {
 }
 
 // Workspace: split partials U and (m, l), then the tensor-core path's extra region.
-size_t decode_ws_bytes(const LayerTable& lt, int batch, int n_items, int dtype) {
-  return decode_ws_parts(lt, batch, n_items) + tc_decode_extra_ws(lt, dtype == DCK_BF16 ? batch : 0);
+size_t decode_ws_bytes(const LayerTable& lt, int batch, int n_items, int dtype, int64_t n_rows) {
+  return decode_ws_parts(lt, batch, n_items) + (dtype == DCK_BF16 ? tc_decode_extra_ws(lt, batch, n_rows) : 0);
 }
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
@@ -152,11 +152,11 @@ dck_status dck_set_timing_events(void* ev_start, void* ev_stop) {
   return DCK_OK;
 }
 
-size_t dck_decode_workspace_size(const dck_layer_desc* desc, int32_t batch) {
-  if (check_desc(desc) != DCK_OK || batch < 0) return 0;
+size_t dck_decode_workspace_size(const dck_layer_desc* desc, int32_t batch, int64_t n_rows) {
+  if (check_desc(desc) != DCK_OK || batch < 0 || n_rows < 0) return 0;
   int sms = 0;
   if (!device_state(nullptr, &sms)) return 0;
-  return decode_ws_bytes(make_table(desc), batch, sms, desc->dtype);
+  return decode_ws_bytes(make_table(desc), batch, sms, desc->dtype, n_rows);
 }
 
 dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const void* kcache, const void* vcache,
@@ -178,7 +178,7 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const
   int sms = 0;
   if (!device_state(&err, &sms)) return DCK_ERR_CUDA;
   const LayerTable lt = make_table(desc);
-  const size_t need = decode_ws_bytes(lt, batch, sms, desc->dtype);
+  const size_t need = decode_ws_bytes(lt, batch, sms, desc->dtype, n_rows);
   if (!workspace || ws_bytes < need || !aligned(workspace, 256)) return DCK_ERR_WORKSPACE;
   if (!simt_supports(lt) || !combine_supports(lt)) return DCK_ERR_UNSUPPORTED;
 

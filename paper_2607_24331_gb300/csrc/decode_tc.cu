@@ -1,4 +1,5 @@
-// Tensor-core (tcgen05) decode attention over DynaCalKV latent caches, bf16.
+// Tensor-core (tcgen05) decode attention over DynaCalKV latent caches, bf16:
+// the scores kernel (key reconstruction, RoPE, scores, online softmax).
 //
 // One persistent CTA per SM walks its share of 128-token tiles (see
 // DecodeArgs).  For every tile and every key group g (Sec. III-C) the group's
@@ -7,7 +8,8 @@
 // (tcgen05.mma, M = 128 tokens, N = 256 or 128, K = r_g, fp32 accumulator in
 // TMEM).  A pair shares every read of the latent operand: one-head MMAs that
 // read fresh shared-memory operands run the tensor pipe at about half rate.
-// Per head:
+// Two 256-column accumulators (all of TMEM) let the epilogue read one unit
+// while the tensor core computes the next.  Per head:
 //
 //  * key mode (several query heads per KV head): the factor is B_g[:, slot(h)],
 //    the product is the reconstructed key K^_h = C_g B_g[:, slot(h)]
@@ -30,21 +32,17 @@
 //
 // Scores are in log2 units; the online softmax keeps a per-head reference max
 // that moves only when a tile's max exceeds it by 8 (probabilities <= 256).
-// The value latents are absorbed in latent space (Sec. III-D, x W^(v) ~ z_v R_v
-// applied after the sum):  U[:, j] += C_v[tile]^T . P[:, j]  (tcgen05.mma,
-// M = 128 rv rows, N = query heads padded to 16, K = tokens; U stays in TMEM).
-// The key accumulator has one 256-column TMEM buffer (U takes the other half),
-// so while the epilogue reads a unit the MMA thread issues a pending r_v chunk
-// of the previous tile's absorption if its inputs are ready.  At the end of each
-// sequence segment U, the reference max and the row sum are written as a split
-// partial; the combine kernel merges splits and applies B_v.
+// Each tile's probabilities P (bf16, laid out as the B operand of the value
+// absorption) and the reference maxima they were computed with go to the
+// workspace; at the end of each sequence segment the reference max and the
+// row sum (over the rounded P) are written as the segment's split partial.
+// The absorption kernel (absorb_tc.cu) forms U = C_v^T P from them.
 //
-// Warp roles (384 threads).  Every TMA or bulk-copy instruction costs its
-// issuing thread a long round trip, so loads are issued by three producer warps,
+// Warp roles (352 threads).  Every TMA or bulk-copy instruction costs its
+// issuing thread a long round trip, so loads are issued by two producer warps,
 // each putting several copies (one per lane) into one instruction:
 //   warp 0     latent pieces of C_g (ring A)
-//   warp 10    value pieces of C_v (ring V, both halves of an r_v chunk at once)
-//   warp 11    factor items (ring W)
+//   warp 10    factor items (ring W)
 //   warp 1     TMEM owner; its lane 0 alone runs the MMA schedule (on this GPU
 //              every barrier test, commit or fence costs a dependent round trip
 //              of 100-200 cycles, so the issuing path is kept to one thread and
@@ -60,15 +58,15 @@
 //           swizzle: UMMA operand A of the reconstruction;
 //   W slot  [nh heads][2 halves][w ranks][64 columns] MN-major: operand B
 //           (N = 128 nh, the 64-column atoms w * 128 bytes apart);
-//   V pair  two slots [128 tokens][64 rv] (r_v chunk halves), MN-major
-//           operand A of the value absorption;
-//   P       [2 token atoms][Hq_pad heads][64 tokens] bf16, K-major operand B.
+//   P       [2 token atoms][Hq_pad heads][64 tokens] bf16, K-major (the
+//           absorption's operand B), staged here and bulk-stored per tile.
 #include <algorithm>
+#include <cmath>
 #include <cstring>
 #include <mutex>
 
-#include "common.cuh"
-#include "sm100.cuh"
+#include "tc_common.cuh"
+#include "tc_host.h"
 #include "tmap.h"
 
 #ifndef DCK_TC_TRACE
@@ -82,32 +80,32 @@ namespace dck {
 namespace {
 
 using namespace sm100;
+using namespace tc;
 
 constexpr int kD = 128;
-constexpr int kSlot = 16384;     // latent and value slots
+constexpr int kSlot = 16384;     // latent slots
 constexpr int kSlotW = 32768;    // factor slots: up to 2 heads x 64 ranks x 128 columns
-constexpr int kNA = 4;            // latent-piece ring depth
-constexpr int kNV = 2;            // value ring depth (one r_v chunk: two halves)
+constexpr int kNA = 4;           // latent-piece ring depth
 constexpr int kMaxGroupsTc = 16;
 constexpr int kMaxPieces = 5;
 constexpr int kMaxHqTc = 32;
 constexpr int kMaxItems = 256;
-constexpr int kThreads = 384;
+constexpr int kThreads = 352;
 constexpr int kEpiThreads = 256;
 constexpr float kRescaleThr = 8.f;  // log2 units: probabilities stay <= 256
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kUCol = 256;     // first TMEM column of the U accumulators
+constexpr uint32_t kKCols = 256;    // TMEM columns of one key accumulator
 constexpr float kTwoPi = 6.28318530717958647692f;
 constexpr float kInvTwoPi = 0.15915494309189533577f;
 constexpr float kLog2e = 1.4426950408889634f;
 
 template <bool kFold>
 struct Ring {
-  static constexpr int NW = kFold ? 3 : 2;  // factor-item ring depth (key mode keeps 16 KB for queries)
+  static constexpr int NW = kFold ? 4 : 3;  // factor-item ring depth (key mode keeps 16 KB for queries)
 };
 
 struct Maps {
-  CUtensorMap kc64, kc32, kc16, vc;
+  CUtensorMap kc64, kc32, kc16;
 };
 
 // Per-group facts the hot loops need; copied to shared memory at kernel start
@@ -126,10 +124,13 @@ struct GroupSm {
 
 struct TcArgs {
   int hq_pad;
-  int n_chunks;                  // rv / 128
   int n_items;                   // factor items per tile
   int64_t fimg_seq_bytes;        // factor image bytes per sequence (query-folded mode)
   const uint8_t* fimg;           // factor images (workspace)
+  uint8_t* pglob;                // per-tile P images (workspace)
+  float* mglob;                  // per-tile reference maxima (workspace)
+  int64_t max_tiles;
+  double om[kD / 2];             // RoPE frequencies theta^(-2i/d), fp64
   GroupSm grp[kMaxGroupsTc];
   int16_t order[kMaxHqTc];       // KV head at each MMA position (group-major, slot order)
   uint32_t item[kMaxItems];      // factor item n: byte offset | (bytes / 4096) << 26
@@ -139,8 +140,7 @@ template <bool kFold>
 struct Smem {
   uint8_t a[kNA][kSlot];
   uint8_t w[Ring<kFold>::NW][kSlotW];
-  uint8_t v[kNV][kSlot];
-  uint8_t p[2 * kMaxHqTc * 128];
+  uint8_t p[2 * kMaxHqTc * 128];            // P image of one tile, staged for its bulk store
   float x[kMaxHqTc * 128];                  // scores [head][token], accumulated atomically
   float qr[kFold ? 1 : kMaxHqTc * kD];      // key mode: rotated queries * log2(e)/sqrt(d)
   double om64[kD / 2];
@@ -150,192 +150,25 @@ struct Smem {
   float redl[4][kMaxHqTc];
   float mref[2][kMaxHqTc];  // reference max per head (log2 units), double-buffered by tile parity
   uint64_t a_full[kNA], a_empty[kNA];
-  uint64_t w_full[Ring<kFold>::NW], w_empty[Ring<kFold>::NW], v_full[kNV], v_empty[kNV];
-  uint64_t k_full, k_empty, p_full, p_empty, u_ready, u_free;
-  uint64_t epi_bar;
+  uint64_t w_full[Ring<kFold>::NW], w_empty[Ring<kFold>::NW];
+  uint64_t k_full[2], k_empty[2], p_done, epi_bar;
   GroupSm grp[kMaxGroupsTc];
   int16_t order[kMaxHqTc];
   uint32_t item[kMaxItems];
   uint32_t tmem_base;
   int abort_flag;
-  int b_first, pre_first, nt_total;
-};
-
-__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-__device__ __forceinline__ void griddep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
-
-__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar, uint64_t pol) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
-          smem_u32(dst)),
-      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(pol)
-      : "memory");
-}
-
-// Moves [src, src + bytes) toward L2 ahead of its TMA loads (16-byte multiples).
-__device__ __forceinline__ void prefetch_l2(const void* src, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
-}
-
-// Bounded wait whose outcome is the same in every lane of the warp.
-__device__ __forceinline__ bool wwait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
-  const bool r = mbar_wait(bar, parity, abort_flag);
-  return __all_sync(0xffffffffu, r);
-}
-
-// Single non-blocking test, same outcome in every lane.
-__device__ __forceinline__ bool wtest(uint64_t* bar, uint32_t parity) {
-  return __all_sync(0xffffffffu, mbar_test(bar, parity));
-}
-
-// Lane 0 waits for the `n` ring slots starting at ring position `cnt` (depth
-// `depth`) to be released; the result is shared with the warp.
-__device__ __forceinline__ bool wait_slots(uint64_t* empty, int depth, int cnt, int n, int lane,
-                                           volatile int* abort_flag) {
-  bool ok = true;
-  if (lane == 0)
-    for (int i = 0; i < n && ok; ++i) {
-      const int c = cnt + i;
-      if (c >= depth) ok = mbar_wait(&empty[c % depth], ((c / depth) - 1) & 1, abort_flag);
-    }
-  return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-}
-
-// Lane 0 waits for ring position `cnt` to be free, then counts how many of the
-// following positions (up to `max_n` in all) are free already, without
-// waiting.  Returns that count to the whole warp, 0 if the wait gave up.  (A
-// position is at most one use ahead of its release, so the parity test
-// cannot see a stale phase.)
-__device__ __forceinline__ int claim_slots(uint64_t* empty, int depth, int cnt, int max_n, int lane,
-                                           volatile int* abort_flag) {
-  int n = 0;
-  if (lane == 0 && (cnt < depth || mbar_wait(&empty[cnt % depth], ((cnt / depth) - 1) & 1, abort_flag))) {
-    n = 1;
-    while (n < max_n) {
-      const int c = cnt + n;
-      if (c >= depth && !mbar_test(&empty[c % depth], ((c / depth) - 1) & 1)) break;
-      ++n;
-    }
-  }
-  return __shfl_sync(0xffffffffu, n, 0);
-}
-
-__device__ __forceinline__ int ntiles_of(const DecodeArgs& a, int b) {
-  const int L = valid_len(a.seq_len, a.seq_start, b, a.n_rows);
-  return (L + kTile - 1) / kTile;
-}
-
-struct Segment {
-  int b, L, t_begin, t_end, ntiles;
-  int64_t row0;
-};
-
-// Walks the sequences overlapping tiles [x, x1) in order.
-struct Walker {
-  int b, pre, x, x1;
-  __device__ bool next(const DecodeArgs& a, Segment& sg) {
-    while (x < x1 && b < a.B) {
-      const int nt = ntiles_of(a, b);
-      if (x >= pre + nt) {
-        pre += nt;
-        ++b;
-        continue;
-      }
-      const int xe = min(x1, pre + nt);
-      sg.b = b;
-      sg.L = valid_len(a.seq_len, a.seq_start, b, a.n_rows);
-      sg.row0 = a.seq_start[b];
-      sg.t_begin = (x - pre) * kTile;
-      sg.t_end = min(sg.L, (xe - pre) * kTile);
-      sg.ntiles = xe - x;
-      x = xe;
-      return true;
-    }
-    return false;
-  }
 };
 
 __device__ __forceinline__ uint32_t swz_of(int w) { return w == 64 ? kSw128 : (w == 32 ? kSw64 : kSw32); }
 
-// Byte offset of P element (head j, token t) inside one P buffer.
+// Byte offset of P element (head j, token t) inside one P image.
 __device__ __forceinline__ uint32_t p_off(int j, int t, int hq_pad) {
   const int atom = t >> 6, col = t & 63;
   return atom * (hq_pad * 128) + (j >> 3) * 1024 + (j & 7) * 128 + ((((col >> 3) ^ (j & 7))) << 4) + ((col & 7) << 1);
 }
 
 // ---------------------------------------------------------------------------
-// Value absorption bookkeeping of the MMA warp: chunks are issued in
-// (tile, chunk) order; `pt`, `pc` name the next one.
-// ---------------------------------------------------------------------------
-
-struct Absorb {
-  int pt, pc;      // next tile (CTA-local tile counter) and r_v chunk to absorb
-  int v_cnt;       // value ring position
-  int seg_first;   // first tile of the current segment
-  int sgc;         // segment counter
-  bool p_seen;     // P of tile pt (and, first tile of a segment, U free) already observed
-};
-
-// Issues chunk (ab.pt, ab.pc) from the single MMA thread.  Non-blocking mode
-// returns false without issuing when its inputs are not ready; blocking mode
-// waits (bounded).  `nvalid`: valid tokens of the tile (rows past it are zeroed).
-template <bool kFold>
-__device__ __forceinline__ bool absorb_chunk(Smem<kFold>& sm, uint32_t tmem, const TcArgs& ta, Absorb& ab,
-                                             int nvalid, bool blocking, volatile int* abort_flag, bool& ok) {
-  const int tt = ab.pt, c = ab.pc;
-  const bool first = tt == ab.seg_first;
-  const uint32_t vpar = (ab.v_cnt / kNV) & 1;
-  if (!ab.p_seen) {
-    if (blocking) {
-      if (!(ok = mbar_wait(&sm.p_full, tt & 1, abort_flag))) return false;
-      if (first && ab.sgc > 0 && !(ok = mbar_wait(&sm.u_free, (ab.sgc - 1) & 1, abort_flag))) return false;
-    } else {
-      if (!mbar_test(&sm.p_full, tt & 1)) return false;
-      if (first && ab.sgc > 0 && !mbar_test(&sm.u_free, (ab.sgc - 1) & 1)) return false;
-    }
-    ab.p_seen = true;
-    tc_fence_after();  // the epilogue's TMEM accesses of U precede the next absorption
-  }
-  if (blocking) {
-    if (!(ok = mbar_wait(&sm.v_full[0], vpar, abort_flag))) return false;
-    if (!(ok = mbar_wait(&sm.v_full[1], vpar, abort_flag))) return false;
-  } else if (!mbar_test(&sm.v_full[1], vpar) || !mbar_test(&sm.v_full[0], vpar)) {
-    return false;
-  }
-  if (nvalid < 128) {  // rows past the sequence end: make them exact zeros
-    for (int r = nvalid; r < 128; ++r)
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        reinterpret_cast<uint4*>(sm.v[0] + r * 128)[q] = make_uint4(0, 0, 0, 0);
-        reinterpret_cast<uint4*>(sm.v[1] + r * 128)[q] = make_uint4(0, 0, 0, 0);
-      }
-    fence_proxy_async_smem();
-  }
-  DCK_TC_TRACE(12);
-  const int hq_pad = ta.hq_pad;
-  const uint32_t idesc_v = idesc_bf16(128, hq_pad, true, false);
-  const uint32_t pbase = smem_u32(sm.p);
-  const uint32_t vb = smem_u32(sm.v[0]);
-#pragma unroll
-  for (int k = 0; k < 8; ++k) {
-    const uint64_t ad = sdesc(vb + k * 2048, kSlot, 1024, kSw128);
-    const uint64_t bd = sdesc(pbase + (k >> 2) * (hq_pad * 128) + (k & 3) * 32, 16, 1024, kSw128);
-    umma_f16(tmem + kUCol + c * hq_pad, ad, bd, idesc_v, (first && k == 0) ? 0u : 1u);
-  }
-  umma_commit(&sm.v_empty[0]);
-  umma_commit(&sm.v_empty[1]);
-  if (c == ta.n_chunks - 1) umma_commit(&sm.p_empty);
-  ab.v_cnt += kNV;
-  if (++ab.pc == ta.n_chunks) {
-    ab.pc = 0;
-    ++ab.pt;
-    ab.p_seen = false;
-  }
-  return true;
-}
-
-// ---------------------------------------------------------------------------
-// the kernel
+// the scores kernel
 // ---------------------------------------------------------------------------
 
 template <bool kFold>
@@ -360,16 +193,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&sm.w_full[i], 1);
       mbar_init(&sm.w_empty[i], 1);
     }
-    for (int i = 0; i < kNV; ++i) {
-      mbar_init(&sm.v_full[i], 1);
-      mbar_init(&sm.v_empty[i], 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.k_full[i], 1);
+      mbar_init(&sm.k_empty[i], kEpiThreads / 32);
     }
-    mbar_init(&sm.k_full, 1);
-    mbar_init(&sm.k_empty, kEpiThreads / 32);
-    mbar_init(&sm.p_full, kEpiThreads / 32);
-    mbar_init(&sm.p_empty, 1);
-    mbar_init(&sm.u_ready, 1);
-    mbar_init(&sm.u_free, kEpiThreads / 32);
+    mbar_init(&sm.p_done, kEpiThreads / 32);
     mbar_init(&sm.epi_bar, kEpiThreads / 32);
     sm.abort_flag = 0;
     fence_mbar_init();
@@ -378,7 +206,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(&sm.tmem_base, kTmemCols);
     tmem_relinquish();
   }
-  {  // P starts at zero (padded head rows stay zero)
+  {  // the P image starts at zero (padded head rows stay zero)
     uint4* pz = reinterpret_cast<uint4*>(&sm.p[0]);
     for (int i = tid; i < (int)(sizeof(sm.p) / 16); i += kThreads) pz[i] = make_uint4(0, 0, 0, 0);
   }
@@ -386,59 +214,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid < lt.Hkv) sm.order[tid] = ta.order[tid];
   for (int n = tid; n < ta.n_items; n += kThreads) sm.item[n] = ta.item[n];
   if (tid < kD / 2) {
-    const double om = exp2(-2.0 * tid / kD * log2((double)a.theta));
-    sm.om64[tid] = om;
-    sm.om32[tid] = (float)om;
+    sm.om64[tid] = ta.om[tid];
+    sm.om32[tid] = (float)ta.om[tid];
   }
-  // total tiles and the first sequence of this item (block-wide scan)
-  {
-    int* scan = reinterpret_cast<int*>(sm.x);
-    const int per = (a.B + kThreads - 1) / kThreads;
-    const int b0 = tid * per;
-    int local = 0;
-    for (int b = b0; b < b0 + per && b < a.B; ++b) {
-      local += ntiles_of(a, b);
-      if (blockIdx.x == 0) {
-        const int64_t L = a.seq_len[b], st = a.seq_start[b];
-        if (L < 0 || st < 0 || st + L > a.n_rows) atomicOr(a.err, kErrBadSeq);
-      }
-    }
-    scan[tid] = local;
-    __syncthreads();
-    for (int off = 1; off < kThreads; off <<= 1) {
-      const int v = tid >= off ? scan[tid - off] : 0;
-      __syncthreads();
-      scan[tid] += v;
-      __syncthreads();
-    }
-    const int NT = scan[kThreads - 1];
-    const int x0 = item_begin(blockIdx.x, NT, a.n_items);
-    int run = tid ? scan[tid - 1] : 0;
-    if (tid == 0) {
-      sm.nt_total = NT;
-      sm.b_first = a.B;
-      sm.pre_first = NT;
-    }
-    __syncthreads();
-    for (int b = b0; b < b0 + per && b < a.B; ++b) {
-      const int nt = ntiles_of(a, b);
-      if (nt > 0 && x0 >= run && x0 < run + nt) {
-        sm.b_first = b;
-        sm.pre_first = run;
-      }
-      run += nt;
-    }
-    __syncthreads();
-    for (int i = tid; i < kMaxHqTc * 128; i += kThreads) sm.x[i] = 0.f;
-  }
+  int NT, b_first, pre_first;
+  tile_scan(a, reinterpret_cast<int*>(sm.x), a.n_items, NT, b_first, pre_first);
+  for (int i = tid; i < kMaxHqTc * 128; i += kThreads) sm.x[i] = 0.f;
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
-  const int NT = sm.nt_total;
-  const int x0 = item_begin(blockIdx.x, NT, a.n_items);
-  const int x1 = item_begin(blockIdx.x + 1, NT, a.n_items);
-  Walker walk{sm.b_first, sm.pre_first, x0, x1};
+  // the per-tile stores are sized for non-overlapping sequences; more tiles
+  // than that is reported as invalid input and nothing is computed
+  const bool fits = NT <= ta.max_tiles;
+  if (!fits && tid == 0 && blockIdx.x == 0) atomicOr(a.err, kErrBadSeq);
+  const int x0 = fits ? item_begin(blockIdx.x, NT, a.n_items) : 0;
+  const int x1 = fits ? item_begin(blockIdx.x + 1, NT, a.n_items) : 0;
+  Walker walk{b_first, pre_first, x0, x1};
   Segment seg;
   DCK_TC_TRACE(0);
 
@@ -471,7 +263,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tma_load_2d_hint(sm.a[sl], m, &sm.a_full[sl], gs.roff + gs.k[p0 + lane], (int32_t)yrow, pol);
               }
               __syncwarp();
-              DCK_TC_TRACE(300 + nb);
               a_cnt += nb;
               p0 += nb;
             }
@@ -480,33 +271,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else if (warp == 10) {
-    // ---- value pieces: both halves of an r_v chunk in one instruction -------
-    if (x0 < x1) {
-      const uint64_t pol = policy_evict_first();
-      int v_cnt = 0;
-      bool ok = true;
-      while (ok && walk.next(a, seg)) {
-        for (int i = 0; i < seg.ntiles && ok; ++i) {
-          const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
-          if (lane == 0) {  // this tile's value rows toward L2 (absorbed during the next tile)
-            const int64_t nr = a.n_rows - yrow < kTile ? a.n_rows - yrow : (int64_t)kTile;
-            if (nr > 0)
-              prefetch_l2(static_cast<const __nv_bfloat16*>(a.vc) + yrow * lt.rv, (uint32_t)(nr * lt.rv * 2));
-          }
-          for (int c = 0; c < ta.n_chunks && ok; ++c) {
-            if (!(ok = wait_slots(sm.v_empty, kNV, v_cnt, kNV, lane, abort_flag))) break;
-            if (lane < kNV) {
-              mbar_expect_tx(&sm.v_full[lane], kSlot);
-              tma_load_2d_hint(sm.v[lane], &maps.vc, &sm.v_full[lane], 128 * c + 64 * lane, (int32_t)yrow, pol);
-            }
-            __syncwarp();
-            DCK_TC_TRACE(3);
-            v_cnt += kNV;
-          }
-        }
-      }
-    }
-  } else if (warp == 11) {
     // ---- factor items: several bulk copies per instruction ------------------
     if (x0 < x1) {
       const uint64_t pol = policy_evict_last();
@@ -528,7 +292,6 @@ __global__ void __launch_bounds__(kThreads, 1)
               bulk_load(sm.w[sl], img + (it & 0x03FFFFFFu), bytes, &sm.w_full[sl], pol);
             }
             __syncwarp();
-            DCK_TC_TRACE(100000 + w_cnt * 10 + nb);
             w_cnt += nb;
             n0 += nb;
           }
@@ -539,15 +302,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---- MMA issuer: one thread runs the whole schedule (warp-wide
     // bookkeeping would only lengthen the path between MMAs) ----------------
     if (lane == 0 && x0 < x1) {
-      int a_cnt = 0, w_cnt = 0, kc = 0, tl = 0;
-      Absorb ab{0, 0, 0, 0, 0, false};
+      int a_cnt = 0, w_cnt = 0, kc = 0;
       bool ok = true;
       while (ok && walk.next(a, seg)) {
-        ab.seg_first = tl;
         for (int i = 0; i < seg.ntiles && ok; ++i) {
-          // the absorption of two tiles back must be complete before this tile's
-          // units: the epilogue's softmax step of the previous tile waits for it
-          while (ok && ab.pt < tl - 1) absorb_chunk<kFold>(sm, tmem, ta, ab, 128, true, abort_flag, ok);
           for (int g = 0; g < lt.G && ok; ++g) {
             const GroupSm& gs = sm.grp[g];
             const int np = gs.np, nu = gs.nu;
@@ -555,9 +313,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int u = 0; u < nu && ok; ++u) {
               const int nh = min(2, gs.nh - 2 * u);
               const uint32_t idesc_k = idesc_bf16(128, kD * nh, false, true);
-              // one key buffer: the epilogue has read the previous unit
-              if (kc >= 1) {
-                if (!(ok = mbar_wait(&sm.k_empty, (kc - 1) & 1, abort_flag))) break;
+              const int buf = kc & 1;
+              if (kc >= 2) {  // the epilogue has read this buffer's previous unit
+                if (!(ok = mbar_wait(&sm.k_empty[buf], ((kc >> 1) - 1) & 1, abort_flag))) break;
                 tc_fence_after();
               }
               DCK_TC_TRACE(10);
@@ -576,11 +334,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                   if (u == 0 && !mbar_test(&sm.a_full[(a_base + p) % kNA], ((a_base + p) / kNA) & 1))
                     miss |= 0x100u << p;
                 }
+              const uint32_t dcol = tmem + buf * kKCols;
               for (int p = 0; p < np; ++p) {
                 const int asl = (a_base + p) % kNA;
                 const int wsl = w_cnt % NW;
-                // an item not ready at the test is waited for here, in ring order (the
-                // factor ring may be shallower than a unit's item count)
                 if (((miss >> (8 + p)) & 1) && !(ok = mbar_wait(&sm.a_full[asl], ((a_base + p) / kNA) & 1, abort_flag)))
                   break;
                 if (((miss >> p) & 1) && !(ok = mbar_wait(&sm.w_full[wsl], (w_cnt / NW) & 1, abort_flag))) break;
@@ -591,41 +348,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int k = 0; k < w / 16; ++k) {
                   const uint64_t ad = sdesc(ab0 + k * 32, 16, 16 * w, swz);
                   const uint64_t bd = sdesc(bb + k * 2048, 128 * w, 1024, kSw128);
-                  umma_f16(tmem, ad, bd, idesc_k, (p > 0 || k > 0) ? 1u : 0u);
+                  umma_f16(dcol, ad, bd, idesc_k, (p > 0 || k > 0) ? 1u : 0u);
                 }
                 umma_commit(&sm.w_empty[wsl]);
                 if (u == nu - 1) umma_commit(&sm.a_empty[asl]);  // last unit of the group: piece done
                 ++w_cnt;
               }
               if (!ok) break;
-              umma_commit(&sm.k_full);
+              umma_commit(&sm.k_full[buf]);
               DCK_TC_TRACE(11);
               ++kc;
-              // while the epilogue drains the unit: one pending absorption chunk, if ready
-              if (ab.pt < tl) absorb_chunk<kFold>(sm, tmem, ta, ab, 128, false, abort_flag, ok);
             }
             a_cnt += np;
           }
-          ++tl;
         }
-        // segment end: the rest of the absorption, the last tile with its valid rows
-        while (ok && ab.pt < tl) {
-          const int nvalid = ab.pt == tl - 1 ? seg.t_end - (seg.t_begin + kTile * (seg.ntiles - 1)) : 128;
-          absorb_chunk<kFold>(sm, tmem, ta, ab, nvalid, true, abort_flag, ok);
-        }
-        if (ok) umma_commit(&sm.u_ready);
-        ++ab.sgc;
       }
     }
     __syncwarp();
   } else if (warp >= 2 && warp <= 9) {
-    // ---- epilogue: RoPE, scores, softmax, P, U readout ----------------------
+    // ---- epilogue: RoPE, scores, softmax, P -------------------------------
     const int e = tid - 64;              // 0 .. 255
     const int quad = warp & 3;           // TMEM lane quadrant
     const int hf = (warp - 2) >> 2;      // frequency half, then head half
     const int tau = quad * 32 + lane;    // token row inside the tile
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
-    int kc = 0, tl = 0, sgc = 0, round = 0;
+    const bool storer = e == 0;          // issues the per-tile bulk store of P (warp 2, lane 0)
+    int kc = 0, tl = 0, round = 0;
     bool ok = true;
     const int jb0 = 16 * hf;  // heads owned at tile and segment ends
 #define EPI_SYNC()                                  \
@@ -638,16 +386,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     while (ok && walk.next(a, seg)) {
       if (!kFold) {
         // rotated queries of this sequence at position L-1, scaled to log2 units
+        // (angle reduced mod 2 pi in fp64, sine and cosine in fp32)
         const double P = (double)(seg.L - 1);
         const float qscale = kLog2e * rsqrtf((float)kD);
         const __nv_bfloat16* qb = static_cast<const __nv_bfloat16*>(a.q) + (int64_t)seg.b * Hq * kD;
         for (int i = e; i < Hq * (kD / 2); i += kEpiThreads) {
           const int j = i / (kD / 2), pi = i % (kD / 2);
-          double sn, cs;
-          sincos(P * sm.om64[pi], &sn, &cs);
-          const double x1v = __bfloat162float(qb[j * kD + pi]), x2v = __bfloat162float(qb[j * kD + pi + kD / 2]);
-          sm.qr[j * kD + pi] = (float)(x1v * cs - x2v * sn) * qscale;
-          sm.qr[j * kD + pi + kD / 2] = (float)(x1v * sn + x2v * cs) * qscale;
+          const double ang = P * sm.om64[pi];
+          float sn, cs;
+          sincosf((float)(ang - 6.283185307179586 * rint(ang * 0.15915494309189535)), &sn, &cs);
+          const float x1v = __bfloat162float(qb[j * kD + pi]), x2v = __bfloat162float(qb[j * kD + pi + kD / 2]);
+          sm.qr[j * kD + pi] = (x1v * cs - x2v * sn) * qscale;
+          sm.qr[j * kD + pi + kD / 2] = (x1v * sn + x2v * cs) * qscale;
         }
       }
       // reference maxima start at -inf: the buffer a tile end reads is that of tile tl - 1
@@ -662,9 +412,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       // running row sums: one per (quadrant, head), kept by the warp owning both
       if (lane < 16 && jb0 + lane < Hq) sm.redl[quad][jb0 + lane] = 0.f;
-      const int tl_first = tl;
       for (int i = 0; i < seg.ntiles && ok; ++i) {
         const int t0 = seg.t_begin + kTile * i;
+        const int64_t x = seg.x0 + i;  // flattened tile index
         const bool valid = t0 + tau < seg.t_end;
         float cs[32], sn[32];
 #pragma unroll
@@ -679,12 +429,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           const GroupSm& gs = sm.grp[g];
           for (int u = 0; u < gs.nu; ++u) {
             const int nh = min(2, gs.nh - 2 * u);
-            if (!(ok = wwait(&sm.k_full, kc & 1, abort_flag))) break;
+            const int buf = kc & 1;
+            if (!(ok = wwait(&sm.k_full[buf], (kc >> 1) & 1, abort_flag))) break;
             tc_fence_after();
             DCK_TC_TRACE(20);
             for (int hh = 0; hh < nh; ++hh) {
               const int j0 = sm.order[gs.h0 + 2 * u + hh] * qpg;
-              const uint32_t cb = tmem + lane_base + hh * kD;
+              const uint32_t cb = tmem + lane_base + buf * kKCols + hh * kD;
               const bool last = hh == nh - 1;
               if (kFold) {
                 // Y columns [64 hf, 64 hf + 64): pairs (2i, 2i+1) of my 32 frequencies,
@@ -698,7 +449,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                   if (last && ps == 1) {
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(&sm.k_empty);
+                    if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
                   }
 #pragma unroll
                   for (int i2 = 0; i2 < 16; ++i2)
@@ -719,7 +470,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                   if (last && ps == 1) {
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(&sm.k_empty);
+                    if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
                   }
 #pragma unroll
                   for (int i2 = 0; i2 < 16; ++i2) {
@@ -742,7 +493,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         if (!ok) break;
-        // ---- tile end: reference max, optional rescale of U, P -------------
+        // ---- tile end: reference max, P ------------------------------------
         // Heads [jb, jb + 16) belong to this warp here (none for hf = 1 when
         // Hq <= 16); every per-head step runs over all 16 at once so that the
         // shared-memory and shuffle latencies overlap.
@@ -773,11 +524,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           const double ang = (double)(t0 + kTile) * sm.om64[e];
           sm.beta[e] = (float)(ang - 6.283185307179586 * floor(ang * 0.15915494309189535));
         }
-        EPI_SYNC();  // per-quadrant maxima are in redm
+        if (storer) bulk_store_wait_read();  // the previous tile's P image has left shared memory
+        EPI_SYNC();  // per-quadrant maxima are in redm; the P image may be rewritten
         DCK_TC_TRACE(28);
         if (!ok) break;
-        float al[16], mr[16];  // rescale factors, reference maxima after this tile
-        bool resc = false;
+        float al[16], mr[16];  // rescale factors of the row sums, reference maxima after this tile
         {
           float tm[16];
 #pragma unroll
@@ -793,42 +544,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (u < nh && (mr[u] == -INFINITY || tm[u] > mr[u] + kRescaleThr)) {
               al[u] = exp2f(mr[u] - tm[u]);
               mr[u] = tm[u];
-              resc = true;
             }
           }
           float v = mr[0];
 #pragma unroll
           for (int u = 1; u < 16; ++u) v = lane == u ? mr[u] : v;
-          if (quad == 0 && lane < nh) sm.mref[tl & 1][jb + lane] = v;
-        }
-        // the previous tile's absorption must be complete before U is rescaled
-        // or P is overwritten
-        if (tl >= 1 && !(ok = wwait(&sm.p_empty, (tl - 1) & 1, abort_flag))) break;
-        DCK_TC_TRACE(30);
-        if (resc && tl != tl_first) {
-          // rescale this warp's heads of U
-          tc_fence_after();
-          for (int c = 0; c < ta.n_chunks; ++c) {
-            float v[16];
-            const uint32_t tad = tmem + lane_base + kUCol + c * hq_pad + jb;
-            tmem_ld16(tad, v);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i2 = 0; i2 < 16; ++i2) v[i2] *= al[i2];
-            tmem_st16(tad, v);
+          if (quad == 0 && lane < nh) {
+            sm.mref[tl & 1][jb + lane] = v;
+            ta.mglob[x * Hq + jb + lane] = v;
           }
-          tmem_wait_st();
-          tc_fence_before();
         }
-        // probabilities -> P (bf16); row sums use the rounded values
-        uint8_t* pbuf = sm.p;
+        // probabilities -> P image (bf16); row sums use the rounded values
         float ps[16];
 #pragma unroll
         for (int u = 0; u < 16; ++u) {
           const __nv_bfloat16 pv = __float2bfloat16_rn(exp2f(sc[u] - mr[u]));
-          if (u < nh) *reinterpret_cast<__nv_bfloat16*>(pbuf + p_off(jb + u, tau, hq_pad)) = pv;
+          if (u < nh) *reinterpret_cast<__nv_bfloat16*>(sm.p + p_off(jb + u, tau, hq_pad)) = pv;
           ps[u] = u < nh ? __bfloat162float(pv) : 0.f;
         }
+        fence_proxy_async_smem();  // the bulk store reads the image through the async proxy
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.p_done);
 #pragma unroll
         for (int o = 16; o; o >>= 1)
 #pragma unroll
@@ -842,32 +578,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (lane < nh) sm.redl[quad][jb + lane] = fmaf(sm.redl[quad][jb + lane], a1, v);
         }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.p_full);
+        if (warp == 2) {  // the whole warp takes the decision, lane 0 issues the store
+          bool r = true;
+          if (storer) r = mbar_wait(&sm.p_done, tl & 1, abort_flag);
+          if (!(ok = __shfl_sync(0xffffffffu, r ? 1 : 0, 0) != 0)) break;
+          if (storer) bulk_store(ta.pglob + x * (hq_pad * 256), sm.p, (uint32_t)(hq_pad * 256));
+          __syncwarp();
+        }
         DCK_TC_TRACE(23);
         ++tl;
       }
       if (!ok) break;
-      // ---- segment end: U, reference max and row sums -> partial slot c + b ---
-      if (!(ok = wwait(&sm.u_ready, sgc & 1, abort_flag))) break;
-      tc_fence_after();
-      const int64_t slot = (int64_t)blockIdx.x + seg.b;
-      for (int c = hf; c < ta.n_chunks; c += 2) {
-        float v0[16], v1[16];
-        tmem_ld16(tmem + lane_base + kUCol + c * hq_pad, v0);
-        if (hq_pad > 16) tmem_ld16(tmem + lane_base + kUCol + c * hq_pad + 16, v1);
-        tmem_wait_ld();
-        float* dst = a.part_u + slot * Hq * lt.rv + c * 128 + tau;
-#pragma unroll
-        for (int i2 = 0; i2 < 16; ++i2) {
-          if (i2 < Hq) dst[(int64_t)i2 * lt.rv] = v0[i2];
-          if (16 + i2 < Hq) dst[(int64_t)(16 + i2) * lt.rv] = v1[i2];
-        }
-      }
-      tc_fence_before();
+      // ---- segment end: reference max and row sums -> partial slot c + b -----
       EPI_SYNC();
       if (!ok) break;
+      const int64_t slot = (int64_t)blockIdx.x + seg.b;
       if (quad == 0) {
         const int j = jb0 + lane;
         if (lane < 16 && j < Hq) {
@@ -875,11 +600,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           a.part_ml[(slot * Hq + j) * 2 + 1] = sm.redl[0][j] + sm.redl[1][j] + sm.redl[2][j] + sm.redl[3][j];
         }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.u_free);
-      ++sgc;
     }
 #undef EPI_SYNC
+    if (storer) bulk_store_wait();  // P images written before the absorption kernel reads them
   }
   tc_fence_before();
   __syncthreads();
@@ -912,6 +635,7 @@ struct PrepItem {
 struct PrepArgs {
   int n_items;
   int64_t seq_bytes;
+  double om[kD / 2];  // RoPE frequencies, fp64
   PrepItem item[kMaxItems];
 };
 
@@ -938,14 +662,15 @@ __global__ void __launch_bounds__(256) factor_prep_kernel(const LayerTable lt, c
       int kv = 0;
       for (int h = 0; h < lt.Hkv; ++h)
         if (lt.head_group[h] == g && lt.head_slot[h] == it.s0 + hh) kv = h;
-      const double om = exp2(-2.0 * i / kD * log2((double)a.theta));
-      double sn, cs;
-      sincos((double)(L - 1) * om, &sn, &cs);
+      // angle (L-1) w_i reduced mod 2 pi in fp64, sine and cosine in fp32
+      const double ang = (double)(L - 1) * pa.om[i];
+      float sn, cs;
+      sincosf((float)(ang - 6.283185307179586 * rint(ang * 0.15915494309189535)), &sn, &cs);
       const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(a.q) + ((int64_t)b * lt.Hq + kv) * kD;
-      const double x1 = __bfloat162float(q[i]), x2 = __bfloat162float(q[i + kD / 2]);
+      const float x1 = __bfloat162float(q[i]), x2 = __bfloat162float(q[i + kD / 2]);
       const float sc = kLog2e * rsqrtf((float)kD);
-      qa[hh][i] = (float)(x1 * cs - x2 * sn) * sc;
-      qb[hh][i] = (float)(x1 * sn + x2 * cs) * sc;
+      qa[hh][i] = (x1 * cs - x2 * sn) * sc;
+      qb[hh][i] = (x1 * sn + x2 * cs) * sc;
     }
     __syncthreads();
   }
@@ -1008,12 +733,10 @@ size_t image_bytes_of(const LayerTable& lt) {
 
 // Tensor maps depend only on the buffers and the layer: cache the last few.
 struct MapsKey {
-  const void *kc, *vc;
+  const void* kc;
   int64_t n_rows;
-  int Rk, rv;
-  bool operator==(const MapsKey& o) const {
-    return kc == o.kc && vc == o.vc && n_rows == o.n_rows && Rk == o.Rk && rv == o.rv;
-  }
+  int Rk;
+  bool operator==(const MapsKey& o) const { return kc == o.kc && n_rows == o.n_rows && Rk == o.Rk; }
 };
 constexpr int kMapsCache = 64;
 std::mutex g_maps_mu;
@@ -1026,8 +749,7 @@ bool build_maps(const LayerTable& lt, const DecodeArgs& a, Maps& maps) {
   const uint64_t rows = (uint64_t)std::max<int64_t>(1, a.n_rows);
   return make_tmap_2d_bf16(&maps.kc64, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 64, kTile, CU_TENSOR_MAP_SWIZZLE_128B) &&
          make_tmap_2d_bf16(&maps.kc32, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 32, kTile, CU_TENSOR_MAP_SWIZZLE_64B) &&
-         make_tmap_2d_bf16(&maps.kc16, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 16, kTile, CU_TENSOR_MAP_SWIZZLE_32B) &&
-         make_tmap_2d_bf16(&maps.vc, a.vc, lt.rv, rows, (uint64_t)lt.rv * 2, 64, kTile, CU_TENSOR_MAP_SWIZZLE_128B);
+         make_tmap_2d_bf16(&maps.kc16, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 16, kTile, CU_TENSOR_MAP_SWIZZLE_32B);
 }
 
 static_assert(sizeof(Smem<true>) + 1024 <= 232448, "shared memory of the query-folded kernel");
@@ -1047,7 +769,6 @@ cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& m
     if (e != cudaSuccess) return e;
     if (dev_ok) attr_done[dev] = 1;
   }
-  if (a.ev0 && record_timing_event(a.ev0, s) != cudaSuccess) return cudaErrorUnknown;
   factor_prep_kernel<kFold><<<dim3(pa.n_items, kFold ? a.B : 1), 256, 0, s>>>(lt, a, pa,
                                                                                 static_cast<uint8_t*>(a.extra));
   cudaError_t e = cudaGetLastError();
@@ -1062,9 +783,7 @@ cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& m
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, decode_tc_kernel<kFold>, maps, lt, a, ta);
-  if (e == cudaSuccess && a.ev1) e = record_timing_event(a.ev1, s);
-  return e;
+  return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kFold>, maps, lt, a, ta);
 }
 
 // Units, items and per-group tables of a layer.  Returns false when the layer
@@ -1073,7 +792,6 @@ bool build_tables(const LayerTable& lt, TcArgs& ta, PrepArgs& pa) {
   std::memset(&ta, 0, sizeof(ta));
   std::memset(&pa, 0, sizeof(pa));
   ta.hq_pad = hq_pad_of(lt.Hq);
-  ta.n_chunks = lt.rv / 128;
   int pos = 0, item = 0, off = 0;
   for (int g = 0; g < lt.G; ++g) {
     GroupSm& gs = ta.grp[g];
@@ -1116,12 +834,34 @@ bool build_tables(const LayerTable& lt, TcArgs& ta, PrepArgs& pa) {
   return true;
 }
 
+// RoPE frequencies w_i = theta^(-2i/d) in fp64 (positions reach 1e5 and more,
+// so the angle t w_i needs the extra precision before its reduction mod 2 pi).
+void rope_freqs(float theta, double* om) {
+  for (int i = 0; i < kD / 2; ++i) om[i] = std::exp2(-2.0 * i / kD * std::log2((double)theta));
+}
+
+// Workspace layout of the tensor-core path (after the split partials):
+// factor images, then the per-tile P images, then the per-tile reference maxima.
+struct ExtraLayout {
+  size_t img, p, m, total;
+};
+
+ExtraLayout extra_layout(const LayerTable& lt, int batch, int64_t n_rows) {
+  ExtraLayout x;
+  const int64_t nt = max_tiles(n_rows, batch);
+  x.img = align_up(lt.qpg == 1 ? image_bytes_of(lt) * std::max(batch, 1) : image_bytes_of(lt), 256);
+  x.p = align_up((size_t)nt * hq_pad_of(lt.Hq) * 256, 256);
+  x.m = align_up((size_t)nt * lt.Hq * sizeof(float), 256);
+  x.total = x.img + x.p + x.m;
+  return x;
+}
+
 }  // namespace
 
 bool tc_decode_supports(const LayerTable& lt, int dtype) {
   if (dtype != DCK_BF16 || lt.d != kD) return false;
   if (lt.Hq > kMaxHqTc || lt.qpg > kMaxQPerKv || lt.G > kMaxGroupsTc) return false;
-  if (lt.rv % 128 || (lt.rv / 128) * hq_pad_of(lt.Hq) > 256) return false;
+  if (lt.rv % 128 || (lt.rv / 128) * hq_pad_of(lt.Hq) > 512) return false;
   for (int g = 0; g < lt.G; ++g)
     if (lt.grp_rank[g] > 256 || lt.grp_rank[g] % 16) return false;
   static thread_local TcArgs ta;
@@ -1129,14 +869,13 @@ bool tc_decode_supports(const LayerTable& lt, int dtype) {
   return build_tables(lt, ta, pa);
 }
 
-// Extra workspace of the tensor-core path: the factor images.
-size_t tc_decode_extra_ws(const LayerTable& lt, int batch) {
+// Extra workspace of the tensor-core path.
+size_t tc_decode_extra_ws(const LayerTable& lt, int batch, int64_t n_rows) {
   if (!tc_decode_supports(lt, DCK_BF16)) return 0;
-  const size_t per = image_bytes_of(lt);
-  return align_up(lt.qpg == 1 ? per * std::max(batch, 1) : per, 256);
+  return extra_layout(lt, batch, n_rows).total;
 }
 
-int tc_decode_launches(const LayerTable&) { return 2; }
+int tc_decode_launches(const LayerTable&) { return 3; }
 
 cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) {
   const bool fold = lt.qpg == 1;
@@ -1144,8 +883,15 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStre
   static thread_local TcArgs ta;
   static thread_local PrepArgs pa;
   if (!build_tables(lt, ta, pa)) return cudaErrorInvalidValue;
-  ta.fimg = static_cast<const uint8_t*>(a.extra);
-  const MapsKey key{a.kc, a.vc, a.n_rows, lt.Rk, lt.rv};
+  rope_freqs(a.theta, ta.om);
+  std::memcpy(pa.om, ta.om, sizeof(ta.om));
+  const ExtraLayout xl = extra_layout(lt, a.B, a.n_rows);
+  uint8_t* base = static_cast<uint8_t*>(a.extra);
+  ta.fimg = base;
+  ta.pglob = base + xl.img;
+  ta.mglob = reinterpret_cast<float*>(base + xl.img + xl.p);
+  ta.max_tiles = max_tiles(a.n_rows, a.B);
+  const MapsKey key{a.kc, a.n_rows, lt.Rk};
   Maps maps;
   bool have = false;
   {
@@ -1164,7 +910,17 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStre
     g_maps_next = (g_maps_next + 1) % kMapsCache;
     g_maps_n = std::min(g_maps_n + 1, kMapsCache);
   }
-  return fold ? launch_mode<true>(lt, a, maps, ta, pa, s) : launch_mode<false>(lt, a, maps, ta, pa, s);
+  if (a.ev0 && record_timing_event(a.ev0, s) != cudaSuccess) return cudaErrorUnknown;
+  cudaError_t e = fold ? launch_mode<true>(lt, a, maps, ta, pa, s) : launch_mode<false>(lt, a, maps, ta, pa, s);
+  if (e != cudaSuccess) return e;
+  TcRegions r;
+  r.pglob = ta.pglob;
+  r.mglob = ta.mglob;
+  r.max_tiles = ta.max_tiles;
+  r.hq_pad = ta.hq_pad;
+  e = launch_absorb_tc(lt, a, r, s);
+  if (e == cudaSuccess && a.ev1) e = record_timing_event(a.ev1, s);
+  return e;
 }
 
 }  // namespace dck

@@ -57,7 +57,7 @@ extern "C" dck_status dck_decode_attention_noalloc(const dck_layer_desc* desc, c
   if (batch == 0)  // nothing to compute; the regular entry point returns DCK_OK without launching
     return dck_decode_attention(desc, q, kcache, vcache, n_rows, B_k, B_v, d_seq_start, d_seq_len, batch,
                                 rope_theta, out, nullptr, 0, stream);
-  const size_t need = dck_decode_workspace_size(desc, batch);
+  const size_t need = dck_decode_workspace_size(desc, batch, n_rows);
   if (need == 0) return DCK_ERR_CUDA;  // the device could not be queried
   if (need > kNoallocScratchBytes) return DCK_ERR_WORKSPACE;  // beyond the fixed 32 MiB scratch
   void* ws = noalloc_scratch();

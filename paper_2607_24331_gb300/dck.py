@@ -75,7 +75,7 @@ def lib() -> ctypes.CDLL:
     L.dck_latent_append.restype = I32
     L.dck_latent_append.argtypes = [D, P, I32, P, P, P, P, P, I64, P, SZ, P]
     L.dck_decode_workspace_size.restype = SZ
-    L.dck_decode_workspace_size.argtypes = [D, I32]
+    L.dck_decode_workspace_size.argtypes = [D, I32, I64]
     L.dck_decode_attention.restype = I32
     L.dck_decode_attention.argtypes = [D, P, P, P, I64, P, P, P, P, I32, F32, P, P, SZ, P]
     L.dck_decode_attention_noalloc.restype = I32
@@ -149,8 +149,8 @@ def dck_validate_desc(layer: Layer) -> int:
     return lib().dck_validate_desc(layer.ref)
 
 
-def dck_decode_workspace_size(layer: Layer, batch: int) -> int:
-    return lib().dck_decode_workspace_size(layer.ref, batch)
+def dck_decode_workspace_size(layer: Layer, batch: int, n_rows: int) -> int:
+    return lib().dck_decode_workspace_size(layer.ref, batch, n_rows)
 
 
 def dck_latent_append_workspace_size(layer: Layer, n_tok: int) -> int:

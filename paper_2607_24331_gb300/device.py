@@ -49,7 +49,7 @@ class DecodeBuffers:
         self.seq_start = torch.from_numpy(S.seq_starts(self.lens_host)).to(device)
         self.seq_len = torch.from_numpy(self.lens_host.astype(np.int32)).to(device)
         self.out = torch.empty((self.B, spec.n_q_heads, spec.head_dim), dtype=dt, device=device)
-        self.ws_bytes = dck.dck_decode_workspace_size(self.layer, self.B)
+        self.ws_bytes = dck.dck_decode_workspace_size(self.layer, self.B, self.n_rows)
         self.workspace = torch.empty(max(self.ws_bytes, 256), dtype=torch.uint8, device=device)
         self.q = self.kcache = self.vcache = self.B_k = self.B_v = None
 

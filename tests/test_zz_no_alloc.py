@@ -45,7 +45,7 @@ def test_noalloc_rejects_requests_beyond_its_scratch():
     spec = S.LayerSpec(4096, 32, 32, 128, (tuple(range(32)),), (256,), 2048, "bf16", 1e4)
     lens = (1,) * 4096
     buf = device.DecodeBuffers(spec, lens).synth(seed=1)   # valid buffers of the full request
-    assert dck.dck_decode_workspace_size(buf.layer, buf.B) > (32 << 20)
+    assert dck.dck_decode_workspace_size(buf.layer, buf.B, buf.n_rows) > (32 << 20)
     r = dck.dck_decode_attention_noalloc(buf.layer, buf.q, buf.kcache, buf.vcache, buf.n_rows, buf.B_k, buf.B_v,
                                          buf.seq_start, buf.seq_len, buf.B, spec.rope_theta, buf.out)
     assert r == dck.DCK_ERR_WORKSPACE
