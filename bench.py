@@ -54,7 +54,7 @@ def load_peaks():
 
 def kernel_source_sha():
     h = hashlib.sha256()
-    for fn in ("decode_tc.cu", "decode_simt.cu", "common.cuh"):
+    for fn in ("decode_tc.cu", "absorb_tc.cu", "tc_common.cuh", "sm100.cuh", "decode_simt.cu", "common.cuh"):
         p = os.path.join(ROOT, "paper_2607_24331_gb300", "csrc", fn)
         if os.path.exists(p):
             h.update(open(p, "rb").read())
@@ -62,7 +62,8 @@ def kernel_source_sha():
 
 
 def profiled_traffic(cfg):
-    """DRAM bytes per launch of the main decode kernel from the committed ncu summary, if current."""
+    """DRAM bytes per call of the attention kernels (factor preparation, scores, absorption) from the
+    committed ncu summary, if it was taken on the current sources."""
     p = os.path.join(ROOT, "profiles", "decode_main_traffic.json")
     if not os.path.exists(p):
         return None
@@ -370,7 +371,8 @@ def main():
         e2e_ms = float(tt.item())
     e2e_value = world * B * K / (e2e_ms / 1e3)
 
-    # ---- roofline of the main attention kernel (one launch = one layer) ----
+    # ---- roofline of the attention kernels of one decode call (factor preparation, scores,
+    # absorption: the region between the timing events; one call = one layer) ----
     peaks = load_peaks()
     buf0 = layers[-1][0]
     alg_bytes = buf0.algorithmic_bytes()
@@ -382,7 +384,7 @@ def main():
         sum((a.numel() + v.numel()) * a.element_size() for (_b, a, v, *_r) in layers)
     roof = {"bound": "hbm", "achieved": achieved_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
             "frac": achieved_gbs / peaks["hbm_gbs"], "traffic": profiled_traffic(args.config),
-            "kernel": "main decode-attention kernel", "kernel_us": 1e6 * k_avg_s,
+            "kernel": "attention kernels of one call (factor prep + scores + absorption)", "kernel_us": 1e6 * k_avg_s,
             "alg_bytes_per_launch": alg_bytes, "peak_source": peaks["source"],
             "tensor_tflops": tflops, "tensor_frac": tflops / peaks["bf16_tflops"],
             "roofline_us": 1e6 * max(alg_bytes / (peaks["hbm_gbs"] * 1e9), flops / (peaks["bf16_tflops"] * 1e12))}
