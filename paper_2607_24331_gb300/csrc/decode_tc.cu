@@ -38,15 +38,18 @@
 // row sum (over the rounded P) are written as the segment's split partial.
 // The absorption kernel (absorb_tc.cu) forms U = C_v^T P from them.
 //
-// Warp roles (352 threads).  Every TMA or bulk-copy instruction costs its
-// issuing thread a long round trip, so loads are issued by two producer warps,
-// each putting several copies (one per lane) into one instruction:
+// Warp roles (384 threads query-folded, 352 key mode).  Every TMA or
+// bulk-copy instruction costs its issuing thread a long round trip, so loads
+// are issued by two producer warps, each putting several copies (one per lane)
+// into one instruction:
 //   warp 0     latent pieces of C_g (ring A)
-//   warp 10    factor items (ring W)
-//   warp 1     TMEM owner; its lane 0 alone runs the MMA schedule (on this GPU
-//              every barrier test, commit or fence costs a dependent round trip
-//              of 100-200 cycles, so the issuing path is kept to one thread and
-//              the fewest such operations per MMA)
+//   warp 10    factor items (ring W; query-folded mode: one ring per MMA thread)
+//   warp 1     TMEM owner; its lane 0 issues MMAs.  On this GPU every barrier
+//              test, commit or fence costs the issuing thread a dependent round
+//              trip of 100-500 cycles, longer than the MMAs of a factor item, so
+//              in query-folded mode lane 0 of warp 11 issues every other unit
+//              into the other accumulator and the two threads' bookkeeping
+//              overlaps the other's MMAs
 //   warps 2-9  epilogue: each TMEM lane quadrant (32 tokens) is served by two
 //              warps that split the 64 RoPE frequency pairs of a head and add
 //              their partial scores with shared-memory atomics.
@@ -90,7 +93,6 @@ constexpr int kMaxGroupsTc = 16;
 constexpr int kMaxPieces = 5;
 constexpr int kMaxHqTc = 32;
 constexpr int kMaxItems = 256;
-constexpr int kThreads = 352;
 constexpr int kEpiThreads = 256;
 constexpr float kRescaleThr = 8.f;  // log2 units: probabilities stay <= 256
 constexpr uint32_t kTmemCols = 512;
@@ -101,7 +103,10 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 template <bool kFold>
 struct Ring {
-  static constexpr int NW = kFold ? 4 : 3;  // factor-item ring depth (key mode keeps 16 KB for queries)
+  static constexpr int NW = kFold ? 4 : 3;  // factor-item slots (key mode keeps 16 KB for queries)
+  static constexpr int kMma = kFold ? 2 : 1;  // MMA-issuing threads, each with its own factor ring
+  static constexpr int NWt = NW / kMma;       // slots of one MMA thread's ring
+  static constexpr int kThreads = kFold ? 384 : 352;
 };
 
 struct Maps {
@@ -140,18 +145,14 @@ template <bool kFold>
 struct Smem {
   uint8_t a[kNA][kSlot];
   uint8_t w[Ring<kFold>::NW][kSlotW];
-  uint8_t p[2 * kMaxHqTc * 128];            // P image of one tile, staged for its bulk store
   float x[kMaxHqTc * 128];                  // scores [head][token], accumulated atomically
   float qr[kFold ? 1 : kMaxHqTc * kD];      // key mode: rotated queries * log2(e)/sqrt(d)
   double om64[kD / 2];
   float om32[kD / 2];
   float beta[kD / 2];
-  float redm[4][kMaxHqTc];
-  float redl[4][kMaxHqTc];
-  float mref[2][kMaxHqTc];  // reference max per head (log2 units), double-buffered by tile parity
   uint64_t a_full[kNA], a_empty[kNA];
   uint64_t w_full[Ring<kFold>::NW], w_empty[Ring<kFold>::NW];
-  uint64_t k_full[2], k_empty[2], p_done, epi_bar;
+  uint64_t k_full[2], k_empty[2], epi_bar;
   GroupSm grp[kMaxGroupsTc];
   int16_t order[kMaxHqTc];
   uint32_t item[kMaxItems];
@@ -161,20 +162,15 @@ struct Smem {
 
 __device__ __forceinline__ uint32_t swz_of(int w) { return w == 64 ? kSw128 : (w == 32 ? kSw64 : kSw32); }
 
-// Byte offset of P element (head j, token t) inside one P image.
-__device__ __forceinline__ uint32_t p_off(int j, int t, int hq_pad) {
-  const int atom = t >> 6, col = t & 63;
-  return atom * (hq_pad * 128) + (j >> 3) * 1024 + (j & 7) * 128 + ((((col >> 3) ^ (j & 7))) << 4) + ((col & 7) << 1);
-}
-
 // ---------------------------------------------------------------------------
 // the scores kernel
 // ---------------------------------------------------------------------------
 
 template <bool kFold>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     decode_tc_kernel(const __grid_constant__ Maps maps, const LayerTable lt, const DecodeArgs a, const TcArgs ta) {
-  constexpr int NW = Ring<kFold>::NW;
+  constexpr int NW = Ring<kFold>::NW, kMma = Ring<kFold>::kMma, NWt = Ring<kFold>::NWt;
+  constexpr int kThreads = Ring<kFold>::kThreads;
   extern __shared__ uint8_t smem_raw[];
   Smem<kFold>& sm =
       *reinterpret_cast<Smem<kFold>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -187,7 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) {
     for (int i = 0; i < kNA; ++i) {
       mbar_init(&sm.a_full[i], 1);
-      mbar_init(&sm.a_empty[i], 1);
+      mbar_init(&sm.a_empty[i], kMma);  // released by every MMA thread
     }
     for (int i = 0; i < NW; ++i) {
       mbar_init(&sm.w_full[i], 1);
@@ -197,7 +193,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&sm.k_full[i], 1);
       mbar_init(&sm.k_empty[i], kEpiThreads / 32);
     }
-    mbar_init(&sm.p_done, kEpiThreads / 32);
     mbar_init(&sm.epi_bar, kEpiThreads / 32);
     sm.abort_flag = 0;
     fence_mbar_init();
@@ -205,10 +200,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     tmem_alloc(&sm.tmem_base, kTmemCols);
     tmem_relinquish();
-  }
-  {  // the P image starts at zero (padded head rows stay zero)
-    uint4* pz = reinterpret_cast<uint4*>(&sm.p[0]);
-    for (int i = tid; i < (int)(sizeof(sm.p) / 16); i += kThreads) pz[i] = make_uint4(0, 0, 0, 0);
   }
   if (tid < lt.G) sm.grp[tid] = ta.grp[tid];
   if (tid < lt.Hkv) sm.order[tid] = ta.order[tid];
@@ -234,13 +225,38 @@ __global__ void __launch_bounds__(kThreads, 1)
   Segment seg;
   DCK_TC_TRACE(0);
 
+  // Factor items of one unit into MMA thread rw's ring (query-folded mode): up to
+  // NWt bulk copies per instruction, one per lane, as their slots come free.
+  auto put_unit_items = [&](int rw, int& wc, int n, int np, const uint8_t* img, uint64_t pol) -> bool {
+    for (int p0 = 0; p0 < np;) {
+      const int nb = claim_slots(sm.w_empty + rw * NWt, NWt, wc, np - p0, lane, abort_flag);
+      if (nb == 0) return false;
+      DCK_TC_TRACE(30 + nb);
+      if (lane < nb) {
+        const int sl = rw * NWt + (wc + lane) % NWt;
+        const uint32_t it = sm.item[n + p0 + lane];
+        const uint32_t bytes = (it >> 26) << 12;
+        mbar_expect_tx(&sm.w_full[sl], bytes);
+        bulk_load(sm.w[sl], img + (it & 0x03FFFFFFu), bytes, &sm.w_full[sl], pol);
+      }
+      __syncwarp();
+      wc += nb;
+      p0 += nb;
+    }
+    return true;
+  };
+
   if (warp == 0) {
-    // ---- latent pieces, issued as soon as their slots are free --------------
+    // ---- latent pieces, issued as soon as their slots are free; in
+    // query-folded mode also the factor items of MMA thread 1, in the order
+    // that thread consumes them (a group's pieces, then its units' items) ------
     if (x0 < x1) {
       const uint64_t pol = policy_evict_first();
-      int a_cnt = 0;
-      bool ok = true;
+      const uint64_t pol_w = policy_evict_last();
+      int a_cnt = 0, wc = 0, kc = 0;
+      bool ok = true, images_ready = false;
       while (ok && walk.next(a, seg)) {
+        const uint8_t* img = ta.fimg + (kFold ? (int64_t)seg.b * ta.fimg_seq_bytes : 0);
         for (int i = 0; i < seg.ntiles && ok; ++i) {
           const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
           if (lane == 0 && i + 1 < seg.ntiles) {  // next tile's latent rows toward L2
@@ -248,6 +264,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (nr > 0)
               prefetch_l2(static_cast<const __nv_bfloat16*>(a.kc) + r0 * lt.Rk, (uint32_t)(nr * lt.Rk * 2));
           }
+          int n = 0;  // factor item index inside the tile
           for (int g = 0; g < lt.G && ok; ++g) {
             const GroupSm& gs = sm.grp[g];
             const int np = gs.np;
@@ -266,43 +283,70 @@ __global__ void __launch_bounds__(kThreads, 1)
               a_cnt += nb;
               p0 += nb;
             }
+            if (kMma == 2)
+              for (int u = 0; u < gs.nu && ok; ++u, ++kc, n += np) {
+                if ((kc & 1) != 1) continue;  // MMA thread 0's unit
+                if (!images_ready) {          // the images are written by the preparation kernel
+                  griddep_wait();
+                  images_ready = true;
+                }
+                ok = put_unit_items(1, wc, n, np, img, pol_w);
+              }
           }
         }
       }
     }
   } else if (warp == 10) {
-    // ---- factor items: several bulk copies per instruction ------------------
+    // ---- factor items: several bulk copies per instruction (query-folded
+    // mode: the ring of MMA thread 0 only) --------------------------------------
     if (x0 < x1) {
       const uint64_t pol = policy_evict_last();
       griddep_wait();  // the images are written by the preparation kernel
       int w_cnt = 0;
       bool ok = true;
+      int wc = 0, kc = 0;  // items put into MMA thread 0's ring, units so far
       while (ok && walk.next(a, seg)) {
         const uint8_t* img = ta.fimg + (kFold ? (int64_t)seg.b * ta.fimg_seq_bytes : 0);
         for (int i = 0; i < seg.ntiles && ok; ++i) {
-          for (int n0 = 0; n0 < ta.n_items && ok;) {
-            const int nb = claim_slots(sm.w_empty, NW, w_cnt, min(NW, ta.n_items - n0), lane, abort_flag);
-            ok = nb > 0;
-            if (!ok) break;
-            if (lane < nb) {
-              const int sl = (w_cnt + lane) % NW;
-              const uint32_t it = sm.item[n0 + lane];
-              const uint32_t bytes = (it >> 26) << 12;
-              mbar_expect_tx(&sm.w_full[sl], bytes);
-              bulk_load(sm.w[sl], img + (it & 0x03FFFFFFu), bytes, &sm.w_full[sl], pol);
+          if (kMma == 1) {  // one ring: claims may span units
+            for (int n0 = 0; n0 < ta.n_items && ok;) {
+              const int nb = claim_slots(sm.w_empty, NW, w_cnt, min(NW, ta.n_items - n0), lane, abort_flag);
+              ok = nb > 0;
+              if (!ok) break;
+              if (lane < nb) {
+                const int sl = (w_cnt + lane) % NW;
+                const uint32_t it = sm.item[n0 + lane];
+                const uint32_t bytes = (it >> 26) << 12;
+                mbar_expect_tx(&sm.w_full[sl], bytes);
+                bulk_load(sm.w[sl], img + (it & 0x03FFFFFFu), bytes, &sm.w_full[sl], pol);
+              }
+              __syncwarp();
+              w_cnt += nb;
+              n0 += nb;
             }
-            __syncwarp();
-            w_cnt += nb;
-            n0 += nb;
+            continue;
+          }
+          int n = 0;
+          for (int g = 0; g < lt.G && ok; ++g) {
+            const int np = sm.grp[g].np, nu = sm.grp[g].nu;
+            for (int u = 0; u < nu && ok; ++u, ++kc, n += np)
+              if ((kc & 1) == 0) ok = put_unit_items(0, wc, n, np, img, pol);
           }
         }
       }
     }
-  } else if (warp == 1) {
-    // ---- MMA issuer: one thread runs the whole schedule (warp-wide
-    // bookkeeping would only lengthen the path between MMAs) ----------------
+  } else if (warp == 1 || (kMma == 2 && warp == 11)) {
+    // ---- MMA issuers: lane 0 of warp 1 (and of warp 11 in query-folded mode)
+    // runs the schedule of every kMma-th unit into its own accumulator, so one
+    // thread's barrier tests and commits overlap the other's MMAs.  Each thread
+    // owns a factor ring (single consumer) and observes every latent piece's
+    // fill in order, releasing the pieces of groups it has no unit in, so no
+    // parity test can see a stale phase. ---------------------------------------
     if (lane == 0 && x0 < x1) {
-      int a_cnt = 0, w_cnt = 0, kc = 0;
+      const int t = warp == 1 ? 0 : 1;
+      uint64_t* wfull = sm.w_full + t * NWt;
+      uint64_t* wempty = sm.w_empty + t * NWt;
+      int a_cnt = 0, w_cnt = 0, kc = 0, own = 0;
       bool ok = true;
       while (ok && walk.next(a, seg)) {
         for (int i = 0; i < seg.ntiles && ok; ++i) {
@@ -310,56 +354,74 @@ __global__ void __launch_bounds__(kThreads, 1)
             const GroupSm& gs = sm.grp[g];
             const int np = gs.np, nu = gs.nu;
             const int a_base = a_cnt;
-            for (int u = 0; u < nu && ok; ++u) {
+            const int uf = kMma == 2 ? (((kc & 1) == t) ? 0 : 1) : 0;  // this thread's first unit of the group
+            if (uf >= nu)  // none: observe the group's pieces, then release them
+              for (int p = 0; p < np && ok; ++p) {
+                const int sl = (a_base + p) % kNA;
+                if ((ok = mbar_wait(&sm.a_full[sl], ((a_base + p) / kNA) & 1, abort_flag))) mbar_arrive(&sm.a_empty[sl]);
+              }
+            for (int u = uf; u < nu && ok; u += kMma) {
               const int nh = min(2, gs.nh - 2 * u);
               const uint32_t idesc_k = idesc_bf16(128, kD * nh, false, true);
-              const int buf = kc & 1;
-              if (kc >= 2) {  // the epilogue has read this buffer's previous unit
-                if (!(ok = mbar_wait(&sm.k_empty[buf], ((kc >> 1) - 1) & 1, abort_flag))) break;
-                tc_fence_after();
-              }
-              DCK_TC_TRACE(10);
-              // readiness of this unit's factor items (and, first unit of the group,
-              // latent pieces): independent tests whose latencies overlap; blocking
-              // waits, in ring order, only for what is not there yet.  Only items
-              // within one turn of the ring are tested: the previous use of their
-              // slot has been consumed, so the parity test cannot see a stale phase
-              // (an item a full turn ahead shares its slot with one still in flight).
+              const int kg = kc + u;                               // unit index of the CTA
+              const int buf = kMma == 2 ? t : (kg & 1);
+              const int use = kMma == 2 ? own : (kg >> 1);         // earlier units in this accumulator
+              // readiness of this unit's factor items (and, at this thread's first
+              // unit of the group, latent pieces): independent tests whose latencies
+              // overlap; blocking waits, in ring order, only for what is not there
+              // yet.  Only items within one turn of the ring are tested: the previous
+              // use of their slot has been consumed, so the parity test cannot see a
+              // stale phase.
               uint32_t miss = 0;
 #pragma unroll
               for (int p = 0; p < kMaxPieces; ++p)
                 if (p < np) {
                   const int c = w_cnt + p;
-                  if (p >= NW || !mbar_test(&sm.w_full[c % NW], (c / NW) & 1)) miss |= 1u << p;
-                  if (u == 0 && !mbar_test(&sm.a_full[(a_base + p) % kNA], ((a_base + p) / kNA) & 1))
+                  if (p >= NWt || !mbar_test(&wfull[c % NWt], (c / NWt) & 1)) miss |= 1u << p;
+                  if (u == uf && !mbar_test(&sm.a_full[(a_base + p) % kNA], ((a_base + p) / kNA) & 1))
                     miss |= 0x100u << p;
                 }
+              // the first piece and item before the accumulator: the operand streams do
+              // not depend on the epilogue, so the MMAs can start as soon as it is free
+              if ((miss & 0x100u) && !(ok = mbar_wait(&sm.a_full[a_base % kNA], (a_base / kNA) & 1, abort_flag))) break;
+              if ((miss & 1u) && !(ok = mbar_wait(&wfull[w_cnt % NWt], (w_cnt / NWt) & 1, abort_flag))) break;
+              miss &= ~0x101u;
+              DCK_TC_TRACE(12);
+              if (use >= 1) {  // the epilogue has read this accumulator's previous unit
+                if (!(ok = mbar_wait(&sm.k_empty[buf], (use - 1) & 1, abort_flag))) break;
+                tc_fence_after();
+              }
+              DCK_TC_TRACE(10);
               const uint32_t dcol = tmem + buf * kKCols;
+              const bool last = u + kMma >= nu;  // this thread's last unit of the group
               for (int p = 0; p < np; ++p) {
                 const int asl = (a_base + p) % kNA;
-                const int wsl = w_cnt % NW;
+                const int wsl = w_cnt % NWt;
                 if (((miss >> (8 + p)) & 1) && !(ok = mbar_wait(&sm.a_full[asl], ((a_base + p) / kNA) & 1, abort_flag)))
                   break;
-                if (((miss >> p) & 1) && !(ok = mbar_wait(&sm.w_full[wsl], (w_cnt / NW) & 1, abort_flag))) break;
+                if (((miss >> p) & 1) && !(ok = mbar_wait(&wfull[wsl], (w_cnt / NWt) & 1, abort_flag))) break;
+                DCK_TC_TRACE(13);
                 const int w = gs.w[p];
                 const uint32_t ab0 = smem_u32(sm.a[asl]);
-                const uint32_t bb = smem_u32(sm.w[wsl]);
+                const uint32_t bb = smem_u32(sm.w[t * NWt + wsl]);
                 const uint32_t swz = swz_of(w);
                 for (int k = 0; k < w / 16; ++k) {
                   const uint64_t ad = sdesc(ab0 + k * 32, 16, 16 * w, swz);
                   const uint64_t bd = sdesc(bb + k * 2048, 128 * w, 1024, kSw128);
                   umma_f16(dcol, ad, bd, idesc_k, (p > 0 || k > 0) ? 1u : 0u);
                 }
-                umma_commit(&sm.w_empty[wsl]);
-                if (u == nu - 1) umma_commit(&sm.a_empty[asl]);  // last unit of the group: piece done
+                umma_commit(&wempty[wsl]);
+                if (last) umma_commit(&sm.a_empty[asl]);  // this thread is done with the piece
+                DCK_TC_TRACE(14);
                 ++w_cnt;
               }
               if (!ok) break;
               umma_commit(&sm.k_full[buf]);
               DCK_TC_TRACE(11);
-              ++kc;
+              ++own;
             }
             a_cnt += np;
+            kc += nu;
           }
         }
       }
@@ -372,10 +434,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int hf = (warp - 2) >> 2;      // frequency half, then head half
     const int tau = quad * 32 + lane;    // token row inside the tile
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
-    const bool storer = e == 0;          // issues the per-tile bulk store of P (warp 2, lane 0)
-    int kc = 0, tl = 0, round = 0;
+    // tile and segment ends: thread e owns head jt and the 16 tokens [16 ct, 16 ct + 16)
+    // of every tile; the 8 owners of a head are adjacent lanes of one warp
+    const int jt = e >> 3, ct = e & 7;
+    int kc = 0, round = 0;
     bool ok = true;
-    const int jb0 = 16 * hf;  // heads owned at tile and segment ends
 #define EPI_SYNC()                                  \
   do {                                              \
     __syncwarp();                                   \
@@ -400,8 +463,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           sm.qr[j * kD + pi + kD / 2] = (x1v * sn + x2v * cs) * qscale;
         }
       }
-      // reference maxima start at -inf: the buffer a tile end reads is that of tile tl - 1
-      if (quad == 0 && lane < 16 && jb0 + lane < Hq) sm.mref[(tl - 1) & 1][jb0 + lane] = -INFINITY;
       // RoPE angle of token t0+tau and pair p: (t0*w_p mod 2pi, fp64) + tau*w_p (fp32);
       // the offsets beta of later tiles are written at the previous tile's end
       if (e < kD / 2) {
@@ -410,12 +471,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       EPI_SYNC();
       if (!ok) break;
-      // running row sums: one per (quadrant, head), kept by the warp owning both
-      if (lane < 16 && jb0 + lane < Hq) sm.redl[quad][jb0 + lane] = 0.f;
+      // head jt's reference max (log2 units; the same in all 8 owners) and this
+      // owner's share of its row sum, rescaled whenever the reference moves
+      float m_run = -INFINITY, l_part = 0.f;
       for (int i = 0; i < seg.ntiles && ok; ++i) {
         const int t0 = seg.t_begin + kTile * i;
         const int64_t x = seg.x0 + i;  // flattened tile index
-        const bool valid = t0 + tau < seg.t_end;
         float cs[32], sn[32];
 #pragma unroll
         for (int ip = 0; ip < 32; ++ip) {
@@ -433,30 +494,41 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!(ok = wwait(&sm.k_full[buf], (kc >> 1) & 1, abort_flag))) break;
             tc_fence_after();
             DCK_TC_TRACE(20);
-            for (int hh = 0; hh < nh; ++hh) {
-              const int j0 = sm.order[gs.h0 + 2 * u + hh] * qpg;
-              const uint32_t cb = tmem + lane_base + buf * kKCols + hh * kD;
-              const bool last = hh == nh - 1;
-              if (kFold) {
-                // Y columns [64 hf, 64 hf + 64): pairs (2i, 2i+1) of my 32 frequencies,
-                // read in two passes of 16 pairs to keep the register footprint small
-                float pa[4] = {0.f, 0.f, 0.f, 0.f};  // independent chains
+            if (kFold) {
+              // Y columns [64 hf, 64 hf + 64) of both heads: pairs (2i, 2i+1) of my 32
+              // frequencies, in two passes of 16 pairs; each pass loads both heads
+              // before its one wait, so a unit costs two TMEM round trips
+              const uint32_t cb = tmem + lane_base + buf * kKCols + 64 * hf;
+              float pa[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};  // independent chains
 #pragma unroll
-                for (int ps = 0; ps < 2; ++ps) {
-                  float y[32];
-                  tmem_ld32(cb + 64 * hf + 32 * ps, y);
-                  tmem_wait_ld();
-                  if (last && ps == 1) {
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
-                  }
+              for (int ps = 0; ps < 2; ++ps) {
+                float y0[32], y1[32];
+                tmem_ld32(cb + 32 * ps, y0);
+                if (nh == 2) tmem_ld32(cb + kD + 32 * ps, y1);
+                tmem_wait_ld();
+                DCK_TC_TRACE(43 + ps);
+                if (ps == 1) {
+                  tc_fence_before();
+                  __syncwarp();
+                  if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
+                }
+#pragma unroll
+                for (int i2 = 0; i2 < 16; ++i2)
+                  pa[0][i2 & 3] = fmaf(cs[16 * ps + i2], y0[2 * i2], fmaf(sn[16 * ps + i2], y0[2 * i2 + 1], pa[0][i2 & 3]));
+                if (nh == 2)
 #pragma unroll
                   for (int i2 = 0; i2 < 16; ++i2)
-                    pa[i2 & 3] = fmaf(cs[16 * ps + i2], y[2 * i2], fmaf(sn[16 * ps + i2], y[2 * i2 + 1], pa[i2 & 3]));
-                }
-                atomicAdd(&sm.x[j0 * 128 + tau], (pa[0] + pa[1]) + (pa[2] + pa[3]));
-              } else {
+                    pa[1][i2 & 3] =
+                        fmaf(cs[16 * ps + i2], y1[2 * i2], fmaf(sn[16 * ps + i2], y1[2 * i2 + 1], pa[1][i2 & 3]));
+              }
+              atomicAdd(&sm.x[sm.order[gs.h0 + 2 * u] * 128 + tau], (pa[0][0] + pa[0][1]) + (pa[0][2] + pa[0][3]));
+              if (nh == 2)
+                atomicAdd(&sm.x[sm.order[gs.h0 + 2 * u + 1] * 128 + tau], (pa[1][0] + pa[1][1]) + (pa[1][2] + pa[1][3]));
+            } else {
+              for (int hh = 0; hh < nh; ++hh) {
+                const int j0 = sm.order[gs.h0 + 2 * u + hh] * qpg;
+                const uint32_t cb = tmem + lane_base + buf * kKCols + hh * kD;
+                const bool last = hh == nh - 1;
                 // two passes of 16 frequency pairs keep the register footprint small
                 float part[kMaxQPerKv];
 #pragma unroll
@@ -494,115 +566,79 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!ok) break;
         // ---- tile end: reference max, P ------------------------------------
-        // Heads [jb, jb + 16) belong to this warp here (none for hf = 1 when
-        // Hq <= 16); every per-head step runs over all 16 at once so that the
-        // shared-memory and shuffle latencies overlap.
         DCK_TC_TRACE(22);
         EPI_SYNC();  // every partial score of the tile is in x
         if (!ok) break;
-        const int jb = jb0;
-        const int nh = max(0, min(16, Hq - jb));
-        float sc[16], mx[16];
-#pragma unroll
-        for (int u = 0; u < 16; ++u) sc[u] = (u < nh && valid) ? sm.x[(jb + u) * 128 + tau] : -INFINITY;
-#pragma unroll
-        for (int u = 0; u < 16; ++u)
-          if (u < nh) sm.x[(jb + u) * 128 + tau] = 0.f;  // ready for the next tile
-#pragma unroll
-        for (int u = 0; u < 16; ++u) mx[u] = sc[u];
-#pragma unroll
-        for (int o = 16; o; o >>= 1)
-#pragma unroll
-          for (int u = 0; u < 16; ++u) mx[u] = fmaxf(mx[u], __shfl_xor_sync(0xffffffffu, mx[u], o));
         {
-          float v = mx[0];
+          const bool own = jt < Hq;
+          const int tb = 16 * ct;  // first token of this owner
+          float sc[16];
+          float4* xr = reinterpret_cast<float4*>(&sm.x[jt * 128 + tb]);
 #pragma unroll
-          for (int u = 1; u < 16; ++u) v = lane == u ? mx[u] : v;
-          if (lane < nh) sm.redm[quad][jb + lane] = v;
+          for (int q = 0; q < 4; ++q) {
+            const float4 v = own ? xr[q] : make_float4(0.f, 0.f, 0.f, 0.f);
+            sc[4 * q] = v.x;
+            sc[4 * q + 1] = v.y;
+            sc[4 * q + 2] = v.z;
+            sc[4 * q + 3] = v.w;
+            if (own) xr[q] = make_float4(0.f, 0.f, 0.f, 0.f);  // ready for the next tile
+          }
+          const int nv = max(0, min(16, seg.t_end - (t0 + tb)));  // tokens inside the sequence
+          float mx = -INFINITY;
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            if (k >= nv || !own) sc[k] = -INFINITY;
+            mx = fmaxf(mx, sc[k]);
+          }
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+          // the reference moves only when the tile's max exceeds it by the threshold
+          if (own && (m_run == -INFINITY || mx > m_run + kRescaleThr)) {
+            l_part *= exp2f(m_run - mx);
+            m_run = mx;
+          }
+          if (own && ct == 0) ta.mglob[x * Hq + jt] = m_run;
+          // probabilities (bf16, the absorption's operand) straight into this tile's
+          // P image; the row sum uses the rounded values
+          uint32_t pk[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const __nv_bfloat162 pv = __floats2bfloat162_rn(own ? exp2f(sc[2 * k] - m_run) : 0.f,
+                                                            own ? exp2f(sc[2 * k + 1] - m_run) : 0.f);
+            const float2 pf = __bfloat1622float2(pv);
+            l_part += pf.x + pf.y;
+            pk[k] = *reinterpret_cast<const uint32_t*>(&pv);
+          }
+          if (jt < hq_pad) {  // padded heads get zero rows
+            // image: [token atom (64)][head row][64 tokens], 128B rows, 16-byte chunks swizzled by row % 8
+            uint8_t* img = ta.pglob + x * (hq_pad * 256) + (tb >> 6) * (hq_pad * 128) + (jt >> 3) * 1024 +
+                           (jt & 7) * 128;
+            const int ch = (tb & 63) >> 3;
+            *reinterpret_cast<uint4*>(img + ((ch ^ (jt & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            *reinterpret_cast<uint4*>(img + (((ch + 1) ^ (jt & 7)) << 4)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          }
         }
         if (e < kD / 2 && i + 1 < seg.ntiles) {  // RoPE phase offsets of the next tile
           const double ang = (double)(t0 + kTile) * sm.om64[e];
           sm.beta[e] = (float)(ang - 6.283185307179586 * floor(ang * 0.15915494309189535));
         }
-        if (storer) bulk_store_wait_read();  // the previous tile's P image has left shared memory
-        EPI_SYNC();  // per-quadrant maxima are in redm; the P image may be rewritten
-        DCK_TC_TRACE(28);
-        if (!ok) break;
-        float al[16], mr[16];  // rescale factors of the row sums, reference maxima after this tile
-        {
-          float tm[16];
-#pragma unroll
-          for (int u = 0; u < 16; ++u) {
-            tm[u] = u < nh ? fmaxf(fmaxf(sm.redm[0][jb + u], sm.redm[1][jb + u]),
-                                   fmaxf(sm.redm[2][jb + u], sm.redm[3][jb + u]))
-                           : -INFINITY;
-            mr[u] = u < nh ? sm.mref[(tl - 1) & 1][jb + u] : 0.f;
-          }
-#pragma unroll
-          for (int u = 0; u < 16; ++u) {
-            al[u] = 1.f;
-            if (u < nh && (mr[u] == -INFINITY || tm[u] > mr[u] + kRescaleThr)) {
-              al[u] = exp2f(mr[u] - tm[u]);
-              mr[u] = tm[u];
-            }
-          }
-          float v = mr[0];
-#pragma unroll
-          for (int u = 1; u < 16; ++u) v = lane == u ? mr[u] : v;
-          if (quad == 0 && lane < nh) {
-            sm.mref[tl & 1][jb + lane] = v;
-            ta.mglob[x * Hq + jb + lane] = v;
-          }
-        }
-        // probabilities -> P image (bf16); row sums use the rounded values
-        float ps[16];
-#pragma unroll
-        for (int u = 0; u < 16; ++u) {
-          const __nv_bfloat16 pv = __float2bfloat16_rn(exp2f(sc[u] - mr[u]));
-          if (u < nh) *reinterpret_cast<__nv_bfloat16*>(sm.p + p_off(jb + u, tau, hq_pad)) = pv;
-          ps[u] = u < nh ? __bfloat162float(pv) : 0.f;
-        }
-        fence_proxy_async_smem();  // the bulk store reads the image through the async proxy
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.p_done);
-#pragma unroll
-        for (int o = 16; o; o >>= 1)
-#pragma unroll
-          for (int u = 0; u < 16; ++u) ps[u] += __shfl_xor_sync(0xffffffffu, ps[u], o);
-        {
-          float v = ps[0], a1 = al[0];
-#pragma unroll
-          for (int u = 1; u < 16; ++u) {
-            v = lane == u ? ps[u] : v;
-            a1 = lane == u ? al[u] : a1;
-          }
-          if (lane < nh) sm.redl[quad][jb + lane] = fmaf(sm.redl[quad][jb + lane], a1, v);
-        }
-        if (warp == 2) {  // the whole warp takes the decision, lane 0 issues the store
-          bool r = true;
-          if (storer) r = mbar_wait(&sm.p_done, tl & 1, abort_flag);
-          if (!(ok = __shfl_sync(0xffffffffu, r ? 1 : 0, 0) != 0)) break;
-          if (storer) bulk_store(ta.pglob + x * (hq_pad * 256), sm.p, (uint32_t)(hq_pad * 256));
-          __syncwarp();
-        }
         DCK_TC_TRACE(23);
-        ++tl;
+        EPI_SYNC();  // x is clear and the next tile's phase offsets are in place
+        if (!ok) break;
       }
       if (!ok) break;
-      // ---- segment end: reference max and row sums -> partial slot c + b -----
-      EPI_SYNC();
-      if (!ok) break;
-      const int64_t slot = (int64_t)blockIdx.x + seg.b;
-      if (quad == 0) {
-        const int j = jb0 + lane;
-        if (lane < 16 && j < Hq) {
-          a.part_ml[(slot * Hq + j) * 2] = sm.mref[(tl - 1) & 1][j];
-          a.part_ml[(slot * Hq + j) * 2 + 1] = sm.redl[0][j] + sm.redl[1][j] + sm.redl[2][j] + sm.redl[3][j];
-        }
+      // ---- segment end: reference max and row sum -> partial slot c + b -------
+      l_part += __shfl_xor_sync(0xffffffffu, l_part, 1);
+      l_part += __shfl_xor_sync(0xffffffffu, l_part, 2);
+      l_part += __shfl_xor_sync(0xffffffffu, l_part, 4);
+      if (jt < Hq && ct == 0) {
+        const int64_t slot = (int64_t)blockIdx.x + seg.b;
+        a.part_ml[(slot * Hq + jt) * 2] = m_run;
+        a.part_ml[(slot * Hq + jt) * 2 + 1] = l_part;
       }
     }
 #undef EPI_SYNC
-    if (storer) bulk_store_wait();  // P images written before the absorption kernel reads them
   }
   tc_fence_before();
   __syncthreads();
@@ -775,7 +811,7 @@ cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& m
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.n_items);
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(Ring<kFold>::kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
