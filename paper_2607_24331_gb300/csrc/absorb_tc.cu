@@ -45,7 +45,7 @@ using namespace tc;
 
 constexpr int kAThreads = 192;
 constexpr int kVSlot = 16384;  // [128 tokens][64 rv] bf16, 128B-swizzled: one half of an r_v chunk
-constexpr int kNVs = 8;        // value slots: four chunks in flight
+constexpr int kNVs = 12;       // value slots: six chunks in flight
 constexpr int kPSlot = 8192;   // P image of one tile (Hq_pad <= 32)
 constexpr int kNP = 2;
 constexpr uint32_t kTmemCols = 512;
@@ -67,6 +67,7 @@ struct ASmem {
   uint8_t p[kNP][kPSlot];
   uint64_t v_full[kNVs], v_empty[kNVs], p_full[kNP], p_empty[kNP];
   uint64_t drain, tile_ok, u_ready, u_free;
+  int pneed[kNP];  // P slot's tile raises some head's reference max (set by the producer before the slot fills)
   int scan[kAThreads];
   uint32_t tmem_base;
   int abort_flag;
@@ -116,29 +117,61 @@ __global__ void __launch_bounds__(kAThreads, 1)
 
   if (warp == 0) {
     // ---- producer ------------------------------------------------------------
+    // The value latents do not depend on the scores kernel, which may still be
+    // running (programmatic dependent launch): the first tile's rows are
+    // prefetched and its first chunks loaded before the wait for that kernel's
+    // probabilities and maxima.
     if (x0 < x1) {
       const uint64_t pol = policy_evict_first();
-      int v_cnt = 0, p_cnt = 0;
-      bool ok = true;
+      int v_cnt = 0, p_cnt = 0, c_pre = 0;
+      bool ok = true, first = true;
       while (ok && walk.next(a, seg)) {
         for (int i = 0; i < seg.ntiles && ok; ++i) {
           const int64_t x = seg.x0 + i;
           const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
-          if (lane == 0 && i + 1 < seg.ntiles) {  // next tile's value rows toward L2
-            const int64_t r0 = yrow + kTile, nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
-            if (nr > 0)
-              prefetch_l2(static_cast<const __nv_bfloat16*>(a.vc) + r0 * lt.rv, (uint32_t)(nr * lt.rv * 2));
+          if (lane == 0) {  // this CTA's first tile, then each next tile, toward L2
+            for (int q = first ? 0 : 1; q < 2; ++q) {
+              if (q == 1 && i + 1 >= seg.ntiles) break;
+              const int64_t r0 = yrow + kTile * q, nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
+              if (nr > 0)
+                prefetch_l2(static_cast<const __nv_bfloat16*>(a.vc) + r0 * lt.rv, (uint32_t)(nr * lt.rv * 2));
+            }
+          }
+          if (first) {  // chunks that fit the empty ring, ahead of the wait
+            c_pre = min(n_chunks, kNVs / 2);
+            for (int c = 0; c < c_pre; ++c) {
+              if (lane < 2) {
+                const int sl = (v_cnt + lane) % kNVs;
+                mbar_expect_tx(&sm.v_full[sl], kVSlot);
+                tma_load_2d_hint(sm.v[sl], &maps.vc, &sm.v_full[sl], 128 * c + 64 * lane, (int32_t)yrow, pol);
+              }
+              __syncwarp();
+              v_cnt += 2;
+            }
+            griddep_wait();
+            first = false;
           }
           if (!(ok = wait_slots(sm.p_empty, kNP, p_cnt, 1, lane, abort_flag))) break;
-          if (lane == 0) {
-            const int sl = p_cnt % kNP;
-            mbar_expect_tx(&sm.p_full[sl], pbytes);
-            bulk_load(sm.p[sl], aa.pglob + x * pbytes, pbytes, &sm.p_full[sl], pol);
+          {
+            // does any head's reference max rise at this tile?  (decided here, once,
+            // for the MMA thread; the epilogue warps take the same decision)
+            bool need = false;
+            if (i > 0) {
+              const float mn = lane < Hq ? aa.mglob[x * Hq + lane] : 0.f;
+              const float mo = lane < Hq ? aa.mglob[(x - 1) * Hq + lane] : 0.f;
+              need = __any_sync(0xffffffffu, mn > mo);
+            }
+            if (lane == 0) {
+              const int sl = p_cnt % kNP;
+              sm.pneed[sl] = need ? 1 : 0;
+              mbar_expect_tx(&sm.p_full[sl], pbytes);
+              bulk_load(sm.p[sl], aa.pglob + x * pbytes, pbytes, &sm.p_full[sl], pol);
+            }
           }
           __syncwarp();
           DCK_AB_TRACE(1);
           ++p_cnt;
-          for (int c = 0; c < n_chunks && ok; ++c) {
+          for (int c = c_pre; c < n_chunks && ok; ++c) {
             if (!(ok = wait_slots(sm.v_empty, kNVs, v_cnt, 2, lane, abort_flag))) break;
             if (lane < 2) {
               const int sl = (v_cnt + lane) % kNVs;
@@ -149,6 +182,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
             DCK_AB_TRACE(2);
             v_cnt += 2;
           }
+          c_pre = 0;
         }
       }
     }
@@ -160,14 +194,13 @@ __global__ void __launch_bounds__(kAThreads, 1)
       bool ok = true;
       while (ok && walk.next(a, seg)) {
         for (int i = 0; i < seg.ntiles && ok; ++i) {
+          const int psl = p_cnt % kNP;
+          if (!(ok = mbar_wait(&sm.p_full[psl], (p_cnt / kNP) & 1, abort_flag))) break;
           if (i > 0) {
-            // did any head's reference max rise at this tile?  Then the epilogue
-            // rescales U once the earlier tiles' MMAs are done (drain) and
-            // releases this tile (tile_ok).
-            const int64_t x = seg.x0 + i;
-            bool need = false;
-            for (int j = 0; j < Hq; ++j) need |= aa.mglob[x * Hq + j] > aa.mglob[(x - 1) * Hq + j];
-            if (need) {
+            // some head's reference max rises at this tile: the epilogue rescales U
+            // once the earlier tiles' MMAs are done (drain) and releases this tile
+            // (tile_ok)
+            if (sm.pneed[psl]) {
               umma_commit(&sm.drain);
               if (!(ok = mbar_wait(&sm.tile_ok, rc & 1, abort_flag))) break;
               tc_fence_after();
@@ -178,36 +211,42 @@ __global__ void __launch_bounds__(kAThreads, 1)
             if (!(ok = mbar_wait(&sm.u_free, (sgc - 1) & 1, abort_flag))) break;
             tc_fence_after();
           }
-          const int psl = p_cnt % kNP;
-          if (!(ok = mbar_wait(&sm.p_full[psl], (p_cnt / kNP) & 1, abort_flag))) break;
           DCK_AB_TRACE(11);
           const int nvalid = i == seg.ntiles - 1 ? seg.t_end - (seg.t_begin + kTile * i) : kTile;
           const uint32_t pbase = smem_u32(sm.p[psl]);
-          for (int c = 0; c < n_chunks && ok; ++c) {
-            const int sl = v_cnt % kNVs;  // even: the chunk's halves are adjacent slots
-            const uint32_t vpar = (v_cnt / kNVs) & 1;
-            if (!(ok = mbar_wait(&sm.v_full[sl], vpar, abort_flag))) break;
-            if (!(ok = mbar_wait(&sm.v_full[sl + 1], vpar, abort_flag))) break;
-            if (nvalid < kTile) {  // rows past the sequence end: exact zeros
-              for (int r = nvalid; r < kTile; ++r)
+          // chunks in pairs: the K = 16 MMAs of one chunk form a dependent chain on
+          // its accumulator (about 120 cycles each at N = Hq_pad), so two chunks'
+          // chains are interleaved
+          for (int c = 0; c < n_chunks && ok; c += 2) {
+            const int nc = min(2, n_chunks - c);
+            uint32_t vb[2] = {0u, 0u};
+            for (int q = 0; q < nc && ok; ++q) {
+              const int sl = (v_cnt + 2 * q) % kNVs;  // even: the chunk's halves are adjacent slots
+              const uint32_t vpar = ((v_cnt + 2 * q) / kNVs) & 1;
+              if (!(ok = mbar_wait(&sm.v_full[sl], vpar, abort_flag))) break;
+              if (!(ok = mbar_wait(&sm.v_full[sl + 1], vpar, abort_flag))) break;
+              if (nvalid < kTile) {  // rows past the sequence end: exact zeros
+                for (int r = nvalid; r < kTile; ++r)
 #pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                  reinterpret_cast<uint4*>(sm.v[sl] + r * 128)[q] = make_uint4(0, 0, 0, 0);
-                  reinterpret_cast<uint4*>(sm.v[sl + 1] + r * 128)[q] = make_uint4(0, 0, 0, 0);
-                }
-              fence_proxy_async_smem();
+                  for (int w = 0; w < 8; ++w) {
+                    reinterpret_cast<uint4*>(sm.v[sl] + r * 128)[w] = make_uint4(0, 0, 0, 0);
+                    reinterpret_cast<uint4*>(sm.v[sl + 1] + r * 128)[w] = make_uint4(0, 0, 0, 0);
+                  }
+                fence_proxy_async_smem();
+              }
+              vb[q] = smem_u32(sm.v[sl]);
             }
-            const uint32_t vb = smem_u32(sm.v[sl]);
+            if (!ok) break;
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
-              const uint64_t ad = sdesc(vb + k * 2048, kVSlot, 1024, kSw128);
               const uint64_t bd = sdesc(pbase + (k >> 2) * (hq_pad * 128) + (k & 3) * 32, 16, 1024, kSw128);
-              umma_f16(tmem + c * hq_pad, ad, bd, idesc_v, (i == 0 && k == 0) ? 0u : 1u);
+              for (int q = 0; q < nc; ++q)
+                umma_f16(tmem + (c + q) * hq_pad, sdesc(vb[q] + k * 2048, kVSlot, 1024, kSw128), bd, idesc_v,
+                         (i == 0 && k == 0) ? 0u : 1u);
             }
-            umma_commit(&sm.v_empty[sl]);
-            umma_commit(&sm.v_empty[sl + 1]);
+            for (int q = 0; q < 2 * nc; ++q) umma_commit(&sm.v_empty[(v_cnt + q) % kNVs]);
             DCK_AB_TRACE(12);
-            v_cnt += 2;
+            v_cnt += 2 * nc;
           }
           if (!ok) break;
           umma_commit(&sm.p_empty[psl]);
@@ -227,6 +266,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     int rc = 0, sgc = 0;
     bool ok = true;
+    griddep_wait();  // the maxima come from the scores kernel
     while (ok && walk.next(a, seg)) {
       for (int i = 1; i < seg.ntiles && ok; ++i) {
         const int64_t x = seg.x0 + i;
@@ -349,8 +389,20 @@ cudaError_t launch_absorb_tc(const LayerTable& lt, const DecodeArgs& a, const Tc
     if (e != cudaSuccess) return e;
     if (dev_ok) attr_done[dev] = 1;
   }
-  absorb_tc_kernel<<<a.n_items, kAThreads, smem, s>>>(maps, lt, a, aa);
-  return cudaGetLastError();
+  // programmatic dependent launch: CTAs start streaming value latents as the
+  // scores kernel's CTAs finish; the kernel waits for that grid before reading
+  // its outputs
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.n_items);
+  cfg.blockDim = dim3(kAThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, absorb_tc_kernel, maps, lt, a, aa);
 }
 
 }  // namespace dck

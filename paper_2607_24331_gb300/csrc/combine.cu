@@ -13,10 +13,11 @@
 // rows as fit kMaxRows, so each head's B_v block is staged about once.
 // CTA `rank` of a cluster owns rows [rank*rv/split, (rank+1)*rv/split) of u
 // and of B_v's column block: it merges those rows of every (sequence, query
-// head) row of its chunk (eight items' loads in flight at a time), stages its
-// B_v rows in shared memory with cp.async (all issued up front), and forms the
-// partial product over its rows.  The cluster adds the partial outputs through
-// distributed shared memory and rank 0 writes o.
+// head) row of its chunk in one pass with a running max (sixteen items' loads in
+// flight at a time), stages its B_v rows in shared memory with cp.async (all
+// issued up front), and forms the partial product over its rows, each output
+// owned by one thread.  The cluster adds the partial outputs through
+// distributed shared memory, every rank reducing and writing a share of o.
 #include <algorithm>
 
 #include <cooperative_groups.h>
@@ -31,7 +32,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kMaxSplit = 8;    // CTAs per cluster (r_v split), portable cluster size
 constexpr int kMaxRows = 16;    // (sequence, query head) rows per cluster
-constexpr int kItemBatch = 8;   // partial items whose loads are in flight together
+constexpr int kItemBatch = 16;  // partial items whose loads are in flight together
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)),
@@ -40,6 +41,12 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
+// Two adjacent elements (16-byte aligned row, even column) as floats.
+__device__ __forceinline__ float2 pair_f32(const float* p) { return *reinterpret_cast<const float2*>(p); }
+__device__ __forceinline__ float2 pair_f32(const __nv_bfloat16* p) {
+  return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(p));
+}
 
 template <typename T, int D>
 __global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, const DecodeArgs a, int bchunk,
@@ -56,14 +63,16 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, 
   const int rr = rv / split;            // rows of u / B_v owned by this CTA (a multiple of 4)
   const int r0 = rank * rr;
 
-  // shared layout: B_v rows [rr][D] T | u rows [kMaxRows][rr] | partial o [kMaxRows][D] | m, 1/l | scan | prefix
+  // shared layout: B_v rows [rr][D] T | u rows [kMaxRows][rr] | received partial o [split][kMaxRows * D / split]
+  // | 1/l | row item ranges [kMaxRows][2] | scan | prefix | item starts [n_items + 1]
   T* sbv = reinterpret_cast<T*>(smem_c);
   float* su = reinterpret_cast<float*>(smem_c + (size_t)rr * D * sizeof(T));
   float* so = su + (size_t)kMaxRows * rr;
-  float* sM = so + kMaxRows * D;
-  float* sinv = sM + kMaxRows;
-  int* scan = reinterpret_cast<int*>(sinv + kMaxRows);
+  float* sinv = so + kMaxRows * D;
+  int* rc = reinterpret_cast<int*>(sinv + kMaxRows);
+  int* scan = rc + 2 * kMaxRows;
   int* prefix = scan + kThreads;
+  int* ibeg = prefix + B + 1;
 
   // stage this CTA's B_v rows (all copies in flight at once)
   {
@@ -79,107 +88,121 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, 
   }
 
   const int NT = build_tile_prefix(a.seq_len, a.seq_start, B, a.n_rows, prefix, scan, a.err, false);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  // per row: reference max over the items and 1 / l (every CTA of the cluster does this)
-  for (int i = warp; i < nrow; i += kThreads / 32) {
-    const int b = b0 + i / qpg, j = h * qpg + i % qpg;
-    float M = -INFINITY, l = 0.f;
-    if (prefix[b + 1] > prefix[b]) {
-      const int c0 = item_of_tile(prefix[b], NT, a.n_items);
-      const int c1 = item_of_tile(prefix[b + 1] - 1, NT, a.n_items);
-      for (int cc = c0 + lane; cc <= c1; cc += 32)
-        if (item_begin(cc, NT, a.n_items) != item_begin(cc + 1, NT, a.n_items))
-          M = fmaxf(M, a.part_ml[(((int64_t)cc + b) * Hq + j) * 2]);
-#pragma unroll
-      for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-      for (int cc = c0 + lane; cc <= c1; cc += 32)
-        if (item_begin(cc, NT, a.n_items) != item_begin(cc + 1, NT, a.n_items)) {
-          const int64_t sl = ((int64_t)cc + b) * Hq + j;
-          l += exp2f(a.part_ml[sl * 2] - M) * a.part_ml[sl * 2 + 1];
-        }
-#pragma unroll
-      for (int o = 16; o; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-    }
-    if (lane == 0) {
-      sM[i] = M;
-      sinv[i] = l > 0.f ? 1.f / l : 0.f;
-    }
+  // first tile of every work item, and the items covering each row's sequence
+  for (int c = threadIdx.x; c <= a.n_items; c += kThreads) ibeg[c] = item_begin(c, NT, a.n_items);
+  if (threadIdx.x < nrow) {
+    const int b = b0 + threadIdx.x / qpg;
+    const bool any = prefix[b + 1] > prefix[b];
+    rc[2 * threadIdx.x] = any ? item_of_tile(prefix[b], NT, a.n_items) : 0;
+    rc[2 * threadIdx.x + 1] = any ? item_of_tile(prefix[b + 1] - 1, NT, a.n_items) : -1;
   }
   __syncthreads();
-  // u rows restricted to [r0, r0 + rr): items summed with independent float4 loads
+
+  // u rows restricted to [r0, r0 + rr), merged over the items in one pass with
+  // a running reference max: each thread owns float4 columns of whole rows and
+  // keeps kItemBatch items' loads in flight.  Every thread of a row sees the
+  // same maxima in the same order, so they agree on M; the thread of column 0
+  // also merges l.
   const int rr4 = rr / 4;
   for (int idx = threadIdx.x; idx < nrow * rr4; idx += kThreads) {
     const int i = idx / rr4, r4 = idx % rr4;
     const int b = b0 + i / qpg, j = h * qpg + i % qpg;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (prefix[b + 1] > prefix[b]) {
-      const int c0 = item_of_tile(prefix[b], NT, a.n_items);
-      const int c1 = item_of_tile(prefix[b + 1] - 1, NT, a.n_items);
-      const float Mi = sM[i];
+    float M = -INFINITY, l = 0.f;
+    const int c0 = rc[2 * i], c1 = rc[2 * i + 1];
+    {
       for (int cc = c0; cc <= c1; cc += kItemBatch) {
-        float w[kItemBatch];
+        float m[kItemBatch], lv[kItemBatch];
         float4 v[kItemBatch];
 #pragma unroll
         for (int u = 0; u < kItemBatch; ++u) {
           const int c = cc + u;
-          const bool live = c <= c1 && item_begin(c, NT, a.n_items) != item_begin(c + 1, NT, a.n_items);
+          const bool live = c <= c1 && ibeg[c] != ibeg[c + 1];
           const int64_t sl = ((int64_t)(live ? c : c0) + b) * Hq + j;
-          w[u] = live ? exp2f(a.part_ml[sl * 2] - Mi) : 0.f;
+          const float2 ml = reinterpret_cast<const float2*>(a.part_ml)[sl];
+          m[u] = live ? ml.x : -INFINITY;
+          lv[u] = ml.y;
           v[u] = reinterpret_cast<const float4*>(a.part_u + sl * rv + r0)[r4];
         }
+        float Mb = M;
+#pragma unroll
+        for (int u = 0; u < kItemBatch; ++u) Mb = fmaxf(Mb, m[u]);
+        if (Mb == -INFINITY) continue;  // nothing live yet
+        const float sc = exp2f(M - Mb);
+        acc.x *= sc;
+        acc.y *= sc;
+        acc.z *= sc;
+        acc.w *= sc;
+        l *= sc;
 #pragma unroll
         for (int u = 0; u < kItemBatch; ++u) {
-          acc.x = fmaf(w[u], v[u].x, acc.x);
-          acc.y = fmaf(w[u], v[u].y, acc.y);
-          acc.z = fmaf(w[u], v[u].z, acc.z);
-          acc.w = fmaf(w[u], v[u].w, acc.w);
+          const float w = exp2f(m[u] - Mb);  // 0 for items that are not live
+          acc.x = fmaf(w, v[u].x, acc.x);
+          acc.y = fmaf(w, v[u].y, acc.y);
+          acc.z = fmaf(w, v[u].z, acc.z);
+          acc.w = fmaf(w, v[u].w, acc.w);
+          l = fmaf(w, lv[u], l);
         }
+        M = Mb;
       }
     }
     reinterpret_cast<float4*>(su + (size_t)i * rr)[r4] = acc;
+    if (r4 == 0) sinv[i] = l > 0.f ? 1.f / l : 0.f;
   }
   cp_async_wait_all();
   __syncthreads();
-  // partial o over this CTA's rows: thread = (column pair, row phase)
+  // partial o over this CTA's rows of B_v: thread = (column pair, every
+  // kGroups-th row of the chunk), so each output has one owner
   constexpr int kPairs = D / 2;
-  constexpr int kPhases = kThreads / kPairs;  // 4 (D = 128) or 8 (D = 64)
-  const int cp = threadIdx.x % kPairs, ph = threadIdx.x / kPairs;
-  float acc[kMaxRows][2];
+  constexpr int kGroups = kThreads / kPairs;        // 4 (D = 128) or 8 (D = 64)
+  constexpr int kRowsPer = kMaxRows / kGroups;      // 4 or 2
+  const int cp = threadIdx.x % kPairs, ig = threadIdx.x / kPairs;
+  float acc[kRowsPer][2];
 #pragma unroll
-  for (int i = 0; i < kMaxRows; ++i) acc[i][0] = acc[i][1] = 0.f;
-  for (int r = ph; r < rr; r += kPhases) {
-    const float x0 = to_f32(sbv[(size_t)r * D + 2 * cp]), x1 = to_f32(sbv[(size_t)r * D + 2 * cp + 1]);
+  for (int q = 0; q < kRowsPer; ++q) acc[q][0] = acc[q][1] = 0.f;
+  for (int r = 0; r < rr; r += 4) {
+    float x0[4], x1[4];
 #pragma unroll
-    for (int i = 0; i < kMaxRows; ++i) {
+    for (int t = 0; t < 4; ++t) {
+      const float2 xv = pair_f32(sbv + (size_t)(r + t) * D + 2 * cp);
+      x0[t] = xv.x;
+      x1[t] = xv.y;
+    }
+#pragma unroll
+    for (int q = 0; q < kRowsPer; ++q) {
+      const int i = ig + kGroups * q;
       if (i < nrow) {
-        const float uv = su[(size_t)i * rr + r];
-        acc[i][0] = fmaf(uv, x0, acc[i][0]);
-        acc[i][1] = fmaf(uv, x1, acc[i][1]);
+        const float4 uv = *reinterpret_cast<const float4*>(&su[(size_t)i * rr + r]);
+        acc[q][0] = fmaf(uv.x, x0[0], fmaf(uv.y, x0[1], fmaf(uv.z, x0[2], fmaf(uv.w, x0[3], acc[q][0]))));
+        acc[q][1] = fmaf(uv.x, x1[0], fmaf(uv.y, x1[1], fmaf(uv.z, x1[2], fmaf(uv.w, x1[3], acc[q][1]))));
       }
     }
   }
-  for (int i = threadIdx.x; i < kMaxRows * D; i += kThreads) so[i] = 0.f;
-  __syncthreads();
+  // cluster-wide sum: output e = i * D + col belongs to rank e % split, which
+  // receives every rank's partial in its slot [rank][e / split] (remote stores,
+  // made visible by the cluster barrier), then reduces and writes its outputs
+  const int share = kMaxRows * D / split;
 #pragma unroll
-  for (int i = 0; i < kMaxRows; ++i)
-    if (i < nrow) {
-      atomicAdd(&so[i * D + 2 * cp], acc[i][0]);
-      atomicAdd(&so[i * D + 2 * cp + 1], acc[i][1]);
-    }
-  // cluster-wide sum of the partial outputs; rank 0 writes
-  cluster.sync();
-  if (rank == 0) {
-    T* out = static_cast<T*>(a.out);
-    for (int idx = threadIdx.x; idx < nrow * D; idx += kThreads) {
-      float v = 0.f;
-      for (int q = 0; q < split; ++q) v += cluster.map_shared_rank(so, q)[idx];
-      const int i = idx / D, e = idx % D;
-      const int b = b0 + i / qpg, j = h * qpg + i % qpg;
-      out[((int64_t)b * Hq + j) * D + e] = from_f32<T>(v * sinv[i]);
-    }
+  for (int q = 0; q < kRowsPer; ++q) {
+    const int i = ig + kGroups * q;
+    if (i < nrow)
+#pragma unroll
+      for (int t = 0; t < 2; ++t) {
+        const int e = i * D + 2 * cp + t;
+        cluster.map_shared_rank(so, e % split)[rank * share + e / split] = acc[q][t];
+      }
   }
-  cluster.sync();  // keep every CTA's shared memory alive until rank 0 has read it
+  cluster.sync();
+  T* out = static_cast<T*>(a.out);
+  for (int pos = threadIdx.x; pos * split < nrow * D; pos += kThreads) {
+    const int e = pos * split + rank;
+    if (e >= nrow * D) break;
+    float v = 0.f;
+    for (int q = 0; q < split; ++q) v += so[q * share + pos];
+    const int i = e / D, col = e % D;
+    const int b = b0 + i / qpg, j = h * qpg + i % qpg;
+    out[((int64_t)b * Hq + j) * D + col] = from_f32<T>(v * sinv[i]);
+  }
 }
 
 template <typename T, int D>
@@ -192,8 +215,8 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   const int bchunk = std::max(1, std::min(a.B, kMaxRows / lt.qpg));
   const int rr = lt.rv / split;
   const size_t smem = (size_t)rr * D * sizeof(T) +
-                      sizeof(float) * ((size_t)kMaxRows * rr + kMaxRows * D + 2 * kMaxRows) +
-                      sizeof(int) * (kThreads + a.B + 1);
+                      sizeof(float) * ((size_t)kMaxRows * rr + kMaxRows * D + kMaxRows) +
+                      sizeof(int) * (2 * kMaxRows + kThreads + a.B + 1 + a.n_items + 1);
   auto k = combine_kernel<T, D>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;

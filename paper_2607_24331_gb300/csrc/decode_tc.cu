@@ -178,6 +178,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
   volatile int* abort_flag = &sm.abort_flag;
   const int hq_pad = ta.hq_pad;
   const int Hq = lt.Hq, qpg = lt.qpg;
+  griddep_launch();  // the absorption kernel may start streaming values as CTAs finish
 
   // ---- setup -------------------------------------------------------------
   if (tid == 0) {
