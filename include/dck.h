@@ -131,9 +131,10 @@ dck_status dck_latent_append(const dck_layer_desc* desc, const void* x, int32_t 
  *   out         [B, Hq, d]
  *   workspace   scratch of at least dck_decode_workspace_size(desc, B, n_rows)
  *               bytes, 256-byte aligned; its contents need no initialisation
- * Work is balanced over the device's SMs by 128-token tiles; the split
- * partials live in the workspace and are merged by a last kernel on the same
- * stream.  The bf16 tensor-core path also keeps per-tile softmax
+ * Work is balanced over the device's SMs by 128-token tiles (the bf16
+ * tensor-core path splits the tiles left over after an even share of whole
+ * tiles per SM further, by groups of heads); the split partials live in the
+ * workspace and are merged by a last kernel on the same stream.  The bf16 tensor-core path also keeps per-tile softmax
  * probabilities there, sized for sequences that do not share cache rows:
  * more than ceil(n_rows / 128) + B tiles in all is reported as DCK_ERR_INVALID
  * by dck_last_device_error and leaves `out` undefined.

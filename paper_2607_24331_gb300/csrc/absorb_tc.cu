@@ -4,8 +4,9 @@
 // with P_tile the bf16 probabilities the scores kernel wrote (already the
 // 128B-swizzled image of the UMMA B operand) and C_v[tile] the tile's value
 // latents [128 tokens x r_v].  The segments and their partial slots are those
-// of the scores kernel (the same flattened tile split over the same number of
-// CTAs), which has already written each segment's reference max and row sum.
+// of the scores kernel (the same split of the flattened tiles over the same
+// number of CTAs: whole main tiles per CTA, every extra tile a segment of its
+// own), which has already written each segment's reference max and row sum.
 //
 // The scores kernel's reference max of a head can rise from one tile to the
 // next (it moves only when a tile's max exceeds it by 8); before such a tile
@@ -102,16 +103,38 @@ __global__ void __launch_bounds__(kAThreads, 1)
     tmem_alloc(&sm.tmem_base, kTmemCols);
     tmem_relinquish();
   }
-  int NT, b_first, pre_first;
-  tile_scan(a, sm.scan, a.n_items, NT, b_first, pre_first);
+  // the work split of the scores kernel: main tiles [x0, x1) in segments per
+  // sequence, then whole extra tiles [e0, e1), each a segment of its own
+  const int NT = tile_count(a, sm.scan);
+  const Split sp(NT, a.n_items, a.split_extra != 0);
+  const bool fits = NT <= aa.max_tiles;  // else the scores kernel has reported the input
+  const int x0 = fits ? sp.main_begin(blockIdx.x, a.n_items) : 0;
+  const int x1 = fits ? sp.main_begin(blockIdx.x + 1, a.n_items) : 0;
+  // extra tiles by r_v chunks: chunks [c_lo, c_hi) of the flattened (extra tile, chunk) list
+  const int xc = sp.R * n_chunks;
+  const int c_lo = fits ? (int)((int64_t)blockIdx.x * xc / a.n_items) : 0;
+  const int c_hi = fits ? (int)((int64_t)(blockIdx.x + 1) * xc / a.n_items) : 0;
+  const int xe0 = sp.NTm + (c_lo < c_hi ? c_lo / n_chunks : 0), xe1 = sp.NTm + (c_lo < c_hi ? (c_hi - 1) / n_chunks + 1 : 0);
+  int bm, pm, bx, px;
+  tile_find(a, sm.scan, x0, bm, pm);
+  tile_find(a, sm.scan, xe0, bx, px);
+  const Walker walk_m{bm, pm, x0, x1, false}, walk_x{bx, px, xe0, xe1, true};
+  const bool has_work = x0 < x1 || xe0 < xe1;
+  // r_v chunks [ca, cb) of flattened tile x in phase ph (0: main, every chunk)
+  auto chunks_of = [&](int ph, int64_t x, int& ca, int& cb) {
+    ca = 0;
+    cb = n_chunks;
+    if (ph) {
+      const int e = (int)(x - sp.NTm);
+      ca = max(c_lo - e * n_chunks, 0);
+      cb = min(c_hi - e * n_chunks, n_chunks);
+    }
+  };
+  const int64_t xbase = extra_slot_base(a.n_items, a.B);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
-  const bool fits = NT <= aa.max_tiles;  // else the scores kernel has reported the input
-  const int x0 = fits ? item_begin(blockIdx.x, NT, a.n_items) : 0;
-  const int x1 = fits ? item_begin(blockIdx.x + 1, NT, a.n_items) : 0;
-  Walker walk{b_first, pre_first, x0, x1};
   Segment seg;
   DCK_AB_TRACE(0);
 
@@ -121,14 +144,17 @@ __global__ void __launch_bounds__(kAThreads, 1)
     // running (programmatic dependent launch): the first tile's rows are
     // prefetched and its first chunks loaded before the wait for that kernel's
     // probabilities and maxima.
-    if (x0 < x1) {
+    if (has_work) {
       const uint64_t pol = policy_evict_first();
-      int v_cnt = 0, p_cnt = 0, c_pre = 0;
+      int v_cnt = 0, p_cnt = 0;
       bool ok = true, first = true;
-      while (ok && walk.next(a, seg)) {
+      for (int ph = 0; ph < 2 && ok; ++ph)
+      for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
         for (int i = 0; i < seg.ntiles && ok; ++i) {
           const int64_t x = seg.x0 + i;
           const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
+          int ca, cb;
+          chunks_of(ph, x, ca, cb);
           if (lane == 0) {  // this CTA's first tile, then each next tile, toward L2
             for (int q = first ? 0 : 1; q < 2; ++q) {
               if (q == 1 && i + 1 >= seg.ntiles) break;
@@ -137,17 +163,18 @@ __global__ void __launch_bounds__(kAThreads, 1)
                 prefetch_l2(static_cast<const __nv_bfloat16*>(a.vc) + r0 * lt.rv, (uint32_t)(nr * lt.rv * 2));
             }
           }
-          if (first) {  // chunks that fit the empty ring, ahead of the wait
-            c_pre = min(n_chunks, kNVs / 2);
-            for (int c = 0; c < c_pre; ++c) {
-              if (lane < 2) {
-                const int sl = (v_cnt + lane) % kNVs;
-                mbar_expect_tx(&sm.v_full[sl], kVSlot);
-                tma_load_2d_hint(sm.v[sl], &maps.vc, &sm.v_full[sl], 128 * c + 64 * lane, (int32_t)yrow, pol);
-              }
-              __syncwarp();
-              v_cnt += 2;
+          // value slot v_cnt + q holds half (q % 2) of chunk ca + q / 2
+          int nbox = 2 * (cb - ca), done = 0;
+          if (first) {  // the boxes that fit the empty ring, ahead of the wait
+            const int nb = min(nbox, kNVs);
+            if (lane < nb) {
+              const int sl = (v_cnt + lane) % kNVs;
+              mbar_expect_tx(&sm.v_full[sl], kVSlot);
+              tma_load_2d_hint(sm.v[sl], &maps.vc, &sm.v_full[sl], 128 * ca + 64 * lane, (int32_t)yrow, pol);
             }
+            __syncwarp();
+            v_cnt += nb;
+            done = nb;
             griddep_wait();
             first = false;
           }
@@ -171,28 +198,30 @@ __global__ void __launch_bounds__(kAThreads, 1)
           __syncwarp();
           DCK_AB_TRACE(1);
           ++p_cnt;
-          for (int c = c_pre; c < n_chunks && ok; ++c) {
-            if (!(ok = wait_slots(sm.v_empty, kNVs, v_cnt, 2, lane, abort_flag))) break;
-            if (lane < 2) {
-              const int sl = (v_cnt + lane) % kNVs;
+          while (done < nbox && ok) {  // as many boxes per instruction as slots are free
+            const int nb = claim_slots(sm.v_empty, kNVs, v_cnt, nbox - done, lane, abort_flag);
+            if (!(ok = nb > 0)) break;
+            if (lane < nb) {
+              const int sl = (v_cnt + lane) % kNVs, q = done + lane;
               mbar_expect_tx(&sm.v_full[sl], kVSlot);
-              tma_load_2d_hint(sm.v[sl], &maps.vc, &sm.v_full[sl], 128 * c + 64 * lane, (int32_t)yrow, pol);
+              tma_load_2d_hint(sm.v[sl], &maps.vc, &sm.v_full[sl], 128 * ca + 64 * q, (int32_t)yrow, pol);
             }
             __syncwarp();
             DCK_AB_TRACE(2);
-            v_cnt += 2;
+            v_cnt += nb;
+            done += nb;
           }
-          c_pre = 0;
         }
       }
     }
   } else if (warp == 1) {
     // ---- MMA issuer (lane 0) ---------------------------------------------------
-    if (lane == 0 && x0 < x1) {
+    if (lane == 0 && has_work) {
       const uint32_t idesc_v = idesc_bf16(128, hq_pad, true, false);
       int v_cnt = 0, p_cnt = 0, rc = 0, sgc = 0;
       bool ok = true;
-      while (ok && walk.next(a, seg)) {
+      for (int ph = 0; ph < 2 && ok; ++ph)
+      for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
         for (int i = 0; i < seg.ntiles && ok; ++i) {
           const int psl = p_cnt % kNP;
           if (!(ok = mbar_wait(&sm.p_full[psl], (p_cnt / kNP) & 1, abort_flag))) break;
@@ -217,8 +246,10 @@ __global__ void __launch_bounds__(kAThreads, 1)
           // chunks in pairs: the K = 16 MMAs of one chunk form a dependent chain on
           // its accumulator (about 120 cycles each at N = Hq_pad), so two chunks'
           // chains are interleaved
-          for (int c = 0; c < n_chunks && ok; c += 2) {
-            const int nc = min(2, n_chunks - c);
+          int ca, cb;
+          chunks_of(ph, seg.x0 + i, ca, cb);
+          for (int c = ca; c < cb && ok; c += 2) {
+            const int nc = min(2, cb - c);
             uint32_t vb[2] = {0u, 0u};
             for (int q = 0; q < nc && ok; ++q) {
               const int sl = (v_cnt + 2 * q) % kNVs;  // even: the chunk's halves are adjacent slots
@@ -267,7 +298,8 @@ __global__ void __launch_bounds__(kAThreads, 1)
     int rc = 0, sgc = 0;
     bool ok = true;
     griddep_wait();  // the maxima come from the scores kernel
-    while (ok && walk.next(a, seg)) {
+    for (int ph = 0; ph < 2 && ok; ++ph)
+      for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
       for (int i = 1; i < seg.ntiles && ok; ++i) {
         const int64_t x = seg.x0 + i;
         // reference maxima of this tile and the previous one, head = lane
@@ -296,13 +328,15 @@ __global__ void __launch_bounds__(kAThreads, 1)
         }
       }
       if (!ok) break;
-      // segment end: U -> partial slot c + b
+      // segment end: U -> partial slot c + b (extra tile e: slot xbase + e)
       if (!(ok = wwait(&sm.u_ready, sgc & 1, abort_flag))) break;
       tc_fence_after();
       DCK_AB_TRACE(22);
-      const int64_t slot = (int64_t)blockIdx.x + seg.b;
+      const int64_t slot = ph ? xbase + (seg.x0 - sp.NTm) : (int64_t)blockIdx.x + seg.b;
       float* dst = a.part_u + slot * Hq * lt.rv + tau;
-      for (int c = 0; c < n_chunks; ++c) {
+      int ca, cb;  // the segment's last tile (extra segments have one)
+      chunks_of(ph, seg.x0 + seg.ntiles - 1, ca, cb);
+      for (int c = ca; c < cb; ++c) {
         float v0[16], v1[16];
         tmem_ld16(tmem + lane_base + c * hq_pad, v0);
         if (hq_pad > 16) tmem_ld16(tmem + lane_base + c * hq_pad + 16, v1);

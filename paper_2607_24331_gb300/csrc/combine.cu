@@ -2,8 +2,9 @@
 //
 // Every work item wrote, for each sequence b it touched and each query head j,
 // the un-normalised latent accumulator u = sum_t 2^(s_t - m) v_t, its reference
-// max m (log2 units) and l = sum_t 2^(s_t - m).  For sequence b this kernel
-// takes the items covering b's tiles, merges them with
+// max m (log2 units) and l = sum_t 2^(s_t - m) (the tensor-core path also one
+// such partial per extra tile, see tc_common.cuh).  For sequence b this kernel
+// takes the partials covering b's tiles, merges them with
 //   M = max m_c,  u = sum_c 2^(m_c - M) u_c,  l = sum_c 2^(m_c - M) l_c
 // and applies the value up-factor once per head (Sec. III-D, x W^(v) ~ z_v R_v):
 //   o_j = (u / l) B_v[:, h d : (h+1) d],  h = KV head of j.
@@ -13,7 +14,7 @@
 // rows as fit kMaxRows, so each head's B_v block is staged about once.
 // CTA `rank` of a cluster owns rows [rank*rv/split, (rank+1)*rv/split) of u
 // and of B_v's column block: it merges those rows of every (sequence, query
-// head) row of its chunk in one pass with a running max (sixteen items' loads in
+// head) row of its chunk in one pass with a running max (twelve partials' loads in
 // flight at a time), stages its B_v rows in shared memory with cp.async (all
 // issued up front), and forms the partial product over its rows, each output
 // owned by one thread.  The cluster adds the partial outputs through
@@ -32,7 +33,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kMaxSplit = 8;    // CTAs per cluster (r_v split), portable cluster size
 constexpr int kMaxRows = 16;    // (sequence, query head) rows per cluster
-constexpr int kItemBatch = 16;  // partial items whose loads are in flight together
+constexpr int kItemBatch = 12;  // partials whose loads are in flight together
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)),
@@ -49,7 +50,7 @@ __device__ __forceinline__ float2 pair_f32(const __nv_bfloat16* p) {
 }
 
 template <typename T, int D>
-__global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, const DecodeArgs a, int bchunk,
+__global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable lt, const DecodeArgs a, int bchunk,
                                                           int split) {
   extern __shared__ __align__(16) uint8_t smem_c[];
   cg::cluster_group cluster = cg::this_cluster();
@@ -64,13 +65,13 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, 
   const int r0 = rank * rr;
 
   // shared layout: B_v rows [rr][D] T | u rows [kMaxRows][rr] | received partial o [split][kMaxRows * D / split]
-  // | 1/l | row item ranges [kMaxRows][2] | scan | prefix | item starts [n_items + 1]
+  // | 1/l | row slot ranges [kMaxRows][4] | scan | prefix | item starts [n_items + 1]
   T* sbv = reinterpret_cast<T*>(smem_c);
   float* su = reinterpret_cast<float*>(smem_c + (size_t)rr * D * sizeof(T));
   float* so = su + (size_t)kMaxRows * rr;
   float* sinv = so + kMaxRows * D;
   int* rc = reinterpret_cast<int*>(sinv + kMaxRows);
-  int* scan = rc + 2 * kMaxRows;
+  int* scan = rc + 4 * kMaxRows;
   int* prefix = scan + kThreads;
   int* ibeg = prefix + B + 1;
 
@@ -88,13 +89,21 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, 
   }
 
   const int NT = build_tile_prefix(a.seq_len, a.seq_start, B, a.n_rows, prefix, scan, a.err, false);
-  // first tile of every work item, and the items covering each row's sequence
-  for (int c = threadIdx.x; c <= a.n_items; c += kThreads) ibeg[c] = item_begin(c, NT, a.n_items);
+  // Partials of sequence b: the items c whose main tiles (the first NTm, split
+  // evenly in whole tiles) cover b's, in slots c + b; with the tensor-core
+  // split, also one slot per extra tile x >= NTm of b, slot xbase + x - NTm.
+  const int NTm = main_tiles(NT, a.n_items, a.split_extra != 0);
+  const int64_t xbase = (int64_t)a.n_items + B - 1;
+  for (int c = threadIdx.x; c <= a.n_items; c += kThreads) ibeg[c] = item_begin(c, NTm, a.n_items);
   if (threadIdx.x < nrow) {
     const int b = b0 + threadIdx.x / qpg;
-    const bool any = prefix[b + 1] > prefix[b];
-    rc[2 * threadIdx.x] = any ? item_of_tile(prefix[b], NT, a.n_items) : 0;
-    rc[2 * threadIdx.x + 1] = any ? item_of_tile(prefix[b + 1] - 1, NT, a.n_items) : -1;
+    const int me = min(prefix[b + 1], NTm);  // end of b's main tiles
+    const bool any = me > prefix[b];
+    int* r = rc + 4 * threadIdx.x;
+    r[0] = any ? item_of_tile(prefix[b], NTm, a.n_items) : 0;           // first main item
+    r[1] = any ? item_of_tile(me - 1, NTm, a.n_items) - r[0] + 1 : 0;  // main items
+    r[2] = max(prefix[b], NTm) - NTm;                                   // first extra tile
+    r[3] = max(prefix[b + 1] - NTm, r[2]) - r[2];                       // extra tiles
   }
   __syncthreads();
 
@@ -109,16 +118,18 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const LayerTable lt, 
     const int b = b0 + i / qpg, j = h * qpg + i % qpg;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     float M = -INFINITY, l = 0.f;
-    const int c0 = rc[2 * i], c1 = rc[2 * i + 1];
-    {
-      for (int cc = c0; cc <= c1; cc += kItemBatch) {
+    const int c0 = rc[4 * i], nm = rc[4 * i + 1], e0 = rc[4 * i + 2], ns = nm + rc[4 * i + 3];
+    if (ns > 0) {
+      const int xb = (int)xbase + e0 - nm;                       // slot of partial q >= nm: xb + q
+      const int s0 = nm > 0 ? c0 + b : xb + nm;                    // a live slot
+      for (int vv = 0; vv < ns; vv += kItemBatch) {
         float m[kItemBatch], lv[kItemBatch];
         float4 v[kItemBatch];
 #pragma unroll
         for (int u = 0; u < kItemBatch; ++u) {
-          const int c = cc + u;
-          const bool live = c <= c1 && ibeg[c] != ibeg[c + 1];
-          const int64_t sl = ((int64_t)(live ? c : c0) + b) * Hq + j;
+          const int q = vv + u;  // q-th partial of the row: main items, then extra tiles
+          const bool live = q < ns && (q >= nm || ibeg[c0 + q] != ibeg[c0 + q + 1]);
+          const int64_t sl = (int64_t)(live ? (q < nm ? c0 + b + q : xb + q) : s0) * Hq + j;
           const float2 ml = reinterpret_cast<const float2*>(a.part_ml)[sl];
           m[u] = live ? ml.x : -INFINITY;
           lv[u] = ml.y;
@@ -216,7 +227,7 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   const int rr = lt.rv / split;
   const size_t smem = (size_t)rr * D * sizeof(T) +
                       sizeof(float) * ((size_t)kMaxRows * rr + kMaxRows * D + kMaxRows) +
-                      sizeof(int) * (2 * kMaxRows + kThreads + a.B + 1 + a.n_items + 1);
+                      sizeof(int) * (4 * kMaxRows + kThreads + a.B + 1 + a.n_items + 1);
   auto k = combine_kernel<T, D>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;

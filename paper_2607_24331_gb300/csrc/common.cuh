@@ -47,6 +47,7 @@ struct DecodeArgs {
   int64_t n_rows;
   int32_t B;
   int32_t n_items;
+  int32_t split_extra;  // tensor-core path: extra tiles split finely, each with its own partial slot
   float theta;
   float* part_u;   // [n_slots, Hq, rv]
   float* part_ml;  // [n_slots, Hq, 2]  (running max in log2 units, sum)
@@ -141,6 +142,15 @@ __device__ __forceinline__ int valid_len(const int32_t* seq_len, const int64_t* 
 
 __device__ __forceinline__ int item_begin(int c, int NT, int n_items) {
   return (int)(((int64_t)c * NT) / n_items);
+}
+
+// Tiles [0, main_tiles) are split in contiguous whole-tile ranges over the
+// n_items work items; with `split_extra` (tensor-core path) and fewer than
+// kFineSplitBelow tiles per item, only n_items * floor(NT / n_items) of them,
+// the rest ("extra tiles") being shared out more finely (see tc_common.cuh).
+constexpr int kFineSplitBelow = 8;
+__host__ __device__ __forceinline__ int main_tiles(int NT, int n_items, bool split_extra) {
+  return split_extra && NT / n_items < kFineSplitBelow ? NT / n_items * n_items : NT;
 }
 
 // The item whose tile range contains tile x (0 <= x < NT).

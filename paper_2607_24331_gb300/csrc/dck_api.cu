@@ -1,5 +1,6 @@
 // C ABI of libdck: argument validation, work planning and kernel dispatch.
 // The formulas and conventions are documented in include/dck.h.
+#include <algorithm>
 #include <atomic>
 #include <cmath>
 #include <cstring>
@@ -111,14 +112,23 @@ LayerTable make_table(const dck_layer_desc* d) {
   return lt;
 }
 
-size_t decode_ws_parts(const LayerTable& lt, int batch, int n_items) {
-  const size_t slots = (size_t)n_items + (batch > 0 ? batch - 1 : 0);
+// Partial slots: c + b for work item c and sequence b it touched (n_items + B - 1),
+// then one per extra tile of the tensor-core path: fewer than n_items, and no
+// more than the call's tiles (ceil(n_rows / 128) + B with non-overlapping sequences).
+size_t n_partial_slots(int batch, int n_items, int64_t n_rows) {
+  const int64_t tiles = (n_rows + 127) / 128 + batch;
+  const int64_t extra = std::min<int64_t>(n_items > 0 ? n_items - 1 : 0, tiles);
+  return (size_t)n_items + (batch > 0 ? batch - 1 : 0) + (size_t)extra;
+}
+
+size_t decode_ws_parts(const LayerTable& lt, int batch, int n_items, int64_t n_rows) {
+  const size_t slots = n_partial_slots(batch, n_items, n_rows);
   return align_up(slots * lt.Hq * lt.rv * sizeof(float), 256) + align_up(slots * lt.Hq * 2 * sizeof(float), 256);
 }
 
 // Workspace: split partials U and (m, l), then the tensor-core path's extra region.
 size_t decode_ws_bytes(const LayerTable& lt, int batch, int n_items, int dtype, int64_t n_rows) {
-  return decode_ws_parts(lt, batch, n_items) + (dtype == DCK_BF16 ? tc_decode_extra_ws(lt, batch, n_rows) : 0);
+  return decode_ws_parts(lt, batch, n_items, n_rows) + (dtype == DCK_BF16 ? tc_decode_extra_ws(lt, batch, n_rows) : 0);
 }
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
@@ -194,19 +204,20 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const
   a.B = batch;
   a.n_items = sms;
   a.theta = rope_theta;
-  const size_t slots = (size_t)sms + batch - 1;
+  const size_t slots = n_partial_slots(batch, sms, n_rows);
   a.part_u = static_cast<float*>(workspace);
   a.part_ml = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                        align_up(slots * lt.Hq * lt.rv * sizeof(float), 256));
   a.out = out;
   a.err = err;
-  a.extra = static_cast<char*>(workspace) + decode_ws_parts(lt, batch, sms);
+  a.extra = static_cast<char*>(workspace) + decode_ws_parts(lt, batch, sms, n_rows);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e;
   const bool use_tc = g_decode_kernel.load() == 0 && n_rows < (int64_t(1) << 31) - 256 &&
                       tc_decode_supports(lt, desc->dtype);
   a.ev0 = g_ev_start.load();
   a.ev1 = g_ev_stop.load();
+  a.split_extra = use_tc ? 1 : 0;
   if (use_tc) e = launch_decode_tc(lt, a, s);
   else e = launch_decode_simt(lt, a, desc->dtype, s);
   if (e != cudaSuccess) return DCK_ERR_CUDA;

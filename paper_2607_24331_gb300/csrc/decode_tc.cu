@@ -93,6 +93,7 @@ constexpr int kMaxGroupsTc = 16;
 constexpr int kMaxPieces = 5;
 constexpr int kMaxHqTc = 32;
 constexpr int kMaxItems = 256;
+constexpr int kMaxUnits = 32;
 constexpr int kEpiThreads = 256;
 constexpr float kRescaleThr = 8.f;  // log2 units: probabilities stay <= 256
 constexpr uint32_t kTmemCols = 512;
@@ -122,9 +123,10 @@ struct GroupSm {
   int8_t h0, nh;         // MMA position of the group's first head, heads
   int8_t nu;             // units (pairs of heads, the last one single when nh is odd)
   int8_t w[kMaxPieces];  // piece widths (ranks)
-  int8_t pad2[3];
+  int8_t pad;
+  int16_t u0;            // the group's first unit in the tile's unit order
   int16_t k[kMaxPieces]; // first rank of each piece
-  int16_t pad3;
+  int16_t i0;            // the group's first factor item in the tile's item order
 };
 
 struct TcArgs {
@@ -138,6 +140,9 @@ struct TcArgs {
   double om[kD / 2];             // RoPE frequencies theta^(-2i/d), fp64
   GroupSm grp[kMaxGroupsTc];
   int16_t order[kMaxHqTc];       // KV head at each MMA position (group-major, slot order)
+  int n_units;                   // units per tile
+  int16_t uitem[kMaxUnits + 1];  // first factor item of each unit (and the item count)
+  int8_t hunit[kMaxHqTc];        // unit of each query head
   uint32_t item[kMaxItems];      // factor item n: byte offset | (bytes / 4096) << 26
 };
 
@@ -155,6 +160,8 @@ struct Smem {
   uint64_t k_full[2], k_empty[2], epi_bar;
   GroupSm grp[kMaxGroupsTc];
   int16_t order[kMaxHqTc];
+  int16_t uitem[kMaxUnits + 1];
+  int8_t hunit[kMaxHqTc];
   uint32_t item[kMaxItems];
   uint32_t tmem_base;
   int abort_flag;
@@ -204,25 +211,49 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
   }
   if (tid < lt.G) sm.grp[tid] = ta.grp[tid];
   if (tid < lt.Hkv) sm.order[tid] = ta.order[tid];
+  if (tid <= ta.n_units) sm.uitem[tid] = ta.uitem[tid];
+  if (tid < Hq) sm.hunit[tid] = ta.hunit[tid];
   for (int n = tid; n < ta.n_items; n += kThreads) sm.item[n] = ta.item[n];
   if (tid < kD / 2) {
     sm.om64[tid] = ta.om[tid];
     sm.om32[tid] = (float)ta.om[tid];
   }
-  int NT, b_first, pre_first;
-  tile_scan(a, reinterpret_cast<int*>(sm.x), a.n_items, NT, b_first, pre_first);
+  // Work of this CTA: main tiles [x0, x1) (every unit), then units [u_lo, u_hi)
+  // of the flattened (extra tile, unit) list, every extra tile a segment of its own.
+  const int U = ta.n_units;
+  const int NT = tile_count(a, reinterpret_cast<int*>(sm.x));
+  const Split sp(NT, a.n_items, a.split_extra != 0);
+  // the per-tile stores are sized for non-overlapping sequences; more tiles
+  // than that is reported as invalid input and nothing is computed
+  const bool fits = NT <= ta.max_tiles;
+  if (!fits && tid == 0 && blockIdx.x == 0) atomicOr(a.err, kErrBadSeq);
+  const int x0 = fits ? sp.main_begin(blockIdx.x, a.n_items) : 0;
+  const int x1 = fits ? sp.main_begin(blockIdx.x + 1, a.n_items) : 0;
+  const int xu = sp.R * U;
+  const int u_lo = fits ? (int)((int64_t)blockIdx.x * xu / a.n_items) : 0;
+  const int u_hi = fits ? (int)((int64_t)(blockIdx.x + 1) * xu / a.n_items) : 0;
+  const int xe0 = sp.NTm + (u_lo < u_hi ? u_lo / U : 0), xe1 = sp.NTm + (u_lo < u_hi ? (u_hi - 1) / U + 1 : 0);
+  int bm, pm, bx, px;
+  tile_find(a, reinterpret_cast<const int*>(sm.x), x0, bm, pm);
+  tile_find(a, reinterpret_cast<const int*>(sm.x), xe0, bx, px);
+  const Walker walk_m{bm, pm, x0, x1, false}, walk_x{bx, px, xe0, xe1, true};
+  const bool has_work = x0 < x1 || xe0 < xe1;
+  const int64_t xbase = extra_slot_base(a.n_items, a.B);
+  // units [ua, ub) of flattened tile x in phase ph (0: main, 1: extra)
+  auto units_of = [&](int ph, int x, int& ua, int& ub) {
+    ua = 0;
+    ub = U;
+    if (ph) {
+      const int e = x - sp.NTm;
+      ua = max(u_lo - e * U, 0);
+      ub = min(u_hi - e * U, U);
+    }
+  };
   for (int i = tid; i < kMaxHqTc * 128; i += kThreads) sm.x[i] = 0.f;
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
-  // the per-tile stores are sized for non-overlapping sequences; more tiles
-  // than that is reported as invalid input and nothing is computed
-  const bool fits = NT <= ta.max_tiles;
-  if (!fits && tid == 0 && blockIdx.x == 0) atomicOr(a.err, kErrBadSeq);
-  const int x0 = fits ? item_begin(blockIdx.x, NT, a.n_items) : 0;
-  const int x1 = fits ? item_begin(blockIdx.x + 1, NT, a.n_items) : 0;
-  Walker walk{b_first, pre_first, x0, x1};
   Segment seg;
   DCK_TC_TRACE(0);
 
@@ -251,90 +282,99 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     // ---- latent pieces, issued as soon as their slots are free; in
     // query-folded mode also the factor items of MMA thread 1, in the order
     // that thread consumes them (a group's pieces, then its units' items) ------
-    if (x0 < x1) {
+    if (has_work) {
       const uint64_t pol = policy_evict_first();
       const uint64_t pol_w = policy_evict_last();
       int a_cnt = 0, wc = 0, kc = 0;
       bool ok = true, images_ready = false;
-      while (ok && walk.next(a, seg)) {
-        const uint8_t* img = ta.fimg + (kFold ? (int64_t)seg.b * ta.fimg_seq_bytes : 0);
-        for (int i = 0; i < seg.ntiles && ok; ++i) {
-          const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
-          if (lane == 0 && i + 1 < seg.ntiles) {  // next tile's latent rows toward L2
-            const int64_t r0 = yrow + kTile, nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
-            if (nr > 0)
-              prefetch_l2(static_cast<const __nv_bfloat16*>(a.kc) + r0 * lt.Rk, (uint32_t)(nr * lt.Rk * 2));
-          }
-          int n = 0;  // factor item index inside the tile
-          for (int g = 0; g < lt.G && ok; ++g) {
-            const GroupSm& gs = sm.grp[g];
-            const int np = gs.np;
-            for (int p0 = 0; p0 < np && ok;) {
-              const int nb = claim_slots(sm.a_empty, kNA, a_cnt, np - p0, lane, abort_flag);
-              ok = nb > 0;
-              if (!ok) break;
-              if (lane < nb) {
-                const int sl = (a_cnt + lane) % kNA;
-                const int w = gs.w[p0 + lane];
-                const CUtensorMap* m = w == 64 ? &maps.kc64 : (w == 32 ? &maps.kc32 : &maps.kc16);
-                mbar_expect_tx(&sm.a_full[sl], kTile * w * 2);
-                tma_load_2d_hint(sm.a[sl], m, &sm.a_full[sl], gs.roff + gs.k[p0 + lane], (int32_t)yrow, pol);
-              }
-              __syncwarp();
-              a_cnt += nb;
-              p0 += nb;
+      for (int ph = 0; ph < 2 && ok; ++ph)
+        for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
+          const uint8_t* img = ta.fimg + (kFold ? (int64_t)seg.b * ta.fimg_seq_bytes : 0);
+          for (int i = 0; i < seg.ntiles && ok; ++i) {
+            const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
+            if (lane == 0 && i + 1 < seg.ntiles) {  // next tile's latent rows toward L2
+              const int64_t r0 = yrow + kTile, nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
+              if (nr > 0)
+                prefetch_l2(static_cast<const __nv_bfloat16*>(a.kc) + r0 * lt.Rk, (uint32_t)(nr * lt.Rk * 2));
             }
-            if (kMma == 2)
-              for (int u = 0; u < gs.nu && ok; ++u, ++kc, n += np) {
-                if ((kc & 1) != 1) continue;  // MMA thread 0's unit
-                if (!images_ready) {          // the images are written by the preparation kernel
-                  griddep_wait();
-                  images_ready = true;
+            int ua, ub;
+            units_of(ph, seg.x0 + i, ua, ub);
+            for (int g = 0; g < lt.G && ok; ++g) {
+              const GroupSm& gs = sm.grp[g];
+              const int np = gs.np;
+              const int lo = max(ua - gs.u0, 0), hi = min(ub - gs.u0, (int)gs.nu);
+              if (lo >= hi) continue;  // none of the group's units in this piece of work
+              for (int p0 = 0; p0 < np && ok;) {
+                const int nb = claim_slots(sm.a_empty, kNA, a_cnt, np - p0, lane, abort_flag);
+                ok = nb > 0;
+                if (!ok) break;
+                if (lane < nb) {
+                  const int sl = (a_cnt + lane) % kNA;
+                  const int w = gs.w[p0 + lane];
+                  const CUtensorMap* m = w == 64 ? &maps.kc64 : (w == 32 ? &maps.kc32 : &maps.kc16);
+                  mbar_expect_tx(&sm.a_full[sl], kTile * w * 2);
+                  tma_load_2d_hint(sm.a[sl], m, &sm.a_full[sl], gs.roff + gs.k[p0 + lane], (int32_t)yrow, pol);
                 }
-                ok = put_unit_items(1, wc, n, np, img, pol_w);
+                __syncwarp();
+                a_cnt += nb;
+                p0 += nb;
               }
+              if (kMma == 2)
+                for (int u = lo; u < hi && ok; ++u, ++kc) {
+                  if ((kc & 1) != 1) continue;  // MMA thread 0's unit
+                  if (!images_ready) {          // the images are written by the preparation kernel
+                    griddep_wait();
+                    images_ready = true;
+                  }
+                  ok = put_unit_items(1, wc, gs.i0 + u * np, np, img, pol_w);
+                }
+            }
           }
         }
-      }
     }
   } else if (warp == 10) {
     // ---- factor items: several bulk copies per instruction (query-folded
     // mode: the ring of MMA thread 0 only) --------------------------------------
-    if (x0 < x1) {
+    if (has_work) {
       const uint64_t pol = policy_evict_last();
       griddep_wait();  // the images are written by the preparation kernel
       int w_cnt = 0;
       bool ok = true;
       int wc = 0, kc = 0;  // items put into MMA thread 0's ring, units so far
-      while (ok && walk.next(a, seg)) {
-        const uint8_t* img = ta.fimg + (kFold ? (int64_t)seg.b * ta.fimg_seq_bytes : 0);
-        for (int i = 0; i < seg.ntiles && ok; ++i) {
-          if (kMma == 1) {  // one ring: claims may span units
-            for (int n0 = 0; n0 < ta.n_items && ok;) {
-              const int nb = claim_slots(sm.w_empty, NW, w_cnt, min(NW, ta.n_items - n0), lane, abort_flag);
-              ok = nb > 0;
-              if (!ok) break;
-              if (lane < nb) {
-                const int sl = (w_cnt + lane) % NW;
-                const uint32_t it = sm.item[n0 + lane];
-                const uint32_t bytes = (it >> 26) << 12;
-                mbar_expect_tx(&sm.w_full[sl], bytes);
-                bulk_load(sm.w[sl], img + (it & 0x03FFFFFFu), bytes, &sm.w_full[sl], pol);
+      for (int ph = 0; ph < 2 && ok; ++ph)
+        for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
+          const uint8_t* img = ta.fimg + (kFold ? (int64_t)seg.b * ta.fimg_seq_bytes : 0);
+          for (int i = 0; i < seg.ntiles && ok; ++i) {
+            int ua, ub;
+            units_of(ph, seg.x0 + i, ua, ub);
+            if (kMma == 1) {  // one ring: claims may span units (the units' items are contiguous)
+              const int n_end = sm.uitem[ub];
+              for (int n0 = sm.uitem[ua]; n0 < n_end && ok;) {
+                const int nb = claim_slots(sm.w_empty, NW, w_cnt, min(NW, n_end - n0), lane, abort_flag);
+                ok = nb > 0;
+                if (!ok) break;
+                if (lane < nb) {
+                  const int sl = (w_cnt + lane) % NW;
+                  const uint32_t it = sm.item[n0 + lane];
+                  const uint32_t bytes = (it >> 26) << 12;
+                  mbar_expect_tx(&sm.w_full[sl], bytes);
+                  bulk_load(sm.w[sl], img + (it & 0x03FFFFFFu), bytes, &sm.w_full[sl], pol);
+                }
+                __syncwarp();
+                w_cnt += nb;
+                n0 += nb;
               }
-              __syncwarp();
-              w_cnt += nb;
-              n0 += nb;
+              continue;
             }
-            continue;
-          }
-          int n = 0;
-          for (int g = 0; g < lt.G && ok; ++g) {
-            const int np = sm.grp[g].np, nu = sm.grp[g].nu;
-            for (int u = 0; u < nu && ok; ++u, ++kc, n += np)
-              if ((kc & 1) == 0) ok = put_unit_items(0, wc, n, np, img, pol);
+            for (int g = 0; g < lt.G && ok; ++g) {
+              const GroupSm& gs = sm.grp[g];
+              const int np = gs.np;
+              const int lo = max(ua - gs.u0, 0), hi = min(ub - gs.u0, (int)gs.nu);
+              for (int u = lo; u < hi && ok; ++u, ++kc)
+                if ((kc & 1) == 0) ok = put_unit_items(0, wc, gs.i0 + u * np, np, img, pol);
+            }
           }
         }
-      }
     }
   } else if (warp == 1 || (kMma == 2 && warp == 11)) {
     // ---- MMA issuers: lane 0 of warp 1 (and of warp 11 in query-folded mode)
@@ -343,28 +383,33 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     // owns a factor ring (single consumer) and observes every latent piece's
     // fill in order, releasing the pieces of groups it has no unit in, so no
     // parity test can see a stale phase. ---------------------------------------
-    if (lane == 0 && x0 < x1) {
+    if (lane == 0 && has_work) {
       const int t = warp == 1 ? 0 : 1;
       uint64_t* wfull = sm.w_full + t * NWt;
       uint64_t* wempty = sm.w_empty + t * NWt;
       int a_cnt = 0, w_cnt = 0, kc = 0, own = 0;
       bool ok = true;
-      while (ok && walk.next(a, seg)) {
+      for (int ph = 0; ph < 2 && ok; ++ph)
+      for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
         for (int i = 0; i < seg.ntiles && ok; ++i) {
+          int ua, ub;
+          units_of(ph, seg.x0 + i, ua, ub);
           for (int g = 0; g < lt.G && ok; ++g) {
             const GroupSm& gs = sm.grp[g];
-            const int np = gs.np, nu = gs.nu;
+            const int np = gs.np;
+            const int lo = max(ua - gs.u0, 0), hi = min(ub - gs.u0, (int)gs.nu);  // the group's units here
+            if (lo >= hi) continue;
             const int a_base = a_cnt;
-            const int uf = kMma == 2 ? (((kc & 1) == t) ? 0 : 1) : 0;  // this thread's first unit of the group
-            if (uf >= nu)  // none: observe the group's pieces, then release them
+            const int uf = lo + (kMma == 2 ? (((kc & 1) == t) ? 0 : 1) : 0);  // this thread's first unit of the group
+            if (uf >= hi)  // none: observe the group's pieces, then release them
               for (int p = 0; p < np && ok; ++p) {
                 const int sl = (a_base + p) % kNA;
                 if ((ok = mbar_wait(&sm.a_full[sl], ((a_base + p) / kNA) & 1, abort_flag))) mbar_arrive(&sm.a_empty[sl]);
               }
-            for (int u = uf; u < nu && ok; u += kMma) {
+            for (int u = uf; u < hi && ok; u += kMma) {
               const int nh = min(2, gs.nh - 2 * u);
               const uint32_t idesc_k = idesc_bf16(128, kD * nh, false, true);
-              const int kg = kc + u;                               // unit index of the CTA
+              const int kg = kc + (u - lo);                        // unit index of the CTA
               const int buf = kMma == 2 ? t : (kg & 1);
               const int use = kMma == 2 ? own : (kg >> 1);         // earlier units in this accumulator
               // readiness of this unit's factor items (and, at this thread's first
@@ -394,7 +439,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
               }
               DCK_TC_TRACE(10);
               const uint32_t dcol = tmem + buf * kKCols;
-              const bool last = u + kMma >= nu;  // this thread's last unit of the group
+              const bool last = u + kMma >= hi;  // this thread's last unit of the group
               for (int p = 0; p < np; ++p) {
                 const int asl = (a_base + p) % kNA;
                 const int wsl = w_cnt % NWt;
@@ -422,7 +467,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
               ++own;
             }
             a_cnt += np;
-            kc += nu;
+            kc += hi - lo;
           }
         }
       }
@@ -447,7 +492,8 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     ok = wwait(&sm.epi_bar, round & 1, abort_flag); \
     ++round;                                        \
   } while (0)
-    while (ok && walk.next(a, seg)) {
+    for (int ph = 0; ph < 2 && ok; ++ph)
+    for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
       if (!kFold) {
         // rotated queries of this sequence at position L-1, scaled to log2 units
         // (angle reduced mod 2 pi in fp64, sine and cosine in fp32)
@@ -475,9 +521,11 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
       // head jt's reference max (log2 units; the same in all 8 owners) and this
       // owner's share of its row sum, rescaled whenever the reference moves
       float m_run = -INFINITY, l_part = 0.f;
+      int ua = 0, ub = 0;  // units of the current tile
       for (int i = 0; i < seg.ntiles && ok; ++i) {
         const int t0 = seg.t_begin + kTile * i;
         const int64_t x = seg.x0 + i;  // flattened tile index
+        units_of(ph, (int)x, ua, ub);
         float cs[32], sn[32];
 #pragma unroll
         for (int ip = 0; ip < 32; ++ip) {
@@ -489,7 +537,8 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
         // per unit (one or two KV heads), in MMA order: partial scores of this frequency half
         for (int g = 0; g < lt.G && ok; ++g) {
           const GroupSm& gs = sm.grp[g];
-          for (int u = 0; u < gs.nu; ++u) {
+          const int lo = max(ua - gs.u0, 0), hi = min(ub - gs.u0, (int)gs.nu);
+          for (int u = lo; u < hi; ++u) {
             const int nh = min(2, gs.nh - 2 * u);
             const int buf = kc & 1;
             if (!(ok = wwait(&sm.k_full[buf], (kc >> 1) & 1, abort_flag))) break;
@@ -571,7 +620,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
         EPI_SYNC();  // every partial score of the tile is in x
         if (!ok) break;
         {
-          const bool own = jt < Hq;
+          const bool own = jt < Hq && sm.hunit[jt] >= ua && sm.hunit[jt] < ub;  // head computed here
           const int tb = 16 * ct;  // first token of this owner
           float sc[16];
           float4* xr = reinterpret_cast<float4*>(&sm.x[jt * 128 + tb]);
@@ -611,7 +660,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
             l_part += pf.x + pf.y;
             pk[k] = *reinterpret_cast<const uint32_t*>(&pv);
           }
-          if (jt < hq_pad) {  // padded heads get zero rows
+          if (own || (jt >= Hq && jt < hq_pad && ua == 0)) {  // padded heads get zero rows
             // image: [token atom (64)][head row][64 tokens], 128B rows, 16-byte chunks swizzled by row % 8
             uint8_t* img = ta.pglob + x * (hq_pad * 256) + (tb >> 6) * (hq_pad * 128) + (jt >> 3) * 1024 +
                            (jt & 7) * 128;
@@ -633,8 +682,8 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
       l_part += __shfl_xor_sync(0xffffffffu, l_part, 1);
       l_part += __shfl_xor_sync(0xffffffffu, l_part, 2);
       l_part += __shfl_xor_sync(0xffffffffu, l_part, 4);
-      if (jt < Hq && ct == 0) {
-        const int64_t slot = (int64_t)blockIdx.x + seg.b;
+      if (jt < Hq && ct == 0 && sm.hunit[jt] >= ua && sm.hunit[jt] < ub) {
+        const int64_t slot = ph ? xbase + (seg.x0 - sp.NTm) : (int64_t)blockIdx.x + seg.b;
         a.part_ml[(slot * Hq + jt) * 2] = m_run;
         a.part_ml[(slot * Hq + jt) * 2 + 1] = l_part;
       }
@@ -829,7 +878,7 @@ bool build_tables(const LayerTable& lt, TcArgs& ta, PrepArgs& pa) {
   std::memset(&ta, 0, sizeof(ta));
   std::memset(&pa, 0, sizeof(pa));
   ta.hq_pad = hq_pad_of(lt.Hq);
-  int pos = 0, item = 0, off = 0;
+  int pos = 0, item = 0, off = 0, unit = 0;
   for (int g = 0; g < lt.G; ++g) {
     GroupSm& gs = ta.grp[g];
     gs.roff = lt.grp_roff[g];
@@ -840,14 +889,19 @@ bool build_tables(const LayerTable& lt, TcArgs& ta, PrepArgs& pa) {
     gs.h0 = (int8_t)pos;
     gs.nh = (int8_t)lt.grp_nh[g];
     gs.nu = (int8_t)((lt.grp_nh[g] + 1) / 2);
+    gs.u0 = (int16_t)unit;
+    gs.i0 = (int16_t)item;
     for (int sl = 0; sl < lt.grp_nh[g]; ++sl)
       for (int h = 0; h < lt.Hkv; ++h)
         if (lt.head_group[h] == g && lt.head_slot[h] == sl) {
           if (pos >= kMaxHqTc) return false;
           ta.order[pos++] = (int16_t)h;
+          for (int jj = 0; jj < lt.qpg; ++jj) ta.hunit[h * lt.qpg + jj] = (int8_t)(unit + sl / 2);
         }
     for (int s0 = 0; s0 < lt.grp_nh[g]; s0 += 2) {
       const int nh = std::min(2, lt.grp_nh[g] - s0);
+      if (unit >= kMaxUnits) return false;
+      ta.uitem[unit++] = (int16_t)item;
       for (int p = 0; p < gs.np; ++p) {
         if (item >= kMaxItems) return false;
         const int w = gs.w[p], bytes = nh * w * 256;
@@ -864,6 +918,8 @@ bool build_tables(const LayerTable& lt, TcArgs& ta, PrepArgs& pa) {
       }
     }
   }
+  ta.n_units = unit;
+  ta.uitem[unit] = (int16_t)item;
   ta.n_items = item;
   pa.n_items = item;
   pa.seq_bytes = off;

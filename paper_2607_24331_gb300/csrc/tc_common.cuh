@@ -88,9 +88,11 @@ struct Segment {
   int64_t row0;  // first cache row of the sequence
 };
 
-// Walks the sequences overlapping flattened tiles [x, x1) in order.
+// Walks the sequences overlapping flattened tiles [x, x1) in order; with
+// `single`, every tile is a segment of its own.
 struct Walker {
   int b, pre, x, x1;
+  bool single;
   __device__ bool next(const DecodeArgs& a, Segment& sg) {
     while (x < x1 && b < a.B) {
       const int nt = ntiles_of(a, b);
@@ -99,7 +101,7 @@ struct Walker {
         ++b;
         continue;
       }
-      const int xe = min(x1, pre + nt);
+      const int xe = single ? x + 1 : min(x1, pre + nt);
       sg.b = b;
       sg.L = valid_len(a.seq_len, a.seq_start, b, a.n_rows);
       sg.row0 = a.seq_start[b];
@@ -114,12 +116,11 @@ struct Walker {
   }
 };
 
-// Block-wide scan over the batch (every thread of the block calls it; `scan`
-// is shared scratch of blockDim.x ints): total tile count, and the first
-// sequence and its tile prefix for flattened tile x0.  Block 0 of the grid
-// reports sequences whose rows fall outside the cache.
-__device__ __forceinline__ void tile_scan(const DecodeArgs& a, int* scan, int n_items, int& NT_out,
-                                          int& b_first, int& pre_first) {
+// Block-wide tile count over the batch (every thread of the block calls it;
+// `scan` is shared scratch of blockDim.x ints and keeps each thread's
+// inclusive prefix for tile_find).  Block 0 of the grid reports sequences
+// whose rows fall outside the cache.
+__device__ __forceinline__ int tile_count(const DecodeArgs& a, int* scan) {
   const int tid = threadIdx.x, nthr = blockDim.x;
   const int per = (a.B + nthr - 1) / nthr;
   const int b0 = tid * per;
@@ -139,30 +140,53 @@ __device__ __forceinline__ void tile_scan(const DecodeArgs& a, int* scan, int n_
     scan[tid] += v;
     __syncthreads();
   }
-  const int NT = scan[nthr - 1];
-  const int x0 = item_begin(blockIdx.x, NT, n_items);
-  int run = tid ? scan[tid - 1] : 0;
-  __syncthreads();
+  return scan[nthr - 1];
+}
+
+// Block-wide lookup (after tile_count, same scan): the sequence owning
+// flattened tile x and its first tile; (B, NT) when no sequence does.
+__device__ __forceinline__ void tile_find(const DecodeArgs& a, const int* scan, int x, int& b_out, int& pre_out) {
+  const int tid = threadIdx.x, nthr = blockDim.x;
+  const int per = (a.B + nthr - 1) / nthr;
+  const int b0 = tid * per;
   __shared__ int s_bf, s_pf;
   if (tid == 0) {
     s_bf = a.B;
-    s_pf = NT;
+    s_pf = scan[nthr - 1];
   }
   __syncthreads();
+  int run = tid ? scan[tid - 1] : 0;
   for (int b = b0; b < b0 + per && b < a.B; ++b) {
     const int nt = ntiles_of(a, b);
-    if (nt > 0 && x0 >= run && x0 < run + nt) {
+    if (nt > 0 && x >= run && x < run + nt) {
       s_bf = b;
       s_pf = run;
     }
     run += nt;
   }
   __syncthreads();
-  NT_out = NT;
-  b_first = s_bf;
-  pre_first = s_pf;
+  b_out = s_bf;
+  pre_out = s_pf;
   __syncthreads();
 }
+
+// Work split of the tensor-core kernels.  With n CTAs and NT tiles, fewer than
+// kFineSplitBelow per CTA, every CTA takes floor(NT / n) whole tiles (the main
+// tiles [0, NTm), in contiguous ranges) and the R = NT - NTm extra tiles are
+// shared out more finely, so that no CTA carries a whole tile more than
+// another (with more tiles per CTA, that imbalance is small and NTm = NT): the scores kernel splits them
+// into their units (CTA c: units [c XU / n, (c+1) XU / n) of the flattened
+// (extra tile, unit) list, XU = R U), the absorption kernel hands out whole
+// extra tiles.  Every extra tile is a segment of its own (its own partial slot
+// extra_base + e, e = x - NTm), so its heads' softmax state never spans CTAs.
+struct Split {
+  int NT, NTm, R;
+  __device__ Split(int nt, int n, bool extra) : NT(nt), NTm(main_tiles(nt, n, extra)), R(NT - NTm) {}
+  __device__ int main_begin(int c, int n) const { return item_begin(c, NTm, n); }
+};
+
+// First partial slot of the extra tiles: after the main slots c + b.
+__host__ __device__ inline int64_t extra_slot_base(int n_items, int batch) { return (int64_t)n_items + batch - 1; }
 
 // Most 128-token tiles a call can have with non-overlapping sequences: the
 // per-tile probability and reference-max stores of the tensor-core path are

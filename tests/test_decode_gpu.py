@@ -119,6 +119,24 @@ def test_full_size_configs_sampled(cfg):
     assert np.isfinite(got).all()
 
 
+@pytest.mark.parametrize("cfg", [1, 2])
+@pytest.mark.parametrize("extra", [5, -1])
+def test_leftover_tiles_split_finely(cfg, extra):
+    """More 128-token tiles than SMs: whole tiles per SM, then the leftover tiles
+    shared out by groups of heads (scores) and r_v chunks (absorption), each with
+    its own partial slot.  extra = -1: one tile short of two per SM."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    nt = sms + (extra if extra > 0 else sms - 1)
+    lens = (64 * 128, (nt - 64 - 1) * 128 + 77)
+    spec = S.workload(cfg).layer
+    di = S.make_decode_inputs(spec, lens, seed=21 + cfg)
+    got, _ = gpu_decode(spec, lens, di=di)
+    for b, j in _sample_pairs(2, spec.n_q_heads, 8, cfg + 40):
+        ref = oracle_decode(di, heads=[j], batch_ids=[b])
+        assert_parity(got[b:b + 1, j:j + 1], ref[b:b + 1, j:j + 1], "bf16", f"cfg{cfg} nt{nt} b{b} j{j}")
+    assert np.isfinite(got).all()
+
+
 @pytest.mark.parametrize("batch", [1, 8, 32, 64])
 def test_32_layer_ragged_sampled(batch):
     """32-layer ragged workload: device-generated inputs (checked bit-exact against the host
