@@ -104,8 +104,11 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 template <bool kFold>
 struct Ring {
-  static constexpr int NW = kFold ? 4 : 3;  // factor-item slots (key mode keeps 16 KB for queries)
-  static constexpr int kMma = kFold ? 2 : 1;  // MMA-issuing threads, each with its own factor ring
+  static constexpr int NW = 4;                // factor-item slots
+  // MMA-issuing threads, each with its own factor ring: two in query-folded
+  // mode; key mode's units carry up to four items, which one thread's ring of
+  // all four slots streams better
+  static constexpr int kMma = kFold ? 2 : 1;
   static constexpr int NWt = NW / kMma;       // slots of one MMA thread's ring
   static constexpr int kThreads = kFold ? 384 : 352;
 };
@@ -162,7 +165,6 @@ struct Smem {
   int16_t order[kMaxHqTc];
   int16_t uitem[kMaxUnits + 1];
   int8_t hunit[kMaxHqTc];
-  uint32_t item[kMaxItems];
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -175,7 +177,8 @@ __device__ __forceinline__ uint32_t swz_of(int w) { return w == 64 ? kSw128 : (w
 
 template <bool kFold>
 __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
-    decode_tc_kernel(const __grid_constant__ Maps maps, const LayerTable lt, const DecodeArgs a, const TcArgs ta) {
+    decode_tc_kernel(const __grid_constant__ Maps maps, const LayerTable lt, const DecodeArgs a,
+                     const __grid_constant__ TcArgs ta) {
   constexpr int NW = Ring<kFold>::NW, kMma = Ring<kFold>::kMma, NWt = Ring<kFold>::NWt;
   constexpr int kThreads = Ring<kFold>::kThreads;
   extern __shared__ uint8_t smem_raw[];
@@ -213,7 +216,6 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
   if (tid < lt.Hkv) sm.order[tid] = ta.order[tid];
   if (tid <= ta.n_units) sm.uitem[tid] = ta.uitem[tid];
   if (tid < Hq) sm.hunit[tid] = ta.hunit[tid];
-  for (int n = tid; n < ta.n_items; n += kThreads) sm.item[n] = ta.item[n];
   if (tid < kD / 2) {
     sm.om64[tid] = ta.om[tid];
     sm.om32[tid] = (float)ta.om[tid];
@@ -266,7 +268,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
       DCK_TC_TRACE(30 + nb);
       if (lane < nb) {
         const int sl = rw * NWt + (wc + lane) % NWt;
-        const uint32_t it = sm.item[n + p0 + lane];
+        const uint32_t it = ta.item[n + p0 + lane];
         const uint32_t bytes = (it >> 26) << 12;
         mbar_expect_tx(&sm.w_full[sl], bytes);
         bulk_load(sm.w[sl], img + (it & 0x03FFFFFFu), bytes, &sm.w_full[sl], pol);
@@ -355,7 +357,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
                 if (!ok) break;
                 if (lane < nb) {
                   const int sl = (w_cnt + lane) % NW;
-                  const uint32_t it = sm.item[n0 + lane];
+                  const uint32_t it = ta.item[n0 + lane];
                   const uint32_t bytes = (it >> 26) << 12;
                   mbar_expect_tx(&sm.w_full[sl], bytes);
                   bulk_load(sm.w[sl], img + (it & 0x03FFFFFFu), bytes, &sm.w_full[sl], pol);
@@ -595,14 +597,29 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
                     if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
                   }
 #pragma unroll
-                  for (int i2 = 0; i2 < 16; ++i2) {
-                    const int ip = 16 * ps + i2;
-                    const float r1 = fmaf(k1v[i2], cs[ip], -k2v[i2] * sn[ip]);
-                    const float r2 = fmaf(k1v[i2], sn[ip], k2v[i2] * cs[ip]);
-                    const float* qrow = sm.qr + j0 * kD + 32 * hf + ip;
+                  for (int i4 = 0; i4 < 16; i4 += 4) {
+                    // four rotated frequency pairs, then each query head's matching
+                    // halves with two 16-byte shared loads
+                    float r1[4], r2[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                      const int ip = 16 * ps + i4 + u;
+                      r1[u] = fmaf(k1v[i4 + u], cs[ip], -k2v[i4 + u] * sn[ip]);
+                      r2[u] = fmaf(k1v[i4 + u], sn[ip], k2v[i4 + u] * cs[ip]);
+                    }
+                    const float* qrow = sm.qr + j0 * kD + 32 * hf + 16 * ps + i4;
 #pragma unroll
                     for (int jj = 0; jj < kMaxQPerKv; ++jj)
-                      if (jj < qpg) part[jj] = fmaf(qrow[jj * kD], r1, fmaf(qrow[jj * kD + 64], r2, part[jj]));
+                      if (jj < qpg) {
+                        const float4 qa = *reinterpret_cast<const float4*>(qrow + jj * kD);
+                        const float4 qb = *reinterpret_cast<const float4*>(qrow + jj * kD + 64);
+                        float v = part[jj];
+                        v = fmaf(qa.x, r1[0], fmaf(qb.x, r2[0], v));
+                        v = fmaf(qa.y, r1[1], fmaf(qb.y, r2[1], v));
+                        v = fmaf(qa.z, r1[2], fmaf(qb.z, r2[2], v));
+                        v = fmaf(qa.w, r1[3], fmaf(qb.w, r2[3], v));
+                        part[jj] = v;
+                      }
                   }
                 }
 #pragma unroll
