@@ -20,6 +20,7 @@
 // owned by one thread.  The cluster adds the partial outputs through
 // distributed shared memory, every rank reducing and writing a share of o.
 #include <algorithm>
+#include <type_traits>
 
 #include <cooperative_groups.h>
 
@@ -43,6 +44,27 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
+__device__ __forceinline__ uint32_t f32_to_tf32(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+  return r;
+}
+// d += a b for one 16 x 8 x 8 tile, tf32 inputs, fp32 accumulators.
+__device__ __forceinline__ void mma_tf32(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Row stride (elements) of the staged B_v rows: padded by 16 bytes on the
+// tensor-core path, whose fragments read four rows at one column.
+template <typename T, int D>
+__host__ __device__ constexpr int ldb() {
+  return D + (std::is_same<T, __nv_bfloat16>::value && D == 128 ? 8 : 0);
+}
+
 // Two adjacent elements (16-byte aligned row, even column) as floats.
 __device__ __forceinline__ float2 pair_f32(const float* p) { return *reinterpret_cast<const float2*>(p); }
 __device__ __forceinline__ float2 pair_f32(const __nv_bfloat16* p) {
@@ -64,11 +86,12 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   const int rr = rv / split;            // rows of u / B_v owned by this CTA (a multiple of 4)
   const int r0 = rank * rr;
 
-  // shared layout: B_v rows [rr][D] T | u rows [kMaxRows][rr] | received partial o [split][kMaxRows * D / split]
+  // shared layout: B_v rows [rr][ldb] T | u rows [kMaxRows][rr + 4] | received partial o [split][kMaxRows * D / split]
   // | 1/l | row slot ranges [kMaxRows][4] | scan | prefix | item starts [n_items + 1]
   T* sbv = reinterpret_cast<T*>(smem_c);
-  float* su = reinterpret_cast<float*>(smem_c + (size_t)rr * D * sizeof(T));
-  float* so = su + (size_t)kMaxRows * rr;
+  float* su = reinterpret_cast<float*>(smem_c + (size_t)rr * ldb<T, D>() * sizeof(T));
+  const int ldu = rr + 4;  // padded u rows: the tensor-core fragments read 8 rows at one column
+  float* so = su + (size_t)kMaxRows * ldu;
   float* sinv = so + kMaxRows * D;
   int* rc = reinterpret_cast<int*>(sinv + kMaxRows);
   int* scan = rc + 4 * kMaxRows;
@@ -82,7 +105,7 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
     constexpr int kSegRow = D * (int)sizeof(T) / 16;
     for (int i = threadIdx.x; i < rr * kSegRow; i += kThreads) {
       const int r = i / kSegRow, c = i % kSegRow;
-      cp_async16(reinterpret_cast<uint8_t*>(sbv + (size_t)r * D) + c * 16,
+      cp_async16(reinterpret_cast<uint8_t*>(sbv + (size_t)r * ldb<T, D>()) + c * 16,
                  reinterpret_cast<const uint8_t*>(Bv + (int64_t)(r0 + r) * ldv) + c * 16);
     }
     cp_async_commit();
@@ -157,11 +180,45 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
         M = Mb;
       }
     }
-    reinterpret_cast<float4*>(su + (size_t)i * rr)[r4] = acc;
+    reinterpret_cast<float4*>(su + (size_t)i * ldu)[r4] = acc;
     if (r4 == 0) sinv[i] = l > 0.f ? 1.f / l : 0.f;
   }
   cp_async_wait_all();
   __syncthreads();
+  const int share = kMaxRows * D / split;
+  if constexpr (std::is_same<T, __nv_bfloat16>::value && D == 128) {
+    // partial o over this CTA's rows of B_v on the tensor cores: o[16 x 128] =
+    // u[16 x rr] B_v[rr x 128], mma m16n8k8 tf32 (B_v's bf16 converts exactly;
+    // u rounds to tf32, a relative 2^-11); warp w owns columns [16 w, 16 w + 16)
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int gid = lane >> 2, tig = lane & 3;
+    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    for (int k0 = 0; k0 < rr; k0 += 8) {
+      uint32_t af[4];
+      af[0] = f32_to_tf32(su[(size_t)gid * ldu + k0 + tig]);
+      af[1] = f32_to_tf32(su[(size_t)(gid + 8) * ldu + k0 + tig]);
+      af[2] = f32_to_tf32(su[(size_t)gid * ldu + k0 + tig + 4]);
+      af[3] = f32_to_tf32(su[(size_t)(gid + 8) * ldu + k0 + tig + 4]);
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+        const int col = 16 * warp + 8 * nt + gid;
+        const uint32_t b0 = (uint32_t)__bfloat16_as_ushort(sbv[(size_t)(k0 + tig) * ldb<T, D>() + col]) << 16;
+        const uint32_t b1 = (uint32_t)__bfloat16_as_ushort(sbv[(size_t)(k0 + tig + 4) * ldb<T, D>() + col]) << 16;
+        mma_tf32(acc[nt], af, b0, b1);
+      }
+    }
+    // outputs (row, col): this thread has rows gid, gid + 8 and columns 2 tig, 2 tig + 1 of each n-tile
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int i = gid + 8 * (q >> 1), col = 16 * warp + 8 * nt + 2 * tig + (q & 1);
+        if (i < nrow) {
+          const int e = i * D + col;
+          cluster.map_shared_rank(so, e % split)[rank * share + e / split] = acc[nt][q];
+        }
+      }
+  } else {
   // partial o over this CTA's rows of B_v: thread = (column pair, every
   // kGroups-th row of the chunk), so each output has one owner
   constexpr int kPairs = D / 2;
@@ -175,7 +232,7 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
     float x0[4], x1[4];
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
-      const float2 xv = pair_f32(sbv + (size_t)(r + t) * D + 2 * cp);
+      const float2 xv = pair_f32(sbv + (size_t)(r + t) * ldb<T, D>() + 2 * cp);
       x0[t] = xv.x;
       x1[t] = xv.y;
     }
@@ -183,7 +240,7 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
     for (int q = 0; q < kRowsPer; ++q) {
       const int i = ig + kGroups * q;
       if (i < nrow) {
-        const float4 uv = *reinterpret_cast<const float4*>(&su[(size_t)i * rr + r]);
+        const float4 uv = *reinterpret_cast<const float4*>(&su[(size_t)i * ldu + r]);
         acc[q][0] = fmaf(uv.x, x0[0], fmaf(uv.y, x0[1], fmaf(uv.z, x0[2], fmaf(uv.w, x0[3], acc[q][0]))));
         acc[q][1] = fmaf(uv.x, x1[0], fmaf(uv.y, x1[1], fmaf(uv.z, x1[2], fmaf(uv.w, x1[3], acc[q][1]))));
       }
@@ -192,7 +249,6 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   // cluster-wide sum: output e = i * D + col belongs to rank e % split, which
   // receives every rank's partial in its slot [rank][e / split] (remote stores,
   // made visible by the cluster barrier), then reduces and writes its outputs
-  const int share = kMaxRows * D / split;
 #pragma unroll
   for (int q = 0; q < kRowsPer; ++q) {
     const int i = ig + kGroups * q;
@@ -202,6 +258,7 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
         const int e = i * D + 2 * cp + t;
         cluster.map_shared_rank(so, e % split)[rank * share + e / split] = acc[q][t];
       }
+  }
   }
   cluster.sync();
   T* out = static_cast<T*>(a.out);
@@ -225,8 +282,8 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   // as many sequences per cluster as its rows allow: each head's B_v block is staged once per chunk
   const int bchunk = std::max(1, std::min(a.B, kMaxRows / lt.qpg));
   const int rr = lt.rv / split;
-  const size_t smem = (size_t)rr * D * sizeof(T) +
-                      sizeof(float) * ((size_t)kMaxRows * rr + kMaxRows * D + kMaxRows) +
+  const size_t smem = (size_t)rr * ldb<T, D>() * sizeof(T) +
+                      sizeof(float) * ((size_t)kMaxRows * (rr + 4) + kMaxRows * D + kMaxRows) +
                       sizeof(int) * (4 * kMaxRows + kThreads + a.B + 1 + a.n_items + 1);
   auto k = combine_kernel<T, D>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
