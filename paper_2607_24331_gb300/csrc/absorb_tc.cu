@@ -83,6 +83,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
   const int Hq = lt.Hq, hq_pad = aa.hq_pad, n_chunks = aa.n_chunks;
   const uint32_t pbytes = (uint32_t)hq_pad * 256;
   DCK_AB_TRACE(99);
+  griddep_launch();  // the combine kernel may stage its factors as CTAs finish
 
   if (tid == 0) {
     for (int i = 0; i < kNVs; ++i) {

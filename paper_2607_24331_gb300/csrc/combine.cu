@@ -130,6 +130,11 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   }
   __syncthreads();
 
+  // Launched under programmatic dependent launch: everything above reads only the
+  // call's inputs; the partials come from the kernels before, complete once the
+  // preceding grid is.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+
   // u rows restricted to [r0, r0 + rr), merged over the items in one pass with
   // a running reference max: each thread owns float4 columns of whole rows and
   // keeps kItemBatch items' loads in flight.  Every thread of a row sees the
@@ -293,13 +298,16 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = split;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  // may start while the previous kernel finishes (B_v staging and tables overlap it)
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, k, lt, a, bchunk, split);
 }
 
