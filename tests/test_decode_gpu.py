@@ -119,6 +119,27 @@ def test_full_size_configs_sampled(cfg):
     assert np.isfinite(got).all()
 
 
+# Layers beyond the benchmark configs that the tensor-core path takes: a head
+# count that pads to the MMA width (24 -> 32), two and eight query heads per KV
+# head, and ranks whose latent pieces include 32- and 16-column widths.
+TC_SHAPES = {
+    "mha24_pad": S.LayerSpec(1024, 24, 24, 128, ((0, 1, 2, 3, 4, 5), (6, 7, 8, 9, 10, 11, 12, 13),
+                                                  tuple(range(14, 24))), (64, 128, 80), 256, "bf16", 1e4),
+    "gqa_qpg2": S.LayerSpec(2048, 16, 8, 128, ((0, 1), (2, 3, 4), (5, 6, 7)), (96, 160, 48), 384, "bf16", 5e5),
+    "gqa_qpg8": S.LayerSpec(2048, 32, 4, 128, ((0, 1), (2, 3)), (112, 64), 128, "bf16", 1e6),
+}
+
+
+@pytest.mark.parametrize("name", sorted(TC_SHAPES))
+def test_tensor_core_layer_shapes(name):
+    spec = TC_SHAPES[name]
+    lens = (1, 200, 700, 129)
+    got, di = gpu_decode(spec, lens, seed=17, q_std=3.0)
+    n = dck.dck_last_launch_count()
+    assert n == 4, f"the tensor-core path (factor preparation, scores, absorption, combine) did not run: {n} launches"
+    assert_parity(got, oracle_decode(di), "bf16", name)
+
+
 @pytest.mark.parametrize("cfg", [1, 2])
 @pytest.mark.parametrize("extra", [5, -1])
 def test_leftover_tiles_split_finely(cfg, extra):
