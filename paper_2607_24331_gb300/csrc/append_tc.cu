@@ -8,8 +8,8 @@
 // swizzle) through a 4-deep mbarrier ring.  Warp 0 issues TMA, warp 1 owns
 // TMEM and issues tcgen05.mma, warps 2-5 drain the accumulator (one TMEM lane
 // quadrant each).  Small batches (<= 256 tokens, the decode-step append) split
-// K over CTAs, accumulate fp32 partials with red.add in the caller's workspace
-// and a second kernel rounds and scatters them.
+// K over CTAs, each storing its fp32 partial in its own slice of the caller's
+// workspace; a second kernel sums the slices, rounds and scatters.
 #include "common.cuh"
 #include "sm100.cuh"
 #include "tmap.h"
@@ -25,6 +25,7 @@ constexpr int kBBytes = kBK * kMaxBN * 2;       // 32 KB
 constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kThreads = 192;
 constexpr int kSplitMaxTok = 256;
+constexpr int kMaxSplit = 16;  // K splits of a small batch
 
 struct AppendParams {
   int n_tok, D, Rk, rv;
@@ -35,7 +36,7 @@ struct AppendParams {
   __nv_bfloat16* kc;
   __nv_bfloat16* vc;
   int64_t n_rows;
-  float* ws;     // split-K accumulator [n_tok][Rk + rv] (ksplit > 1)
+  float* ws;     // split-K partials [ksplit][n_tok][Rk + rv] (ksplit > 1)
   int* err;
 };
 
@@ -145,9 +146,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           o[1] = pk[1];
         }
       } else {
-        float* w = p.ws + (int64_t)m * (p.Rk + p.rv) + (is_k ? 0 : p.Rk) + n0 + c;
+        float4* w = reinterpret_cast<float4*>(p.ws + ((int64_t)blockIdx.z * p.n_tok + m) * (p.Rk + p.rv) +
+                                              (is_k ? 0 : p.Rk) + n0 + c);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) atomicAdd(w + i, v[i]);
+        for (int i = 0; i < 4; ++i) w[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
       }
     }
   }
@@ -160,7 +162,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0 && *abort_flag) atomicOr(p.err, kErrTimeout);
 }
 
-__global__ void append_finalize_kernel(const float* __restrict__ ws, int n_tok, int Rk, int rv,
+__global__ void append_finalize_kernel(const float* __restrict__ ws, int n_tok, int Rk, int rv, int ksplit,
                                        const int64_t* __restrict__ rows, __nv_bfloat16* kc, __nv_bfloat16* vc,
                                        int64_t n_rows, int* err) {
   const int N = Rk + rv;
@@ -171,7 +173,8 @@ __global__ void append_finalize_kernel(const float* __restrict__ ws, int n_tok, 
     return;
   }
   for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < N; c += gridDim.x * blockDim.x) {
-    const float v = ws[(int64_t)m * N + c];
+    float v = 0.f;
+    for (int z = 0; z < ksplit; ++z) v += ws[((int64_t)z * n_tok + m) * N + c];
     if (c < Rk) kc[row * Rk + c] = __float2bfloat16_rn(v);
     else vc[row * rv + (c - Rk)] = __float2bfloat16_rn(v);
   }
@@ -183,7 +186,7 @@ int plan_ksplit(int n_tok, int D, int Rk, int rv, int sms) {
   const int ntiles = (Rk + kMaxBN - 1) / kMaxBN + (rv + kMaxBN - 1) / kMaxBN;
   const int kblocks = (D + kBK - 1) / kBK;
   int ks = sms / max(1, mt * ntiles);
-  ks = max(1, min(ks, min(16, kblocks)));
+  ks = max(1, min(ks, min(kMaxSplit, kblocks)));
   return ks;
 }
 
@@ -194,7 +197,7 @@ bool tc_append_supports(int D, int Rk, int rv, int dtype) {
 }
 
 size_t tc_append_workspace(int n_tok, int Rk, int rv) {
-  return n_tok <= kSplitMaxTok ? align_up((size_t)n_tok * (Rk + rv) * sizeof(float), 256) : 0;
+  return n_tok <= kSplitMaxTok ? align_up((size_t)kMaxSplit * n_tok * (Rk + rv) * sizeof(float), 256) : 0;
 }
 
 cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, const void* A_v, int Rk, int rv,
@@ -227,16 +230,12 @@ cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, c
   const size_t smem = kStages * kStageBytes + 1024 + 256;
   cudaError_t e = cudaFuncSetAttribute(append_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  if (p.ksplit > 1) {
-    e = cudaMemsetAsync(ws, 0, (size_t)n_tok * (Rk + rv) * sizeof(float), s);
-    if (e != cudaSuccess) return e;
-  }
   dim3 grid(ntiles, (n_tok + kBM - 1) / kBM, p.ksplit);
   append_tc_kernel<<<grid, kThreads, smem, s>>>(tx, tk, tv, p);
   e = cudaGetLastError();
   if (e != cudaSuccess || p.ksplit == 1) return e;
   dim3 g2((Rk + rv + 255) / 256, n_tok);
-  append_finalize_kernel<<<g2, 256, 0, s>>>(p.ws, n_tok, Rk, rv, rows, p.kc, p.vc, n_rows, err);
+  append_finalize_kernel<<<g2, 256, 0, s>>>(p.ws, n_tok, Rk, rv, p.ksplit, rows, p.kc, p.vc, n_rows, err);
   return cudaGetLastError();
 }
 
