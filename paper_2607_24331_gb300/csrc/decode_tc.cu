@@ -94,8 +94,6 @@ constexpr int kMaxPieces = 5;
 constexpr int kMaxHqTc = 32;
 constexpr int kMaxItems = 256;
 constexpr int kMaxUnits = 32;
-constexpr int kPrepThreads = 256;
-constexpr int kPrepIters = 8;  // 16-byte chunks per preparation thread: items hold <= 2 x 64 x 16
 constexpr int kEpiThreads = 256;
 constexpr float kRescaleThr = 8.f;  // log2 units: probabilities stay <= 256
 constexpr uint32_t kTmemCols = 512;
@@ -752,49 +750,24 @@ struct PrepArgs {
 //   a_i B[:, i] + b_i B[:, i+64]  and  b_i B[:, i] - a_i B[:, i+64]
 // with (a, b) the halves of RoPE(q_{b,h}, L_b - 1) * log2(e)/sqrt(d).
 template <bool kFold>
-__global__ void __launch_bounds__(kPrepThreads) factor_prep_kernel(const LayerTable lt, const DecodeArgs a, const PrepArgs pa,
+__global__ void __launch_bounds__(256) factor_prep_kernel(const LayerTable lt, const DecodeArgs a, const PrepArgs pa,
                                                           uint8_t* __restrict__ img) {
   griddep_launch();
   const int n = blockIdx.x, b = blockIdx.y;
   const PrepItem it = pa.item[n];
   const int g = it.g, ws = it.ws, nh = it.nh;
   __shared__ float qa[2][kD / 2], qb[2][kD / 2];
-  const int total = nh * ws * 16;  // 16-byte output chunks, at most kPrepIters per thread
-  const int64_t ld = (int64_t)lt.grp_nh[g] * kD;
-  const __nv_bfloat16* __restrict__ Bg = static_cast<const __nv_bfloat16*>(a.Bk) + lt.grp_boff[g] + it.s0 * kD;
-  // thread -> (head, row, 8-column chunk): nh x ws rows x 16 chunks (2 halves x 8).
-  // The factor values are loaded first, so that their latency overlaps the
-  // rotated query's.  Query-folded mode: chunk (half, c8) holds the pairs
-  // i = 32 half + 4 c8 .. +3, i.e. B[k][i..i+3] and B[k][64+i..]; key mode copies
-  // the 8 columns 64 half + 8 c8 .. +7.
-  uint4 raw[kPrepIters];
-#pragma unroll
-  for (int q = 0; q < kPrepIters; ++q) {
-    const int idx = threadIdx.x + q * blockDim.x;
-    raw[q] = make_uint4(0, 0, 0, 0);
-    if (idx < total) {
-      const int hh = idx / (ws * 16), r = (idx >> 4) % ws, ch = idx & 15;
-      const __nv_bfloat16* row = Bg + hh * kD + (int64_t)(it.k0 + r) * ld;
-      if (kFold) {
-        const int i0 = 32 * (ch >> 3) + 4 * (ch & 7);
-        const uint2 x = *reinterpret_cast<const uint2*>(row + i0);
-        const uint2 y = *reinterpret_cast<const uint2*>(row + kD / 2 + i0);
-        raw[q] = make_uint4(x.x, x.y, y.x, y.y);
-      } else {
-        raw[q] = *reinterpret_cast<const uint4*>(row + 8 * ch);
-      }
-    }
-  }
   if (kFold) {
     const int L = valid_len(a.seq_len, a.seq_start, b, a.n_rows);
     if (L == 0) return;  // no tile of this sequence is ever processed
     if (threadIdx.x < nh * (kD / 2)) {
       const int hh = threadIdx.x / (kD / 2), i = threadIdx.x % (kD / 2);
+      const int kv = it.kv[hh];
       // angle (L-1) w_i reduced mod 2 pi in fp64, sine and cosine in fp32
       const double ang = (double)(L - 1) * pa.om[i];
       float sn, cs;
       sincosf((float)(ang - 6.283185307179586 * rint(ang * 0.15915494309189535)), &sn, &cs);
-      const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(a.q) + ((int64_t)b * lt.Hq + it.kv[hh]) * kD;
+      const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(a.q) + ((int64_t)b * lt.Hq + kv) * kD;
       const float x1 = __bfloat162float(q[i]), x2 = __bfloat162float(q[i + kD / 2]);
       const float sc = kLog2e * rsqrtf((float)kD);
       qa[hh][i] = (x1 * cs - x2 * sn) * sc;
@@ -802,31 +775,36 @@ __global__ void __launch_bounds__(kPrepThreads) factor_prep_kernel(const LayerTa
     }
     __syncthreads();
   }
+  const int64_t ld = (int64_t)lt.grp_nh[g] * kD;
   uint8_t* dst = img + (kFold ? (int64_t)b * pa.seq_bytes : 0) + it.off;
-#pragma unroll
-  for (int q = 0; q < kPrepIters; ++q) {
-    const int idx = threadIdx.x + q * blockDim.x;
-    if (idx >= total) break;
+  // thread -> (head, row, 8-column chunk): nh x ws rows x 16 chunks (2 halves x 8)
+  for (int idx = threadIdx.x; idx < nh * ws * 16; idx += blockDim.x) {
     const int hh = idx / (ws * 16), r = (idx >> 4) % ws, ch = idx & 15;
     const int half = ch >> 3, c8 = ch & 7;
-    uint4 out = raw[q];
+    const __nv_bfloat16* __restrict__ Bs =
+        static_cast<const __nv_bfloat16*>(a.Bk) + lt.grp_boff[g] + (it.s0 + hh) * kD;
+    const int k = it.k0 + r;
+    float v[8];
     if (kFold) {
-      // output columns 2i, 2i+1 of the pairs i = i0 .. i0+3 (a bf16 is the top
-      // half of the fp32 with the same value)
-      const int i0 = 32 * half + 4 * c8;
-      const uint32_t xw[2] = {raw[q].x, raw[q].y}, yw[2] = {raw[q].z, raw[q].w};
-      uint32_t ow[4];
+      // output columns col = 64*half + 8*c8 + t, t even/odd -> pair i = col/2
 #pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        const uint32_t xb = xw[t >> 1], yb = yw[t >> 1];
-        const float x = __uint_as_float((t & 1) ? (xb & 0xffff0000u) : (xb << 16));
-        const float y = __uint_as_float((t & 1) ? (yb & 0xffff0000u) : (yb << 16));
-        const float A = qa[hh][i0 + t], Bq = qb[hh][i0 + t];
-        const __nv_bfloat162 o = __floats2bfloat162_rn(fmaf(A, x, Bq * y), fmaf(Bq, x, -A * y));
-        ow[t] = (uint32_t)__bfloat16_as_ushort(o.x) | ((uint32_t)__bfloat16_as_ushort(o.y) << 16);
+      for (int t = 0; t < 8; t += 2) {
+        const int i = (64 * half + 8 * c8 + t) >> 1;
+        const float x = __bfloat162float(Bs[k * ld + i]);
+        const float y = __bfloat162float(Bs[k * ld + kD / 2 + i]);
+        v[t] = fmaf(qa[hh][i], x, qb[hh][i] * y);
+        v[t + 1] = fmaf(qb[hh][i], x, -qa[hh][i] * y);
       }
-      out = make_uint4(ow[0], ow[1], ow[2], ow[3]);
+    } else {
+      const uint4 raw = *reinterpret_cast<const uint4*>(Bs + k * ld + 64 * half + 8 * c8);
+      const __nv_bfloat16* h8 = reinterpret_cast<const __nv_bfloat16*>(&raw);
+#pragma unroll
+      for (int t = 0; t < 8; ++t) v[t] = __bfloat162float(h8[t]);
     }
+    uint4 out;
+    __nv_bfloat162* o2 = reinterpret_cast<__nv_bfloat162*>(&out);
+#pragma unroll
+    for (int t = 0; t < 4; ++t) o2[t] = __floats2bfloat162_rn(v[2 * t], v[2 * t + 1]);
     *reinterpret_cast<uint4*>(dst + (hh * 2 + half) * (ws * 128) + r * 128 + ((c8 ^ (r & 7)) << 4)) = out;
   }
 }
@@ -892,9 +870,7 @@ cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& m
     if (e != cudaSuccess) return e;
     if (dev_ok) attr_done[dev] = 1;
   }
-  // one block per item, a thread per 16-byte chunk of it (2 x 64 ranks x 16 chunks
-  // for the largest items): the factor loads of a thread are all in flight at once
-  factor_prep_kernel<kFold><<<dim3(pa.n_items, kFold ? a.B : 1), kPrepThreads, 0, s>>>(lt, a, pa,
+  factor_prep_kernel<kFold><<<dim3(pa.n_items, kFold ? a.B : 1), 256, 0, s>>>(lt, a, pa,
                                                                                 static_cast<uint8_t*>(a.extra));
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
