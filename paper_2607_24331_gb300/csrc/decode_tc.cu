@@ -153,7 +153,9 @@ template <bool kFold>
 struct Smem {
   uint8_t a[kNA][kSlot];
   uint8_t w[Ring<kFold>::NW][kSlotW];
-  float x[kMaxHqTc * 128];                  // scores [head][token], accumulated atomically
+  // scores [head][token]: query-folded mode keeps one array per frequency half
+  // (plain stores, summed at the tile end); key mode accumulates atomically
+  float x[kFold ? 2 * kMaxHqTc * 128 : kMaxHqTc * 128];
   float qr[kFold ? 1 : kMaxHqTc * kD];      // key mode: rotated queries * log2(e)/sqrt(d)
   double om64[kD / 2];
   float om32[kD / 2];
@@ -251,7 +253,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
       ub = min(u_hi - e * U, U);
     }
   };
-  for (int i = tid; i < kMaxHqTc * 128; i += kThreads) sm.x[i] = 0.f;
+  for (int i = tid; i < (int)(sizeof(sm.x) / sizeof(float)); i += kThreads) sm.x[i] = 0.f;
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -573,9 +575,9 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
                     pa[1][i2 & 3] =
                         fmaf(cs[16 * ps + i2], y1[2 * i2], fmaf(sn[16 * ps + i2], y1[2 * i2 + 1], pa[1][i2 & 3]));
               }
-              atomicAdd(&sm.x[sm.order[gs.h0 + 2 * u] * 128 + tau], (pa[0][0] + pa[0][1]) + (pa[0][2] + pa[0][3]));
-              if (nh == 2)
-                atomicAdd(&sm.x[sm.order[gs.h0 + 2 * u + 1] * 128 + tau], (pa[1][0] + pa[1][1]) + (pa[1][2] + pa[1][3]));
+              float* xh = sm.x + hf * (kMaxHqTc * 128);  // this frequency half's scores
+              xh[sm.order[gs.h0 + 2 * u] * 128 + tau] = (pa[0][0] + pa[0][1]) + (pa[0][2] + pa[0][3]);
+              if (nh == 2) xh[sm.order[gs.h0 + 2 * u + 1] * 128 + tau] = (pa[1][0] + pa[1][1]) + (pa[1][2] + pa[1][3]);
             } else {
               for (int hh = 0; hh < nh; ++hh) {
                 const int j0 = sm.order[gs.h0 + 2 * u + hh] * qpg;
@@ -641,14 +643,19 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
           const int tb = 16 * ct;  // first token of this owner
           float sc[16];
           float4* xr = reinterpret_cast<float4*>(&sm.x[jt * 128 + tb]);
+          const float4* xr2 = reinterpret_cast<const float4*>(&sm.x[(kFold ? kMaxHqTc * 128 : 0) + jt * 128 + tb]);
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
-            const float4 v = own ? xr[q] : make_float4(0.f, 0.f, 0.f, 0.f);
+            float4 v = own ? xr[q] : make_float4(0.f, 0.f, 0.f, 0.f);
+            if (kFold && own) {  // the other frequency half (every score is stored each tile)
+              const float4 w = xr2[q];
+              v = make_float4(v.x + w.x, v.y + w.y, v.z + w.z, v.w + w.w);
+            }
             sc[4 * q] = v.x;
             sc[4 * q + 1] = v.y;
             sc[4 * q + 2] = v.z;
             sc[4 * q + 3] = v.w;
-            if (own) xr[q] = make_float4(0.f, 0.f, 0.f, 0.f);  // ready for the next tile
+            if (!kFold && own) xr[q] = make_float4(0.f, 0.f, 0.f, 0.f);  // key mode: ready for the next tile's sums
           }
           const int nv = max(0, min(16, seg.t_end - (t0 + tb)));  // tokens inside the sequence
           float mx = -INFINITY;
