@@ -83,6 +83,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // programmatic dependent launch: the set-up above overlaps the previous
+  // kernel's tail; every global access comes after that kernel is complete
+  pdl_wait();
+  pdl_launch_dependents();
   const uint32_t tmem = *tmem_slot;
   const CUtensorMap* tmb = is_k ? &tm_ak : &tm_av;
 
@@ -165,6 +169,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 __global__ void append_finalize_kernel(const float* __restrict__ ws, int n_tok, int Rk, int rv, int ksplit,
                                        const int64_t* __restrict__ rows, __nv_bfloat16* kc, __nv_bfloat16* vc,
                                        int64_t n_rows, int* err) {
+  pdl_wait();  // the split partials come from the kernel before
+  pdl_launch_dependents();
   const int N = Rk + rv;
   const int m = blockIdx.y;
   const int64_t row = rows[m];
@@ -231,12 +237,11 @@ cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, c
   cudaError_t e = cudaFuncSetAttribute(append_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid(ntiles, (n_tok + kBM - 1) / kBM, p.ksplit);
-  append_tc_kernel<<<grid, kThreads, smem, s>>>(tx, tk, tv, p);
-  e = cudaGetLastError();
+  e = launch_pdl(append_tc_kernel, grid, dim3(kThreads), smem, s, tx, tk, tv, p);
   if (e != cudaSuccess || p.ksplit == 1) return e;
   dim3 g2((Rk + rv + 255) / 256, n_tok);
-  append_finalize_kernel<<<g2, 256, 0, s>>>(p.ws, n_tok, Rk, rv, p.ksplit, rows, p.kc, p.vc, n_rows, err);
-  return cudaGetLastError();
+  return launch_pdl(append_finalize_kernel, g2, dim3(256), 0, s, (const float*)p.ws, n_tok, Rk, rv, p.ksplit, rows,
+                    p.kc, p.vc, n_rows, err);
 }
 
 }  // namespace dck

@@ -144,6 +144,29 @@ __device__ __forceinline__ int item_begin(int c, int NT, int n_items) {
   return (int)(((int64_t)c * NT) / n_items);
 }
 
+// Programmatic dependent launch: a kernel launched with launch_pdl may start
+// while the previous kernel on the stream finishes; pdl_wait() returns once
+// that kernel is complete and its memory visible (a no-op without PDL), and
+// pdl_launch_dependents() lets the next kernel launch early in turn.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 // Tiles [0, main_tiles) are split in contiguous whole-tile ranges over the
 // n_items work items; with `split_extra` (tensor-core path) and fewer than
 // kFineSplitBelow tiles per item, only n_items * floor(NT / n_items) of them,
