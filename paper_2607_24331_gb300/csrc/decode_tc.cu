@@ -51,8 +51,10 @@
 //              into the other accumulator and the two threads' bookkeeping
 //              overlaps the other's MMAs
 //   warps 2-9  epilogue: each TMEM lane quadrant (32 tokens) is served by two
-//              warps that split the 64 RoPE frequency pairs of a head and add
-//              their partial scores with shared-memory atomics.
+//              warps that split the 64 RoPE frequency pairs of a head; their
+//              partial scores meet in shared memory (query-folded mode: one
+//              array per frequency half, summed at the tile end; key mode:
+//              atomics).
 // Every wait is bounded (about 2 s); on expiry the CTA stops issuing work,
 // records kErrTimeout, waits for work in flight and still releases TMEM.
 //
@@ -61,8 +63,8 @@
 //           swizzle: UMMA operand A of the reconstruction;
 //   W slot  [nh heads][2 halves][w ranks][64 columns] MN-major: operand B
 //           (N = 128 nh, the 64-column atoms w * 128 bytes apart);
-//   P       [2 token atoms][Hq_pad heads][64 tokens] bf16, K-major (the
-//           absorption's operand B), staged here and bulk-stored per tile.
+// P ([2 token atoms][Hq_pad heads][64 tokens] bf16, K-major: the absorption's
+// operand B) is written straight to the workspace by the tile-end owners.
 #include <algorithm>
 #include <cmath>
 #include <cstring>
