@@ -150,6 +150,9 @@ __global__ void __launch_bounds__(kAThreads, 1)
       const uint64_t pol = policy_evict_first();
       int v_cnt = 0, p_cnt = 0;
       bool ok = true, first = true;
+      // reference maxima (lane = head) of the previous tile and, loaded a tile
+      // ahead so that their latency hides behind the value loads, of this one
+      float m_prev = 0.f, m_pf = 0.f;
       for (int ph = 0; ph < 2 && ok; ++ph)
       for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
         for (int i = 0; i < seg.ntiles && ok; ++i) {
@@ -185,11 +188,15 @@ __global__ void __launch_bounds__(kAThreads, 1)
             // does any head's reference max rise at this tile?  (decided here, once,
             // for the MMA thread; the epilogue warps take the same decision)
             bool need = false;
-            if (i > 0) {
-              const float mn = lane < Hq ? aa.mglob[x * Hq + lane] : 0.f;
-              const float mo = lane < Hq ? aa.mglob[(x - 1) * Hq + lane] : 0.f;
-              need = __any_sync(0xffffffffu, mn > mo);
+            float m_now;
+            if (i == 0) {
+              m_now = lane < Hq ? aa.mglob[x * Hq + lane] : 0.f;
+            } else {
+              m_now = m_pf;
+              need = __any_sync(0xffffffffu, m_now > m_prev);
             }
+            if (i + 1 < seg.ntiles) m_pf = lane < Hq ? aa.mglob[(x + 1) * Hq + lane] : 0.f;
+            m_prev = m_now;
             if (lane == 0) {
               const int sl = p_cnt % kNP;
               sm.pneed[sl] = need ? 1 : 0;
