@@ -208,7 +208,7 @@ size_t tc_append_workspace(int n_tok, int Rk, int rv) {
 
 cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, const void* A_v, int Rk, int rv,
                              const int64_t* rows, void* kc, void* vc, int64_t n_rows, void* ws, size_t ws_bytes,
-                             int* err, cudaStream_t s) {
+                             int* err, cudaStream_t s, int* n_launches) {
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -237,6 +237,7 @@ cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, c
   cudaError_t e = cudaFuncSetAttribute(append_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid(ntiles, (n_tok + kBM - 1) / kBM, p.ksplit);
+  *n_launches = p.ksplit > 1 ? 2 : 1;
   e = launch_pdl(append_tc_kernel, grid, dim3(kThreads), smem, s, tx, tk, tv, p);
   if (e != cudaSuccess || p.ksplit == 1) return e;
   dim3 g2((Rk + rv + 255) / 256, n_tok);

@@ -19,7 +19,7 @@ bool tc_append_supports(int D, int Rk, int rv, int dtype);
 size_t tc_append_workspace(int n_tok, int Rk, int rv);
 cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, const void* A_v, int Rk, int rv,
                              const int64_t* rows, void* kc, void* vc, int64_t n_rows, void* ws, size_t ws_bytes,
-                             int* err, cudaStream_t s);
+                             int* err, cudaStream_t s, int* n_launches);
 }  // namespace dck
 
 using namespace dck;
@@ -249,18 +249,19 @@ dck_status dck_latent_append(const dck_layer_desc* desc, const void* x, int32_t 
   if (!device_state(&err, nullptr)) return DCK_ERR_CUDA;
   const LayerTable lt = make_table(desc);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int launches = 1;  // kernels this call put on the stream
   cudaError_t e;
   if (tc_append_supports(desc->hidden, lt.Rk, lt.rv, desc->dtype)) {
     const size_t need = tc_append_workspace(n_tok, lt.Rk, lt.rv);
     if (need && (!workspace || ws_bytes < need || !aligned(workspace, 256))) return DCK_ERR_WORKSPACE;
     e = launch_append_tc(x, n_tok, desc->hidden, A_k, A_v, lt.Rk, lt.rv, d_rows, kcache, vcache, n_rows, workspace,
-                         ws_bytes, err, s);
+                         ws_bytes, err, s, &launches);
   } else {
     e = launch_append_simt(x, n_tok, desc->hidden, A_k, A_v, lt.Rk, lt.rv, d_rows, kcache, vcache, n_rows,
                            desc->dtype, err, s);
   }
   if (e != cudaSuccess) return DCK_ERR_CUDA;
-  g_last_launches = 1;
+  g_last_launches = launches;
   return DCK_OK;
 }
 
