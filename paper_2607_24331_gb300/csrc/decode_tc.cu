@@ -52,9 +52,8 @@
 //              overlaps the other's MMAs
 //   warps 2-9  epilogue: each TMEM lane quadrant (32 tokens) is served by two
 //              warps that split the 64 RoPE frequency pairs of a head; their
-//              partial scores meet in shared memory (query-folded mode: one
-//              array per frequency half, summed at the tile end; key mode:
-//              atomics).
+//              partial scores go to one shared-memory array per frequency
+//              half, summed at the tile end.
 // Every wait is bounded (about 2 s); on expiry the CTA stops issuing work,
 // records kErrTimeout, waits for work in flight and still releases TMEM.
 //
@@ -106,7 +105,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 template <bool kFold>
 struct Ring {
-  static constexpr int NW = 4;                // factor-item slots
+  static constexpr int NW = kFold ? 4 : 3;    // factor-item slots (key mode keeps 16 KB for queries)
   // MMA-issuing threads, each with its own factor ring: two in query-folded
   // mode; key mode's units carry up to four items, which one thread's ring of
   // all four slots streams better
@@ -155,9 +154,9 @@ template <bool kFold>
 struct Smem {
   uint8_t a[kNA][kSlot];
   uint8_t w[Ring<kFold>::NW][kSlotW];
-  // scores [head][token]: query-folded mode keeps one array per frequency half
-  // (plain stores, summed at the tile end); key mode accumulates atomically
-  float x[kFold ? 2 * kMaxHqTc * 128 : kMaxHqTc * 128];
+  // scores [frequency half][query head][token]: each half's partial scores by
+  // plain stores, summed at the tile end
+  float x[2 * kMaxHqTc * 128];
   float qr[kFold ? 1 : kMaxHqTc * kD];      // key mode: rotated queries * log2(e)/sqrt(d)
   double om64[kD / 2];
   float om32[kD / 2];
@@ -626,9 +625,10 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
                       }
                   }
                 }
+                float* xh = sm.x + hf * (kMaxHqTc * 128);  // this frequency half's scores
 #pragma unroll
                 for (int jj = 0; jj < kMaxQPerKv; ++jj)
-                  if (jj < qpg) atomicAdd(&sm.x[(j0 + jj) * 128 + tau], part[jj]);
+                  if (jj < qpg) xh[(j0 + jj) * 128 + tau] = part[jj];
               }
             }
             DCK_TC_TRACE(21);
@@ -644,12 +644,12 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
           const bool own = jt < Hq && sm.hunit[jt] >= ua && sm.hunit[jt] < ub;  // head computed here
           const int tb = 16 * ct;  // first token of this owner
           float sc[16];
-          float4* xr = reinterpret_cast<float4*>(&sm.x[jt * 128 + tb]);
-          const float4* xr2 = reinterpret_cast<const float4*>(&sm.x[(kFold ? kMaxHqTc * 128 : 0) + jt * 128 + tb]);
+          const float4* xr = reinterpret_cast<const float4*>(&sm.x[jt * 128 + tb]);
+          const float4* xr2 = reinterpret_cast<const float4*>(&sm.x[kMaxHqTc * 128 + jt * 128 + tb]);
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             float4 v = own ? xr[q] : make_float4(0.f, 0.f, 0.f, 0.f);
-            if (kFold && own) {  // the other frequency half (every score is stored each tile)
+            if (own) {  // plus the other frequency half (every score is stored each tile)
               const float4 w = xr2[q];
               v = make_float4(v.x + w.x, v.y + w.y, v.z + w.z, v.w + w.w);
             }
@@ -657,7 +657,6 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
             sc[4 * q + 1] = v.y;
             sc[4 * q + 2] = v.z;
             sc[4 * q + 3] = v.w;
-            if (!kFold && own) xr[q] = make_float4(0.f, 0.f, 0.f, 0.f);  // key mode: ready for the next tile's sums
           }
           const int nv = max(0, min(16, seg.t_end - (t0 + tb)));  // tokens inside the sequence
           float mx = -INFINITY;
