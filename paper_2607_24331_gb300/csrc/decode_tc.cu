@@ -157,7 +157,12 @@ struct Smem {
   // scores [frequency half][query head][token]: each half's partial scores by
   // plain stores, summed at the tile end
   float x[2 * kMaxHqTc * 128];
-  float qr[kFold ? 1 : kMaxHqTc * kD];      // key mode: rotated queries * log2(e)/sqrt(d)
+  // key mode: rotated queries * log2(e)/sqrt(d), bf16 [query head][d] (the
+  // B operand of the warps' score MMAs), and per epilogue warp a staging tile
+  // of its 32 tokens' rotated keys [token][32] bf16 (the A operand), 16-byte
+  // chunks swizzled by (token / 2) % 4
+  __nv_bfloat16 qr[kFold ? 2 : kMaxHqTc * kD];
+  uint8_t kst[kFold ? 1 : kEpiThreads / 32][kFold ? 16 : 32 * 64];
   double om64[kD / 2];
   float om32[kD / 2];
   float beta[kD / 2];
@@ -173,6 +178,25 @@ struct Smem {
 };
 
 __device__ __forceinline__ uint32_t swz_of(int w) { return w == 64 ? kSw128 : (w == 32 ? kSw64 : kSw32); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return (uint32_t)__bfloat16_as_ushort(h.x) | ((uint32_t)__bfloat16_as_ushort(h.y) << 16);
+}
+// Four 8x8 b16 matrices from shared memory; lane i gives the row address of row
+// i % 8 of matrix i / 8.
+__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+// d += a b for one 16 x 8 x 16 tile, bf16 inputs, fp32 accumulators.
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
 
 // ---------------------------------------------------------------------------
 // the scores kernel
@@ -511,8 +535,8 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
           float sn, cs;
           sincosf((float)(ang - 6.283185307179586 * rint(ang * 0.15915494309189535)), &sn, &cs);
           const float x1v = __bfloat162float(qb[j * kD + pi]), x2v = __bfloat162float(qb[j * kD + pi + kD / 2]);
-          sm.qr[j * kD + pi] = (x1v * cs - x2v * sn) * qscale;
-          sm.qr[j * kD + pi + kD / 2] = (x1v * sn + x2v * cs) * qscale;
+          sm.qr[j * kD + pi] = __float2bfloat16_rn((x1v * cs - x2v * sn) * qscale);
+          sm.qr[j * kD + pi + kD / 2] = __float2bfloat16_rn((x1v * sn + x2v * cs) * qscale);
         }
       }
       // RoPE angle of token t0+tau and pair p: (t0*w_p mod 2pi, fp64) + tau*w_p (fp32);
@@ -580,14 +604,19 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
               xh[sm.order[gs.h0 + 2 * u] * 128 + tau] = (pa[0][0] + pa[0][1]) + (pa[0][2] + pa[0][3]);
               if (nh == 2) xh[sm.order[gs.h0 + 2 * u + 1] * 128 + tau] = (pa[1][0] + pa[1][1]) + (pa[1][2] + pa[1][3]);
             } else {
+              // per head: rotate the key's 32 frequency pairs of this half (two
+              // passes of 16), stage them as bf16, and form the scores of the
+              // head's qpg query heads with mma m16n8k16 (rows: the warp's 32
+              // tokens in two m-tiles; k: 16 rotated x-halves, then 16 y-halves
+              // per pass; n: query heads, padded to 8)
+              const int gid = lane >> 2, tig = lane & 3;
+              uint8_t* st = sm.kst[warp - 2];
+              const uint32_t st_addr = smem_u32(st);
               for (int hh = 0; hh < nh; ++hh) {
                 const int j0 = sm.order[gs.h0 + 2 * u + hh] * qpg;
                 const uint32_t cb = tmem + lane_base + buf * kKCols + hh * kD;
                 const bool last = hh == nh - 1;
-                // two passes of 16 frequency pairs keep the register footprint small
-                float part[kMaxQPerKv];
-#pragma unroll
-                for (int jj = 0; jj < kMaxQPerKv; ++jj) part[jj] = 0.f;
+                float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
 #pragma unroll
                 for (int ps = 0; ps < 2; ++ps) {
                   float k1v[16], k2v[16];
@@ -599,36 +628,52 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
                   }
+                  // this lane's token: rotated x-halves (chunks 0, 1) and y-halves (2, 3)
+                  uint32_t rw[16];
 #pragma unroll
-                  for (int i4 = 0; i4 < 16; i4 += 4) {
-                    // four rotated frequency pairs, then each query head's matching
-                    // halves with two 16-byte shared loads
-                    float r1[4], r2[4];
+                  for (int w = 0; w < 8; ++w) {
+                    const int ip = 16 * ps + 2 * w;
+                    const float a0 = fmaf(k1v[2 * w], cs[ip], -k2v[2 * w] * sn[ip]);
+                    const float a1 = fmaf(k1v[2 * w + 1], cs[ip + 1], -k2v[2 * w + 1] * sn[ip + 1]);
+                    const float b0 = fmaf(k1v[2 * w], sn[ip], k2v[2 * w] * cs[ip]);
+                    const float b1 = fmaf(k1v[2 * w + 1], sn[ip + 1], k2v[2 * w + 1] * cs[ip + 1]);
+                    rw[w] = pack_bf16x2(a0, a1);
+                    rw[8 + w] = pack_bf16x2(b0, b1);
+                  }
+                  __syncwarp();  // the previous pass's fragments have been read
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                      const int ip = 16 * ps + i4 + u;
-                      r1[u] = fmaf(k1v[i4 + u], cs[ip], -k2v[i4 + u] * sn[ip]);
-                      r2[u] = fmaf(k1v[i4 + u], sn[ip], k2v[i4 + u] * cs[ip]);
+                  for (int c = 0; c < 4; ++c)
+                    *reinterpret_cast<uint4*>(st + lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4)) =
+                        make_uint4(rw[4 * c], rw[4 * c + 1], rw[4 * c + 2], rw[4 * c + 3]);
+                  __syncwarp();
+#pragma unroll
+                  for (int ks = 0; ks < 2; ++ks) {  // x-halves, then y-halves
+                    // B: query head n = gid (zero past qpg), k = 2 tig .. and 2 tig + 8 ..
+                    uint32_t bq0 = 0u, bq1 = 0u;
+                    if (gid < qpg) {
+                      const __nv_bfloat16* qrow = sm.qr + (j0 + gid) * kD + 64 * ks + 32 * hf + 16 * ps;
+                      bq0 = *reinterpret_cast<const uint32_t*>(qrow + 2 * tig);
+                      bq1 = *reinterpret_cast<const uint32_t*>(qrow + 2 * tig + 8);
                     }
-                    const float* qrow = sm.qr + j0 * kD + 32 * hf + 16 * ps + i4;
 #pragma unroll
-                    for (int jj = 0; jj < kMaxQPerKv; ++jj)
-                      if (jj < qpg) {
-                        const float4 qa = *reinterpret_cast<const float4*>(qrow + jj * kD);
-                        const float4 qb = *reinterpret_cast<const float4*>(qrow + jj * kD + 64);
-                        float v = part[jj];
-                        v = fmaf(qa.x, r1[0], fmaf(qb.x, r2[0], v));
-                        v = fmaf(qa.y, r1[1], fmaf(qb.y, r2[1], v));
-                        v = fmaf(qa.z, r1[2], fmaf(qb.z, r2[2], v));
-                        v = fmaf(qa.w, r1[3], fmaf(qb.w, r2[3], v));
-                        part[jj] = v;
-                      }
+                    for (int mt = 0; mt < 2; ++mt) {
+                      // A: tokens 16 mt .. +15, k chunks 2 ks and 2 ks + 1 of the staged rows
+                      const int r = 16 * mt + (lane & 7) + 8 * ((lane >> 3) & 1), ch = 2 * ks + (lane >> 4);
+                      uint32_t af[4];
+                      ldmatrix_x4(af, st_addr + r * 64 + ((ch ^ ((r >> 1) & 3)) << 4));
+                      mma_bf16_16816(acc[mt], af, bq0, bq1);
+                    }
                   }
                 }
+                // scores: token (16 mt + gid [+ 8]) of this quadrant, query heads 2 tig, 2 tig + 1
                 float* xh = sm.x + hf * (kMaxHqTc * 128);  // this frequency half's scores
 #pragma unroll
-                for (int jj = 0; jj < kMaxQPerKv; ++jj)
-                  if (jj < qpg) xh[(j0 + jj) * 128 + tau] = part[jj];
+                for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+                  for (int q = 0; q < 4; ++q) {
+                    const int jj = 2 * tig + (q & 1), t = quad * 32 + 16 * mt + gid + 8 * (q >> 1);
+                    if (jj < qpg) xh[(j0 + jj) * 128 + t] = acc[mt][q];
+                  }
               }
             }
             DCK_TC_TRACE(21);
