@@ -18,9 +18,12 @@
 // lane per r_v row of a chunk.
 //
 // Warps: 0 producer (P images by bulk copy, value chunks by TMA, next tile's
-// values prefetched toward L2), 1 TMEM owner whose lane 0 issues the MMAs
-// (M = 128 r_v rows, N = Hq_pad, K = 16 tokens; 8 per chunk and tile),
-// 2-5 epilogue (one TMEM lane quadrant each: rescales and the U readout).
+// values prefetched toward L2), 1 and 6 MMA issuers (lane 0 of each; M = 128
+// r_v rows, N = Hq_pad, K = 16 tokens; 8 per chunk and tile), each taking half
+// of a tile's r_v chunks from its own ring of value slots (a single thread's
+// MMA issue, commits and barrier tests took longer than the values took to
+// arrive); warp 1 owns TMEM.  2-5 epilogue (one TMEM lane quadrant each:
+// rescales and the U readout).
 // Every wait is bounded; on expiry the CTA records kErrTimeout and releases
 // TMEM after the work in flight has landed.
 #include <algorithm>
@@ -44,9 +47,9 @@ namespace {
 using namespace sm100;
 using namespace tc;
 
-constexpr int kAThreads = 192;
-constexpr int kVSlot = 16384;  // [128 tokens][64 rv] bf16, 128B-swizzled: one half of an r_v chunk
-constexpr int kNVs = 12;       // value slots: six chunks in flight
+constexpr int kAThreads = 224;
+constexpr int kVSlot = 32768;  // one r_v chunk: [2 halves][128 tokens][64 rv] bf16, 128B-swizzled
+constexpr int kNVr = 3;        // value slots of each MMA thread's ring: six chunks in flight
 constexpr int kPSlot = 8192;   // P image of one tile (Hq_pad <= 32)
 constexpr int kNP = 2;
 constexpr uint32_t kTmemCols = 512;
@@ -64,9 +67,9 @@ struct AbsArgs {
 };
 
 struct ASmem {
-  uint8_t v[kNVs][kVSlot];
+  uint8_t v[2 * kNVr][kVSlot];  // ring of MMA thread t: slots [t kNVr, (t + 1) kNVr)
   uint8_t p[kNP][kPSlot];
-  uint64_t v_full[kNVs], v_empty[kNVs], p_full[kNP], p_empty[kNP];
+  uint64_t v_full[2 * kNVr], v_empty[2 * kNVr], p_full[kNP], p_empty[kNP];
   uint64_t drain, tile_ok, u_ready, u_free;
   int pneed[kNP];  // P slot's tile raises some head's reference max (set by the producer before the slot fills)
   int scan[kAThreads];
@@ -86,17 +89,17 @@ __global__ void __launch_bounds__(kAThreads, 1)
   griddep_launch();  // the combine kernel may stage its factors as CTAs finish
 
   if (tid == 0) {
-    for (int i = 0; i < kNVs; ++i) {
+    for (int i = 0; i < 2 * kNVr; ++i) {
       mbar_init(&sm.v_full[i], 1);
       mbar_init(&sm.v_empty[i], 1);
     }
     for (int i = 0; i < kNP; ++i) {
       mbar_init(&sm.p_full[i], 1);
-      mbar_init(&sm.p_empty[i], 1);
+      mbar_init(&sm.p_empty[i], 2);  // released by both MMA threads
     }
-    mbar_init(&sm.drain, 1);
+    mbar_init(&sm.drain, 2);
     mbar_init(&sm.tile_ok, 4);
-    mbar_init(&sm.u_ready, 1);
+    mbar_init(&sm.u_ready, 2);
     mbar_init(&sm.u_free, 4);
     sm.abort_flag = 0;
     fence_mbar_init();
@@ -132,6 +135,8 @@ __global__ void __launch_bounds__(kAThreads, 1)
       cb = min(c_hi - e * n_chunks, n_chunks);
     }
   };
+  // the two MMA threads split a tile's chunks [ca, cb) at cm: thread 0 [ca, cm), thread 1 [cm, cb)
+  auto chunk_mid = [](int ca, int cb) { return ca + (cb - ca + 1) / 2; };
   const int64_t xbase = extra_slot_base(a.n_items, a.B);
   tc_fence_before();
   __syncthreads();
@@ -148,7 +153,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
     // probabilities and maxima.
     if (has_work) {
       const uint64_t pol = policy_evict_first();
-      int v_cnt = 0, p_cnt = 0;
+      int v_cnt[2] = {0, 0}, p_cnt = 0;
       bool ok = true, first = true;
       // reference maxima (lane = head) of the previous tile and, loaded a tile
       // ahead so that their latency hides behind the value loads, of this one
@@ -168,18 +173,38 @@ __global__ void __launch_bounds__(kAThreads, 1)
                 prefetch_l2(static_cast<const __nv_bfloat16*>(a.vc) + r0 * lt.rv, (uint32_t)(nr * lt.rv * 2));
             }
           }
-          // value slot v_cnt + q holds half (q % 2) of chunk ca + q / 2
-          int nbox = 2 * (cb - ca), done = 0;
-          if (first) {  // the boxes that fit the empty ring, ahead of the wait
-            const int nb = min(nbox, kNVs);
-            if (lane < nb) {
-              const int sl = (v_cnt + lane) % kNVs;
-              mbar_expect_tx(&sm.v_full[sl], kVSlot);
-              tma_load_2d_hint(sm.v[sl], &maps.vc, &sm.v_full[sl], 128 * ca + 64 * lane, (int32_t)yrow, pol);
+          // chunks go to the two MMA threads' rings alternately (thread 0: [ca, cm),
+          // thread 1: [cm, cb)), each chunk one slot filled by two boxes (lanes 0, 1)
+          const int cm = chunk_mid(ca, cb), nch = cb - ca;
+          int done = 0;
+          // the j-th chunk issued for this tile, and its ring
+          auto chunk_at = [&](int j, int& c, int& r) {
+            const int n0 = cm - ca, n1 = cb - cm, m = min(n0, n1);
+            if (j < 2 * m) {
+              r = j & 1;
+              c = (r ? cm : ca) + (j >> 1);
+            } else {
+              r = n0 > n1 ? 0 : 1;
+              c = (r ? cm : ca) + m + (j - 2 * m);
             }
+          };
+          auto issue_chunk = [&](int c, int r) {
+            const int sl = r * kNVr + v_cnt[r] % kNVr;
+            if (lane == 0) mbar_expect_tx(&sm.v_full[sl], kVSlot);
             __syncwarp();
-            v_cnt += nb;
-            done = nb;
+            if (lane < 2)
+              tma_load_2d_hint(sm.v[sl] + lane * (kVSlot / 2), &maps.vc, &sm.v_full[sl], 128 * c + 64 * lane,
+                               (int32_t)yrow, pol);
+            __syncwarp();
+            ++v_cnt[r];
+          };
+          if (first) {  // the chunks that fit the empty rings, ahead of the wait
+            for (; done < nch; ++done) {
+              int c, r;
+              chunk_at(done, c, r);
+              if (v_cnt[r] >= kNVr) break;
+              issue_chunk(c, r);
+            }
             griddep_wait();
             first = false;
           }
@@ -207,27 +232,24 @@ __global__ void __launch_bounds__(kAThreads, 1)
           __syncwarp();
           DCK_AB_TRACE(1);
           ++p_cnt;
-          while (done < nbox && ok) {  // as many boxes per instruction as slots are free
-            const int nb = claim_slots(sm.v_empty, kNVs, v_cnt, nbox - done, lane, abort_flag);
-            if (!(ok = nb > 0)) break;
-            if (lane < nb) {
-              const int sl = (v_cnt + lane) % kNVs, q = done + lane;
-              mbar_expect_tx(&sm.v_full[sl], kVSlot);
-              tma_load_2d_hint(sm.v[sl], &maps.vc, &sm.v_full[sl], 128 * ca + 64 * q, (int32_t)yrow, pol);
-            }
-            __syncwarp();
+          for (; done < nch && ok; ++done) {
+            int c, r;
+            chunk_at(done, c, r);
+            if (!(ok = wait_slots(sm.v_empty + r * kNVr, kNVr, v_cnt[r], 1, lane, abort_flag))) break;
+            issue_chunk(c, r);
             DCK_AB_TRACE(2);
-            v_cnt += nb;
-            done += nb;
           }
         }
       }
     }
-  } else if (warp == 1) {
-    // ---- MMA issuer (lane 0) ---------------------------------------------------
+  } else if (warp == 1 || warp == 6) {
+    // ---- MMA issuers: lane 0 of warp 1 takes chunks [ca, cm) of every tile,
+    // lane 0 of warp 6 chunks [cm, cb), each from its own value ring; both wait
+    // for every P slot and every hand-off with the epilogue, and both release --
     if (lane == 0 && has_work) {
+      const int t = warp == 1 ? 0 : 1;
       const uint32_t idesc_v = idesc_bf16(128, hq_pad, true, false);
-      int v_cnt = 0, p_cnt = 0, rc = 0, sgc = 0;
+      int vs = 0, vph = 0, p_cnt = 0, rc = 0, sgc = 0;
       bool ok = true;
       for (int ph = 0; ph < 2 && ok; ++ph)
       for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
@@ -257,36 +279,40 @@ __global__ void __launch_bounds__(kAThreads, 1)
           // chains are interleaved
           int ca, cb;
           chunks_of(ph, seg.x0 + i, ca, cb);
-          for (int c = ca; c < cb && ok; c += 2) {
-            const int nc = min(2, cb - c);
+          const int cm = chunk_mid(ca, cb);
+          const int c0 = t ? cm : ca, c1 = t ? cb : cm;
+          for (int c = c0; c < c1 && ok; c += 2) {
+            const int nc = min(2, c1 - c);
             uint32_t vb[2] = {0u, 0u};
+            int sl[2] = {0, 0};
             for (int q = 0; q < nc && ok; ++q) {
-              const int sl = (v_cnt + 2 * q) % kNVs;  // even: the chunk's halves are adjacent slots
-              const uint32_t vpar = ((v_cnt + 2 * q) / kNVs) & 1;
-              if (!(ok = mbar_wait(&sm.v_full[sl], vpar, abort_flag))) break;
-              if (!(ok = mbar_wait(&sm.v_full[sl + 1], vpar, abort_flag))) break;
+              sl[q] = t * kNVr + vs;
+              if (!(ok = mbar_wait(&sm.v_full[sl[q]], vph, abort_flag))) break;
+              if (++vs == kNVr) {
+                vs = 0;
+                vph ^= 1;
+              }
               if (nvalid < kTile) {  // rows past the sequence end: exact zeros
                 for (int r = nvalid; r < kTile; ++r)
 #pragma unroll
                   for (int w = 0; w < 8; ++w) {
-                    reinterpret_cast<uint4*>(sm.v[sl] + r * 128)[w] = make_uint4(0, 0, 0, 0);
-                    reinterpret_cast<uint4*>(sm.v[sl + 1] + r * 128)[w] = make_uint4(0, 0, 0, 0);
+                    reinterpret_cast<uint4*>(sm.v[sl[q]] + r * 128)[w] = make_uint4(0, 0, 0, 0);
+                    reinterpret_cast<uint4*>(sm.v[sl[q]] + kVSlot / 2 + r * 128)[w] = make_uint4(0, 0, 0, 0);
                   }
                 fence_proxy_async_smem();
               }
-              vb[q] = smem_u32(sm.v[sl]);
+              vb[q] = smem_u32(sm.v[sl[q]]);
             }
             if (!ok) break;
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
               const uint64_t bd = sdesc(pbase + (k >> 2) * (hq_pad * 128) + (k & 3) * 32, 16, 1024, kSw128);
               for (int q = 0; q < nc; ++q)
-                umma_f16(tmem + (c + q) * hq_pad, sdesc(vb[q] + k * 2048, kVSlot, 1024, kSw128), bd, idesc_v,
+                umma_f16(tmem + (c + q) * hq_pad, sdesc(vb[q] + k * 2048, kVSlot / 2, 1024, kSw128), bd, idesc_v,
                          (i == 0 && k == 0) ? 0u : 1u);
             }
-            for (int q = 0; q < 2 * nc; ++q) umma_commit(&sm.v_empty[(v_cnt + q) % kNVs]);
+            for (int q = 0; q < nc; ++q) umma_commit(&sm.v_empty[sl[q]]);
             DCK_AB_TRACE(12);
-            v_cnt += 2 * nc;
           }
           if (!ok) break;
           umma_commit(&sm.p_empty[psl]);
