@@ -220,7 +220,8 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--config", type=int, default=1)
+    ap.add_argument("--config", type=int, default=1,
+                    help="0 tiny fp32, 1 MHA B16xT4096 (default), 2/3 GQA, 4 32-layer step, 5 MHA with fixed groups of 4")
     ap.add_argument("--batch", type=int, default=None, help="batch of the 32-layer workload (config 4)")
     ap.add_argument("--impl", default="dck", choices=["dck", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time for cpu_baseline")

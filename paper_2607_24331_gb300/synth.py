@@ -294,13 +294,21 @@ def llama3_gqa_layer() -> LayerSpec:
                      (192, 256, 256), 384, "bf16", 5e5)
 
 
+def recalkv_mha_layer() -> LayerSpec:
+    """The Llama-2-7B-like MHA layer with ReCalKV's fixed grouping (Sec. III-C): groups of
+    four consecutive heads and one uniform rank r/K per group, at the same total rank
+    (sum r_g = 1024) and value rank as the DynaCalKV layer."""
+    return LayerSpec(4096, 32, 32, 128, groups_from_sizes((4,) * 8, range(32)), (128,) * 8, 1024, "bf16", 1e4)
+
+
 def ragged_lens(seed: int, batch: int, lo: int = 1024, hi: int = 16384) -> Tuple[int, ...]:
     key = stream_key(seed, 1000 + batch, TID["lens"])
     return tuple(int(v) for v in uniform_ints(key, batch, lo, hi))
 
 
 def workload(cfg: int, batch: Optional[int] = None) -> Workload:
-    """The five benchmark workloads (0: tiny fp32 MHA ... 4: 32-layer ragged MHA step)."""
+    """The five benchmark workloads (0: tiny fp32 MHA ... 4: 32-layer ragged MHA step), and
+    5: the MHA layer of workload 1 with ReCalKV's fixed groups of four at equal total rank."""
     if cfg == 0:
         return Workload("tiny-fp32-mha D512 H8 d64 B1 T512", tiny_mha_layer(), (512,))
     if cfg == 1:
@@ -314,6 +322,8 @@ def workload(cfg: int, batch: Optional[int] = None) -> Workload:
         b = 8 if batch is None else batch
         return Workload(f"llama2-7b-mha 32 layers B{b} ragged T~U[1024,16384]",
                         llama2_mha_layer(), ragged_lens(0, b), n_layers=32)
+    if cfg == 5:
+        return Workload("llama2-7b-mha recalkv-groups D4096 H32 d128 B16 T4096", recalkv_mha_layer(), (4096,) * 16)
     raise ValueError(cfg)
 
 

@@ -104,7 +104,7 @@ def _sample_pairs(B, Hq, n, seed):
     return sorted(pairs)
 
 
-@pytest.mark.parametrize("cfg", [1, 2, 3])
+@pytest.mark.parametrize("cfg", [1, 2, 3, 5])
 def test_full_size_configs_sampled(cfg):
     """Full benchmark workload, inputs from the host generator, sampled oracle outputs."""
     w = S.workload(cfg)
