@@ -9,7 +9,11 @@
 // TMEM and issues tcgen05.mma, warps 2-5 drain the accumulator (one TMEM lane
 // quadrant each).  Small batches (<= 256 tokens, the decode-step append) split
 // K over CTAs, each storing its fp32 partial in its own slice of the caller's
-// workspace; a second kernel sums the slices, rounds and scatters.
+// workspace; a second kernel sums the slices, rounds and scatters.  The ring
+// has only as many stages as a CTA has K blocks, so split CTAs of two K blocks
+// fit two to an SM and the whole split runs in one wave.
+#include <algorithm>
+
 #include "common.cuh"
 #include "sm100.cuh"
 #include "tmap.h"
@@ -25,13 +29,14 @@ constexpr int kBBytes = kBK * kMaxBN * 2;       // 32 KB
 constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kThreads = 192;
 constexpr int kSplitMaxTok = 256;
-constexpr int kMaxSplit = 16;  // K splits of a small batch
+constexpr int kMaxSplit = 32;  // K splits of a small batch
 
 struct AppendParams {
   int n_tok, D, Rk, rv;
   int nt_k;      // N tiles over the key output
   int kblocks;   // ceil(D / 64)
   int ksplit;
+  int stages;    // ring depth: min(kStages, K blocks of one CTA)
   const int64_t* rows;
   __nv_bfloat16* kc;
   __nv_bfloat16* vc;
@@ -52,7 +57,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                      const __grid_constant__ CUtensorMap tm_av, const AppendParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
+  const int nst = p.stages;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + nst * kStageBytes);
   uint64_t* empty = full + kStages;
   uint64_t* acc_bar = empty + kStages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_bar + 1);
@@ -68,7 +74,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nboxes = (nt + 63) / 64;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < nst; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
@@ -94,8 +100,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tm_x);
     tma_prefetch_desc(tmb);
     for (int kb = kb0; kb < kb1; ++kb) {
-      const int i = kb - kb0, s = i % kStages;
-      if (i >= kStages && !mbar_wait(&empty[s], ((i / kStages) - 1) & 1, abort_flag)) break;
+      const int i = kb - kb0, s = i % nst;
+      if (i >= nst && !mbar_wait(&empty[s], ((i / nst) - 1) & 1, abort_flag)) break;
       uint8_t* a = smem + s * kStageBytes;
       uint8_t* b = a + kABytes;
       mbar_expect_tx(&full[s], kABytes + nboxes * (kBK * 64 * 2));
@@ -105,8 +111,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1 && lane == 0) {
     const uint32_t idesc = idesc_bf16(kBM, nt, false, true);
     for (int kb = kb0; kb < kb1; ++kb) {
-      const int i = kb - kb0, s = i % kStages;
-      if (!mbar_wait(&full[s], (i / kStages) & 1, abort_flag)) break;
+      const int i = kb - kb0, s = i % nst;
+      if (!mbar_wait(&full[s], (i / nst) & 1, abort_flag)) break;
       tc_fence_after();
       const uint32_t a = smem_u32(smem + s * kStageBytes);
       const uint32_t b = a + kABytes;
@@ -178,9 +184,20 @@ __global__ void append_finalize_kernel(const float* __restrict__ ws, int n_tok, 
     if (threadIdx.x == 0 && blockIdx.x == 0) atomicOr(err, kErrBadRow);
     return;
   }
+  const int64_t zs = (int64_t)n_tok * N;  // stride between the splits' slices
   for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < N; c += gridDim.x * blockDim.x) {
-    float v = 0.f;
-    for (int z = 0; z < ksplit; ++z) v += ws[((int64_t)z * n_tok + m) * N + c];
+    const float* w = ws + (int64_t)m * N + c;
+    float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f;  // four loads in flight, summed in split order per chain
+    int z = 0;
+    for (; z + 4 <= ksplit; z += 4) {
+      const float a0 = w[z * zs], a1 = w[(z + 1) * zs], a2 = w[(z + 2) * zs], a3 = w[(z + 3) * zs];
+      v0 += a0;
+      v1 += a1;
+      v2 += a2;
+      v3 += a3;
+    }
+    for (; z < ksplit; ++z) v0 += w[z * zs];
+    const float v = (v0 + v1) + (v2 + v3);
     if (c < Rk) kc[row * Rk + c] = __float2bfloat16_rn(v);
     else vc[row * rv + (c - Rk)] = __float2bfloat16_rn(v);
   }
@@ -191,7 +208,8 @@ int plan_ksplit(int n_tok, int D, int Rk, int rv, int sms) {
   const int mt = (n_tok + kBM - 1) / kBM;
   const int ntiles = (Rk + kMaxBN - 1) / kMaxBN + (rv + kMaxBN - 1) / kMaxBN;
   const int kblocks = (D + kBK - 1) / kBK;
-  int ks = sms / max(1, mt * ntiles);
+  // up to two CTAs per SM (split CTAs of at most two K blocks take 96 KB of shared memory)
+  int ks = 2 * sms / max(1, mt * ntiles);
   ks = max(1, min(ks, min(kMaxSplit, kblocks)));
   return ks;
 }
@@ -220,6 +238,7 @@ cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, c
   p.nt_k = (Rk + kMaxBN - 1) / kMaxBN;
   p.kblocks = (D + kBK - 1) / kBK;
   p.ksplit = plan_ksplit(n_tok, D, Rk, rv, sms);
+  p.stages = std::min(kStages, (p.kblocks + p.ksplit - 1) / p.ksplit);
   p.rows = rows;
   p.kc = static_cast<__nv_bfloat16*>(kc);
   p.vc = static_cast<__nv_bfloat16*>(vc);
@@ -233,8 +252,10 @@ cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, c
       !make_tmap_2d_bf16(&tv, A_v, rv, D, (uint64_t)rv * 2, 64, kBK, CU_TENSOR_MAP_SWIZZLE_128B))
     return cudaErrorInvalidValue;
   const int ntiles = p.nt_k + (rv + kMaxBN - 1) / kMaxBN;
-  const size_t smem = kStages * kStageBytes + 1024 + 256;
-  cudaError_t e = cudaFuncSetAttribute(append_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  const size_t smem = (size_t)p.stages * kStageBytes + 1024 + 256;
+  // the attribute is an upper bound for every launch (prefill uses all kStages stages)
+  cudaError_t e = cudaFuncSetAttribute(append_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)(kStages * kStageBytes + 1024 + 256));
   if (e != cudaSuccess) return e;
   dim3 grid(ntiles, (n_tok + kBM - 1) / kBM, p.ksplit);
   *n_launches = p.ksplit > 1 ? 2 : 1;
