@@ -212,6 +212,31 @@ def run_reference(args):
 
 
 # ---------------------------------------------------------------------------
+# whole-job numbers over ranks (weak scaling: every rank runs its own replica)
+# ---------------------------------------------------------------------------
+
+def rank_seed(seed: int, rank: int) -> int:
+    """Data seed of a rank's replica: each rank decodes its own sequences."""
+    return seed + rank * 1000
+
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The slowest rank's time: the job finishes when its last rank does."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, batch: int, steps: int, t_ms: float) -> float:
+    """Decode tokens per second of the whole job: every rank decodes `batch` queries per step."""
+    return world * batch * steps / (t_ms / 1e3)
+
+
+# ---------------------------------------------------------------------------
 # the GPU arm
 # ---------------------------------------------------------------------------
 
@@ -253,7 +278,7 @@ def main():
     dt = device.TORCH_DTYPE[spec.dtype]
     layers = []
     for l in range(w.n_layers):
-        buf = device.DecodeBuffers(spec, w.seq_lens, device=dev).synth(seed=w.seed + rank * 1000, layer=l)
+        buf = device.DecodeBuffers(spec, w.seq_lens, device=dev).synth(seed=rank_seed(w.seed, rank), layer=l)
         A_k = torch.empty((spec.hidden, spec.rank_k), dtype=dt, device=dev)
         A_v = torch.empty((spec.hidden, spec.rank_v), dtype=dt, device=dev)
         device.synth_fill(A_k, S.stream_key(w.seed, l, S.TID["A_k"]), 1.0 / math.sqrt(spec.hidden))
@@ -334,13 +359,9 @@ def main():
     launches[0] = per_step_launches * K
     gpu_launches = launches[0]
     step_ms = [a.elapsed_time(b) for a, b in ev]
-    t_ms = sum(step_ms)
-    if world > 1:
-        tt = torch.tensor([t_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t_ms = float(tt.item())
+    t_ms = max_over_ranks(sum(step_ms), world, dev)
     ms_per_step = t_ms / K
-    value = world * B * K / (t_ms / 1e3)
+    value = job_throughput(world, B, K, t_ms)
 
     # ---- end to end: host inputs -> device -> result back, every step ----
     q_host = [torch.empty(buf.q.shape, dtype=dt, pin_memory=True) for (buf, *_r) in layers]
@@ -374,12 +395,8 @@ def main():
         e2e_step()
         eev[k][1].record(stream)
         eev[k][1].synchronize()   # the result is on the host before the next step starts
-    e2e_ms = sum(a.elapsed_time(b) for a, b in eev)
-    if world > 1:
-        tt = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
-    e2e_value = world * B * K / (e2e_ms / 1e3)
+    e2e_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in eev), world, dev)
+    e2e_value = job_throughput(world, B, K, e2e_ms)
 
     # ---- roofline of the attention kernels of one decode call (factor preparation, scores,
     # absorption: the region between the timing events; one call = one layer) ----
