@@ -11,15 +11,19 @@ Contents
 * ``decode.py``  - decode attention over grouped low-rank key latents and a
   whole-matrix value latent (Sec. III-A, III-C, III-D), with RoPE applied to
   the reconstructed keys and to the query; plain definition, fp64.
+* ``prefill.py`` - causal prefill attention over the same caches: many new
+  tokens per sequence, each attending to its prefix (the decode call is one
+  new token); plain definition, fp64.
 * ``append.py``  - the latent projection z = x L of new tokens (Sec. III-A).
 * ``layout.py``  - parameter counts of grouped key factors (Sec. III-C,
   Table I).
 
-Parity status: every function is pinned by ``tests/test_oracle_pins.py``
-(closed forms, library routines, invariants and brute force); none is
-"parity unpinned".
+Parity status: every function is pinned by ``tests/test_oracle_pins.py`` and
+``tests/test_prefill_oracle_pins.py`` (closed forms, library routines,
+invariants and brute force); none is "parity unpinned".
 """
 
 from .decode import decode_attention, rope, rope_freqs, kv_head_of  # noqa: F401
+from .prefill import prefill_attention  # noqa: F401
 from .append import latent_append  # noqa: F401
 from .layout import grouped_key_params, recalkv_key_params  # noqa: F401
