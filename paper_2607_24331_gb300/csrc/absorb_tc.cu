@@ -11,10 +11,10 @@
 // The scores kernel's reference max of a head can rise from one tile to the
 // next (it moves only when a tile's max exceeds it by 8); before such a tile
 // the epilogue warps rescale U by exp2(m_old - m_new) in TMEM, after the MMAs
-// of the earlier tiles have completed.  The MMA thread and the epilogue both
+// of the earlier tiles have completed.  The MMA threads and the epilogue all
 // read from the stored maxima which tiles need this and hand off only there
-// (drain, then tile_ok), so each hand-off phase follows the MMA thread's own
-// commit.  U = [r_v / 128 chunks][Hq_pad heads] fp32 accumulators, one TMEM
+// (drain, which both MMA threads commit, then tile_ok, which both wait for), so
+// each hand-off phase follows the MMA threads' own commits.  U = [r_v / 128 chunks][Hq_pad heads] fp32 accumulators, one TMEM
 // lane per r_v row of a chunk.
 //
 // Warps: 0 producer (P images by bulk copy, value chunks by TMA, next tile's
