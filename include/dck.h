@@ -204,6 +204,18 @@ dck_status dck_set_timing_events(void* ev_start, void* ev_stop);
 int32_t dck_last_launch_count(void);
 
 /*
+ * Self-test of failure detection (not part of the method; the paper has no
+ * counterpart): launches on `stream` one block that waits, through the same
+ * bounded mbarrier wait every tensor-core kernel uses, on a barrier that
+ * nothing arrives at.  After `limit_cycles` SM clock cycles (1000 .. 4e9) the
+ * wait gives up, the kernel records a timeout in the device error word and
+ * returns, so the next dck_last_device_error reports DCK_ERR_TIMEOUT and the
+ * CUDA context stays usable.  Returns DCK_ERR_INVALID for a limit outside that
+ * range (nothing is launched), DCK_ERR_CUDA if the launch fails, else DCK_OK.
+ */
+dck_status dck_selftest_bounded_wait(int64_t limit_cycles, void* stream);
+
+/*
  * Seeded synthetic input (not part of the method): fills n elements of `dst`
  * with the counter-based Gaussian stream `key` starting at element `start`:
  * SplitMix64 draws 2i and 2i+1, the sum of their eight 16-bit fields s,

@@ -17,6 +17,7 @@ int tc_decode_launches(const LayerTable& lt);
 cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s);
 bool tc_append_supports(int D, int Rk, int rv, int dtype);
 size_t tc_append_workspace(int n_tok, int Rk, int rv);
+cudaError_t launch_bounded_wait_selftest(long long limit_cycles, int* err, cudaStream_t s);
 cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, const void* A_v, int Rk, int rv,
                              const int64_t* rows, void* kc, void* vc, int64_t n_rows, void* ws, size_t ws_bytes,
                              int* err, cudaStream_t s, int* n_launches);
@@ -276,6 +277,15 @@ dck_status dck_last_device_error(void* stream) {
   if (v & kErrTimeout) return DCK_ERR_TIMEOUT;
   if (v) return DCK_ERR_INVALID;
   return DCK_OK;
+}
+
+dck_status dck_selftest_bounded_wait(int64_t limit_cycles, void* stream) {
+  if (limit_cycles < 1000 || limit_cycles > 4000000000LL) return DCK_ERR_INVALID;
+  int* err = nullptr;
+  if (!device_state(&err, nullptr)) return DCK_ERR_CUDA;
+  return launch_bounded_wait_selftest((long long)limit_cycles, err, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? DCK_OK
+             : DCK_ERR_CUDA;
 }
 
 dck_status dck_synth_gaussian(void* dst, int64_t n, uint64_t key, int64_t start, float scale, int32_t dtype,

@@ -28,6 +28,7 @@ EXPORTED = (
     "dck_status_string", "dck_validate_desc", "dck_latent_append_workspace_size", "dck_latent_append",
     "dck_decode_workspace_size", "dck_decode_attention", "dck_last_device_error", "dck_set_decode_kernel",
     "dck_last_launch_count", "dck_synth_gaussian", "dck_set_timing_events", "dck_decode_attention_noalloc",
+    "dck_selftest_bounded_wait",
 )
 
 
@@ -88,6 +89,8 @@ def lib() -> ctypes.CDLL:
     L.dck_last_launch_count.argtypes = []
     L.dck_set_timing_events.restype = I32
     L.dck_set_timing_events.argtypes = [P, P]
+    L.dck_selftest_bounded_wait.restype = I32
+    L.dck_selftest_bounded_wait.argtypes = [I64, P]
     L.dck_synth_gaussian.restype = I32
     L.dck_synth_gaussian.argtypes = [P, I64, U64, I64, F32, I32, P]
     _lib = L
@@ -200,6 +203,12 @@ def dck_set_timing_events(ev_start, ev_stop) -> int:
     p0 = None if ev_start is None else ev_start.cuda_event
     p1 = None if ev_stop is None else ev_stop.cuda_event
     return lib().dck_set_timing_events(p0, p1)
+
+
+def dck_selftest_bounded_wait(limit_cycles: int, stream=None) -> int:
+    """One kernel whose bounded wait on a barrier nothing arrives at gives up after
+    ``limit_cycles`` SM cycles; the timeout shows in the next dck_last_device_error."""
+    return lib().dck_selftest_bounded_wait(int(limit_cycles), _stream(stream))
 
 
 def check(status: int, what: str) -> None:

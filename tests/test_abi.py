@@ -68,3 +68,9 @@ def test_malformed_descriptors(kw, expect):
 
 def test_null_descriptor():
     assert dck.lib().dck_validate_desc(None) == dck.DCK_ERR_INVALID
+
+
+def test_selftest_rejects_limits_out_of_range_without_launching():
+    # checked on the host before any CUDA call (stream handle 0 is never used)
+    assert dck.dck_selftest_bounded_wait(10, 0) == dck.DCK_ERR_INVALID
+    assert dck.dck_selftest_bounded_wait(5_000_000_000, 0) == dck.DCK_ERR_INVALID
