@@ -144,6 +144,16 @@ def gpu_identifier(torch, dev):
         return str(dev)
 
 
+def workload_config(w, world: int) -> dict:
+    """The `config` of a bench line, the same for the GPU arm and the reference arm."""
+    ctx = (sorted(int(x) for x in set(w.seq_lens))[:4] if w.n_layers == 1
+           else f"ragged U[1024,16384], mean {sum(w.seq_lens) / len(w.seq_lens):.0f}")
+    return {"workload": w.name, "batch": w.batch, "context": ctx, "layers": w.n_layers,
+            "step": "latent append of B tokens + decode attention, per layer",
+            "l2": "flushed between steps (512 MB write outside the timed events)",
+            "parallelism": f"replicas x{world}"}
+
+
 # ---------------------------------------------------------------------------
 # the oracle as CPU baseline (rank 0 only)
 # ---------------------------------------------------------------------------
@@ -210,8 +220,7 @@ def run_reference(args):
     line = {"metric": METRIC, "value": value, "unit": UNIT, "impl": "reference", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name, "batch": w.batch, "context": list(sorted(set(w.seq_lens)))[:4],
-                       "layers": w.n_layers},
+            "config": workload_config(w, args.gpus),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
                              "sample": f"each step: 2 (sequence, query-head) pairs over full contexts, fp64 numpy"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -427,11 +436,7 @@ def main():
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
             "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if spec.dtype == "bf16" else "f32", "data": "synthetic (seeded Gaussian latents/factors)",
-            "config": {"workload": w.name, "batch": B, "context": sorted(set(w.seq_lens))[:4]
-                       if w.n_layers == 1 else f"ragged U[1024,16384], mean {np.mean(w.seq_lens):.0f}",
-                       "layers": w.n_layers, "step": "latent append of B tokens + decode attention, per layer",
-                       "l2": "flushed between steps (512 MB write outside the timed events)",
-                       "parallelism": f"replicas x{world}"},
+            "config": workload_config(w, world),
             "latent_gbs": step_alg_bytes / (ms_per_step / 1e3) / 1e9,
             "context_tokens_per_s": world * sum(w.seq_lens) * w.n_layers / (ms_per_step / 1e3),
             "ms_per_step_median": statistics.median(step_ms), "ms_per_step_warm_l2": warm_ms,

@@ -56,3 +56,14 @@ def test_single_rank_needs_no_process_group():
 
     assert bench.max_over_ranks(3.0, 1, "cpu") == 3.0
     assert bench.job_throughput(1, 8, 10, 2.0) == pytest.approx(8 * 10 / 2e-3)
+
+
+def test_both_bench_arms_report_the_same_config():
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2607_24331_gb300 import synth as S
+
+    for cfg in (1, 4):
+        c = bench.workload_config(S.workload(cfg), 2)
+        assert c["workload"] == S.workload(cfg).name and c["parallelism"] == "replicas x2"
+        assert set(c) == {"workload", "batch", "context", "layers", "step", "l2", "parallelism"}
