@@ -253,6 +253,76 @@ def job_throughput(world: int, batch: int, steps: int, t_ms: float) -> float:
 
 
 # ---------------------------------------------------------------------------
+# per-kernel breakdown of one decode call
+# ---------------------------------------------------------------------------
+
+def decode_kernel_names(dck, buf):
+    """Kernels of one decode call, in launch order (from the launch count of a plain call)."""
+    dck.check(buf.run(), "decode")
+    n = dck.dck_last_launch_count()
+    if n == 4:
+        return ["factor_prep", "scores", "absorb", "combine"]
+    if n == 2:
+        return ["decode_simt", "combine"]
+    return [f"kernel{i}" for i in range(n)]
+
+
+def kernel_work(buf, name):
+    """Algorithmic bytes and tensor flops of one kernel of a decode call."""
+    s = buf.spec
+    el = 2 if s.dtype == "bf16" else 4
+    d = s.head_dim
+    key_flops = buf.n_rows * 2 * sum(r * len(g) for g, r in zip(s.groups, s.ranks)) * d
+    val_flops = buf.n_rows * 2 * s.n_q_heads * s.rank_v
+    bk = s.bk_offsets()[-1] * el
+    bv = s.rank_v * s.n_kv_heads * d * el
+    qo = buf.B * s.n_q_heads * d * el
+    if name == "scores":
+        return buf.n_rows * s.rank_k * el + bk + qo, key_flops
+    if name == "absorb":
+        return buf.n_rows * s.rank_v * el, val_flops
+    if name == "combine":
+        return bv + qo, 0
+    if name == "factor_prep":
+        return bk + qo, 0
+    if name == "decode_simt":
+        return buf.n_rows * (s.rank_k + s.rank_v) * el + bk + qo, 0
+    return 0, 0
+
+
+def kernel_breakdown(dck, torch, stream, flush, buf, step_fn, names, peaks, K):
+    """Each kernel of the last layer's decode call timed between hook events recorded after every
+    launch (a separate capture: events between kernels stop a kernel from starting early under
+    programmatic dependent launch, so these sum to a little more than the call's own time)."""
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
+    for e_ in evs:
+        e_.record(stream)
+    torch.cuda.synchronize()
+    dck.check(dck.dck_set_timing_events(evs), "timing events")
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step_fn()
+    dck.check(dck.dck_set_timing_events(None), "timing events")
+    per = [[] for _ in names]
+    for k in range(max(K, 3) + 2):
+        flush.fill_(k & 0xFF)
+        g.replay()
+        torch.cuda.synchronize()
+        if k >= 2:
+            for i in range(len(names)):
+                per[i].append(evs[i].elapsed_time(evs[i + 1]))
+    out = []
+    for i, n in enumerate(names):
+        us = 1e3 * statistics.median(per[i])
+        by, fl = kernel_work(buf, n)
+        ent = {"kernel": n, "us": us, "alg_bytes": by, "tensor_flops": fl,
+               "hbm_frac": by / (us * 1e-6) / 1e9 / peaks["hbm_gbs"] if us > 0 else None,
+               "tensor_frac": fl / (us * 1e-6) / 1e12 / peaks["bf16_tflops"] if us > 0 else None}
+        out.append(ent)
+    return out
+
+
+# ---------------------------------------------------------------------------
 # the GPU arm
 # ---------------------------------------------------------------------------
 
@@ -328,20 +398,22 @@ def main():
     torch.cuda.synchronize()
     assert dck.dck_last_device_error(stream) == dck.DCK_OK
 
-    # ---- device-resident timed region: the step is captured once as a CUDA graph ----
+    # ---- device-resident timed region: the step is captured once as a CUDA graph;
+    # two hook events bracket each decode call (every kernel of it) ----
     K = args.steps
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
     kev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
     for e_ in kev:               # torch creates the CUDA event on first record
         e_.record(stream)
     torch.cuda.synchronize()
-    dck.check(dck.dck_set_timing_events(*kev), "timing events")
+    dck.check(dck.dck_set_timing_events(list(kev)), "timing events")
     graph = torch.cuda.CUDAGraph()
     launches[0] = 0
     with torch.cuda.graph(graph):
         step()
     per_step_launches = launches[0]
-    dck.check(dck.dck_set_timing_events(None, None), "timing events")
+    dck.check(dck.dck_set_timing_events(None), "timing events")
+    decode_kernels = decode_kernel_names(dck, layers[-1][0])
     for _ in range(args.warmup):
         flush.fill_(1)
         graph.replay()
@@ -414,8 +486,8 @@ def main():
     e2e_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in eev), world, dev)
     e2e_value = job_throughput(world, B, K, e2e_ms)
 
-    # ---- roofline of the attention kernels of one decode call (factor preparation, scores,
-    # absorption: the region between the timing events; one call = one layer) ----
+    # ---- roofline of one whole decode call (every kernel between the two hook events;
+    # one call = one layer), then a per-kernel breakdown from a separate capture ----
     peaks = load_peaks()
     buf0 = layers[-1][0]
     alg_bytes = buf0.algorithmic_bytes()
@@ -427,11 +499,12 @@ def main():
         sum((a.numel() + v.numel()) * a.element_size() for (_b, a, v, *_r) in layers)
     roof = {"bound": "hbm", "achieved": achieved_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
             "frac": achieved_gbs / peaks["hbm_gbs"], "traffic": profiled_traffic(args.config),
-            "kernel": "attention kernels of one call (factor prep + scores + absorption)", "kernel_us": 1e6 * k_avg_s,
+            "kernel": "one whole decode call: " + " + ".join(decode_kernels), "kernel_us": 1e6 * k_avg_s,
             "alg_bytes_per_launch": alg_bytes, "peak_source": peaks["source"],
             "tensor_tflops": tflops, "tensor_frac": tflops / peaks["bf16_tflops"],
             "roofline_us": 1e6 * max(alg_bytes / (peaks["hbm_gbs"] * 1e9), flops / (peaks["bf16_tflops"] * 1e12)),
-            "frac_of_nominal_8000gbs": achieved_gbs / NOMINAL_HBM_GBS}
+            "frac_of_nominal_8000gbs": achieved_gbs / NOMINAL_HBM_GBS,
+            "breakdown": kernel_breakdown(dck, torch, stream, flush, buf0, step, decode_kernels, peaks, K)}
 
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
             "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,

@@ -184,23 +184,31 @@ dck_status dck_decode_attention_noalloc(const dck_layer_desc* desc, const void* 
 dck_status dck_last_device_error(void* stream);
 
 /*
- * Kernel selection for the decode path (testing and measurement):
- *   0 = automatic (tensor-core kernel where supported, else the CUDA-core kernel)
+ * Test and measurement hooks.  Each acts only on later calls made by the
+ * calling thread (the settings are per thread), so concurrent callers on
+ * other threads and streams never see them.
+ *
+ * dck_set_decode_kernel - kernel selection of the decode path:
+ *   0 = automatic (tensor-core kernels where supported, else the CUDA-core kernel)
  *   1 = CUDA-core kernel only
- * Returns the previous value.  Affects subsequent calls in this process.
+ * Returns this thread's previous value.
  */
 int32_t dck_set_decode_kernel(int32_t which);
 
 /*
- * Measurement hook: when both are non-NULL, every later dck_decode_attention
- * call records the CUDA event ev_start (a cudaEvent_t) on its stream right
- * before its main attention kernel and ev_stop right after it, so a caller
- * can time that kernel alone.  NULL, NULL turns the hook off.  The events are
- * owned by the caller.
+ * dck_set_timing_events - timing hook of dck_decode_attention: `events` holds
+ * n CUDA events (cudaEvent_t, owned by the caller, 2 <= n <= 16).  Each later
+ * decode call records events[0] on its stream before its first kernel and
+ * events[min(k, n - 1)] after its k-th kernel (k = 1, 2, ...): n = 2 brackets
+ * the whole call, n = (kernels + 1) brackets every kernel.  Recording events
+ * between kernels can delay a kernel that would otherwise start early
+ * (programmatic dependent launch), so per-kernel brackets are for a
+ * breakdown, not for timing the call.  n = 0 switches the hook off (events
+ * is then ignored); any other invalid argument returns DCK_ERR_INVALID.
  */
-dck_status dck_set_timing_events(void* ev_start, void* ev_stop);
+dck_status dck_set_timing_events(void* const* events, int32_t n);
 
-/* Number of kernels the last decode / append call launched on the host side. */
+/* Number of kernels this thread's last decode / append call launched. */
 int32_t dck_last_launch_count(void);
 
 /*

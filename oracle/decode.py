@@ -113,16 +113,19 @@ def decode_attention(spec, q, kcache, vcache, B_k, B_v, seq_start, seq_lens,
         r0 = int(seq_start[b])
         t_pos = np.arange(L) + pos_offset
         q_pos = L - 1 + pos_offset
+        kv_cache = {}  # KV head -> (rotated keys, values): shared by its query heads
         for j in js:
             h = kv_head_of(j, Hq, Hkv)
-            g, s = _group_slot(groups, h)
-            r_g, n_g = ranks[g], len(groups[g])
-            Bg = B_k[blk_off[g]:blk_off[g + 1]].reshape(r_g, n_g * d)
-            C_g = kcache[r0:r0 + L, rank_off[g]:rank_off[g] + r_g]
-            k = C_g @ Bg[:, s * d:(s + 1) * d]                     # step 1, keys
-            v = vcache[r0:r0 + L] @ B_v[:, h * d:(h + 1) * d]      # step 1, values
-            k_rot = rope(k, t_pos, spec.rope_theta)                 # step 2
-            q_rot = rope(q[b, j], q_pos, spec.rope_theta)
+            if h not in kv_cache:
+                g, s = _group_slot(groups, h)
+                r_g, n_g = ranks[g], len(groups[g])
+                Bg = B_k[blk_off[g]:blk_off[g + 1]].reshape(r_g, n_g * d)
+                C_g = kcache[r0:r0 + L, rank_off[g]:rank_off[g] + r_g]
+                k = C_g @ Bg[:, s * d:(s + 1) * d]                     # step 1, keys
+                v = vcache[r0:r0 + L] @ B_v[:, h * d:(h + 1) * d]      # step 1, values
+                kv_cache[h] = (rope(k, t_pos, spec.rope_theta), v)      # step 2, keys
+            k_rot, v = kv_cache[h]
+            q_rot = rope(q[b, j], q_pos, spec.rope_theta)               # step 2, query
             sigma = (k_rot @ q_rot) / math.sqrt(d)                  # step 3
             e = np.exp(sigma - sigma.max())
             p = e / e.sum()
@@ -135,9 +138,25 @@ def decode_attention(spec, q, kcache, vcache, B_k, B_v, seq_start, seq_lens,
 
 
 def max_rel_err(got: np.ndarray, ref: np.ndarray) -> float:
-    """max |got - ref| / ||ref||_inf, the parity measure of the decode output."""
+    """max |got - ref| / ||ref||_inf, the parity measure of the decode output.
+
+    Only the entries the reference evaluated (finite in ``ref``; a subset of
+    heads or sequences leaves the rest NaN) are compared, and the scale is the
+    reference's largest magnitude over those entries.  A non-finite ``got`` at
+    any compared entry gives +inf, so it fails every tolerance; so does a
+    reference with nothing evaluated or all zeros (nothing to normalise by).
+    """
     ref = np.asarray(ref, dtype=np.float64)
     got = np.asarray(got, dtype=np.float64)
+    if got.shape != ref.shape:
+        raise ValueError(f"shape mismatch: got {got.shape}, reference {ref.shape}")
     m = np.isfinite(ref)
-    scale = np.abs(ref[m]).max()
-    return float(np.abs(got[m] - ref[m]).max() / scale)
+    if not m.any():
+        return math.inf
+    g, r = got[m], ref[m]
+    if not np.isfinite(g).all():
+        return math.inf
+    scale = np.abs(r).max()
+    if scale == 0.0:
+        return 0.0 if (g == 0.0).all() else math.inf
+    return float(np.abs(g - r).max() / scale)

@@ -308,7 +308,8 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, k, lt, a, bchunk, split);
+  e = cudaLaunchKernelEx(&cfg, k, lt, a, bchunk, split);
+  return e != cudaSuccess ? e : hook_launched(a.hook, s);
 }
 
 }  // namespace

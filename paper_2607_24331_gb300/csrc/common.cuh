@@ -53,10 +53,21 @@ struct DecodeArgs {
   float* part_ml;  // [n_slots, Hq, 2]  (running max in log2 units, sum)
   void* out;       // [B, Hq, d]
   int* err;
-  void* ev0;       // optional cudaEvent_t recorded right before / after the main kernel
-  void* ev1;
+  struct LaunchHook* hook;  // host-side launch count and optional timing events (never read by kernels)
   void* extra;     // workspace region of the tensor-core path (per-sequence folded factors)
 };
+
+// Host-side record of the kernels one entry-point call puts on its stream.
+// When `n_ev` > 0, ev[0] (a cudaEvent_t) is recorded before the call's first
+// kernel and ev[min(k, n_ev - 1)] after its k-th kernel, so that a caller can
+// time the whole call (n_ev = 2) or every kernel of it (n_ev = kernels + 1).
+struct LaunchHook {
+  void* const* ev = nullptr;
+  int n_ev = 0;
+  int count = 0;
+};
+inline cudaError_t hook_begin(LaunchHook* h, cudaStream_t s);     // before the first kernel
+inline cudaError_t hook_launched(LaunchHook* h, cudaStream_t s);  // after each kernel launch
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -68,6 +79,10 @@ cudaError_t launch_append_simt(const void* x, int n_tok, int D, const void* A_k,
                                int* err, cudaStream_t s);
 cudaError_t launch_synth_gaussian(void* dst, int64_t n, uint64_t key, int64_t start, float scale, int dtype,
                                   cudaStream_t s);
+// Host-side argument checks shared by the decode entry points (no CUDA call).
+dck_status decode_precheck(const dck_layer_desc* desc, const void* q, const void* kcache, const void* vcache,
+                           int64_t n_rows, const void* B_k, const void* B_v, const int64_t* d_seq_start,
+                           const int32_t* d_seq_len, int32_t batch, float rope_theta, const void* out);
 
 // ---------------------------------------------------------------------------
 // device helpers
@@ -203,5 +218,18 @@ inline cudaError_t record_timing_event(void* ev, cudaStream_t s) {
   if (st == cudaStreamCaptureStatusActive)
     return cudaEventRecordWithFlags(static_cast<cudaEvent_t>(ev), s, cudaEventRecordExternal);
   return cudaEventRecord(static_cast<cudaEvent_t>(ev), s);
+}
+
+inline cudaError_t hook_begin(LaunchHook* h, cudaStream_t s) {
+  if (!h || h->n_ev <= 0) return cudaSuccess;
+  return record_timing_event(h->ev[0], s);
+}
+
+inline cudaError_t hook_launched(LaunchHook* h, cudaStream_t s) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || !h) return e;
+  ++h->count;
+  if (h->n_ev <= 0) return cudaSuccess;
+  return record_timing_event(h->ev[h->count < h->n_ev - 1 ? h->count : h->n_ev - 1], s);
 }
 }  // namespace dck

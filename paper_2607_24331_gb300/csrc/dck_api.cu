@@ -13,7 +13,6 @@ bool simt_supports(const LayerTable& lt);
 bool combine_supports(const LayerTable& lt);
 bool tc_decode_supports(const LayerTable& lt, int dtype);
 size_t tc_decode_extra_ws(const LayerTable& lt, int batch, int64_t n_rows);
-int tc_decode_launches(const LayerTable& lt);
 cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s);
 bool tc_append_supports(int D, int Rk, int rv, int dtype);
 size_t tc_append_workspace(int n_tok, int Rk, int rv);
@@ -34,10 +33,13 @@ constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 int* g_err_ptr[kMaxDevices] = {};
 int g_sm_count[kMaxDevices] = {};
-std::atomic<int> g_decode_kernel{0};
-std::atomic<int> g_last_launches{0};
-std::atomic<void*> g_ev_start{nullptr};
-std::atomic<void*> g_ev_stop{nullptr};
+// Test and measurement hooks: per calling thread, so that a hook set by one
+// thread never acts on a call made by another.
+constexpr int kMaxHookEvents = 16;
+thread_local int t_decode_kernel = 0;
+thread_local int t_last_launches = 0;
+thread_local void* t_events[kMaxHookEvents] = {};
+thread_local int t_n_events = 0;
 
 bool device_state(int** err, int* sms) {
   int dev = 0;
@@ -152,14 +154,24 @@ const char* dck_status_string(int32_t s) {
 
 dck_status dck_validate_desc(const dck_layer_desc* desc) { return check_desc(desc); }
 
-int32_t dck_set_decode_kernel(int32_t which) { return g_decode_kernel.exchange(which); }
+int32_t dck_set_decode_kernel(int32_t which) {
+  const int prev = t_decode_kernel;
+  t_decode_kernel = which;
+  return prev;
+}
 
-int32_t dck_last_launch_count(void) { return g_last_launches.load(); }
+int32_t dck_last_launch_count(void) { return t_last_launches; }
 
-dck_status dck_set_timing_events(void* ev_start, void* ev_stop) {
-  if ((ev_start == nullptr) != (ev_stop == nullptr)) return DCK_ERR_INVALID;
-  g_ev_start = ev_start;
-  g_ev_stop = ev_stop;
+dck_status dck_set_timing_events(void* const* events, int32_t n) {
+  if (n == 0) {
+    t_n_events = 0;
+    return DCK_OK;
+  }
+  if (!events || n < 2 || n > kMaxHookEvents) return DCK_ERR_INVALID;
+  for (int i = 0; i < n; ++i)
+    if (!events[i]) return DCK_ERR_INVALID;
+  for (int i = 0; i < n; ++i) t_events[i] = events[i];
+  t_n_events = n;
   return DCK_OK;
 }
 
@@ -170,11 +182,14 @@ size_t dck_decode_workspace_size(const dck_layer_desc* desc, int32_t batch, int6
   return decode_ws_bytes(make_table(desc), batch, sms, desc->dtype, n_rows);
 }
 
-dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const void* kcache, const void* vcache,
-                                int64_t n_rows, const void* B_k, const void* B_v, const int64_t* d_seq_start,
-                                const int32_t* d_seq_len, int32_t batch, float rope_theta, void* out,
-                                void* workspace, size_t ws_bytes, void* stream) {
-  g_last_launches = 0;
+}  // extern "C"
+
+namespace dck {
+// Host-side argument checks of a decode call, in the order every decode entry
+// point applies them, before any CUDA call.
+dck_status decode_precheck(const dck_layer_desc* desc, const void* q, const void* kcache, const void* vcache,
+                           int64_t n_rows, const void* B_k, const void* B_v, const int64_t* d_seq_start,
+                           const int32_t* d_seq_len, int32_t batch, float rope_theta, const void* out) {
   dck_status st = check_desc(desc);
   if (st != DCK_OK) return st;
   if (batch < 0 || batch > kMaxBatch || n_rows < 0) return DCK_ERR_INVALID;
@@ -185,6 +200,20 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const
   if (!aligned(q, el) || !aligned(out, el) || !aligned(kcache, 16) || !aligned(vcache, 16) || !aligned(B_k, 16) ||
       !aligned(B_v, 16))
     return DCK_ERR_INVALID;
+  return DCK_OK;
+}
+}  // namespace dck
+
+extern "C" {
+
+dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const void* kcache, const void* vcache,
+                                int64_t n_rows, const void* B_k, const void* B_v, const int64_t* d_seq_start,
+                                const int32_t* d_seq_len, int32_t batch, float rope_theta, void* out,
+                                void* workspace, size_t ws_bytes, void* stream) {
+  t_last_launches = 0;
+  const dck_status st =
+      decode_precheck(desc, q, kcache, vcache, n_rows, B_k, B_v, d_seq_start, d_seq_len, batch, rope_theta, out);
+  if (st != DCK_OK || batch == 0) return st;
   int* err = nullptr;
   int sms = 0;
   if (!device_state(&err, &sms)) return DCK_ERR_CUDA;
@@ -214,17 +243,19 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const
   a.extra = static_cast<char*>(workspace) + decode_ws_parts(lt, batch, sms, n_rows);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e;
-  const bool use_tc = g_decode_kernel.load() == 0 && n_rows < (int64_t(1) << 31) - 256 &&
+  const bool use_tc = t_decode_kernel == 0 && n_rows < (int64_t(1) << 31) - 256 &&
                       tc_decode_supports(lt, desc->dtype);
-  a.ev0 = g_ev_start.load();
-  a.ev1 = g_ev_stop.load();
+  LaunchHook hook;
+  hook.ev = t_events;
+  hook.n_ev = t_n_events;
+  a.hook = &hook;
   a.split_extra = use_tc ? 1 : 0;
   if (use_tc) e = launch_decode_tc(lt, a, s);
   else e = launch_decode_simt(lt, a, desc->dtype, s);
   if (e != cudaSuccess) return DCK_ERR_CUDA;
   e = launch_combine(lt, a, desc->dtype, s);
+  t_last_launches = hook.count;
   if (e != cudaSuccess) return DCK_ERR_CUDA;
-  g_last_launches = (use_tc ? tc_decode_launches(lt) : 1) + 1;
   return DCK_OK;
 }
 
@@ -238,7 +269,7 @@ size_t dck_latent_append_workspace_size(const dck_layer_desc* desc, int32_t n_to
 dck_status dck_latent_append(const dck_layer_desc* desc, const void* x, int32_t n_tok, const void* A_k,
                              const void* A_v, const int64_t* d_rows, void* kcache, void* vcache, int64_t n_rows,
                              void* workspace, size_t ws_bytes, void* stream) {
-  g_last_launches = 0;
+  t_last_launches = 0;
   dck_status st = check_desc(desc);
   if (st != DCK_OK) return st;
   if (n_tok < 0 || n_rows < 0) return DCK_ERR_INVALID;
@@ -262,7 +293,7 @@ dck_status dck_latent_append(const dck_layer_desc* desc, const void* x, int32_t 
                            desc->dtype, err, s);
   }
   if (e != cudaSuccess) return DCK_ERR_CUDA;
-  g_last_launches = launches;
+  t_last_launches = launches;
   return DCK_OK;
 }
 

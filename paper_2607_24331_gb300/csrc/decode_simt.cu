@@ -211,11 +211,9 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid(a.n_items, lt.Hkv);
-  if (a.ev0 && record_timing_event(a.ev0, s) != cudaSuccess) return cudaErrorUnknown;
+  if ((e = hook_begin(a.hook, s)) != cudaSuccess) return e;
   k<<<grid, kThreads, smem, s>>>(lt, a);
-  e = cudaGetLastError();
-  if (e == cudaSuccess && a.ev1) e = record_timing_event(a.ev1, s);
-  return e;
+  return hook_launched(a.hook, s);
 }
 
 }  // namespace

@@ -925,7 +925,7 @@ cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& m
   }
   factor_prep_kernel<kFold><<<dim3(pa.n_items, kFold ? a.B : 1), 256, 0, s>>>(lt, a, pa,
                                                                                 static_cast<uint8_t*>(a.extra));
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = hook_launched(a.hook, s);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.n_items);
@@ -937,7 +937,8 @@ cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& m
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kFold>, maps, lt, a, ta);
+  e = cudaLaunchKernelEx(&cfg, decode_tc_kernel<kFold>, maps, lt, a, ta);
+  return e != cudaSuccess ? e : hook_launched(a.hook, s);
 }
 
 // Units, items and per-group tables of a layer.  Returns false when the layer
@@ -1039,8 +1040,6 @@ size_t tc_decode_extra_ws(const LayerTable& lt, int batch, int64_t n_rows) {
   return extra_layout(lt, batch, n_rows).total;
 }
 
-int tc_decode_launches(const LayerTable&) { return 3; }
-
 cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) {
   const bool fold = lt.qpg == 1;
   if (!a.extra) return cudaErrorInvalidValue;
@@ -1074,8 +1073,9 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStre
     g_maps_next = (g_maps_next + 1) % kMapsCache;
     g_maps_n = std::min(g_maps_n + 1, kMapsCache);
   }
-  if (a.ev0 && record_timing_event(a.ev0, s) != cudaSuccess) return cudaErrorUnknown;
-  cudaError_t e = fold ? launch_mode<true>(lt, a, maps, ta, pa, s) : launch_mode<false>(lt, a, maps, ta, pa, s);
+  cudaError_t e = hook_begin(a.hook, s);
+  if (e != cudaSuccess) return e;
+  e = fold ? launch_mode<true>(lt, a, maps, ta, pa, s) : launch_mode<false>(lt, a, maps, ta, pa, s);
   if (e != cudaSuccess) return e;
   TcRegions r;
   r.pglob = ta.pglob;
@@ -1083,8 +1083,7 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStre
   r.max_tiles = ta.max_tiles;
   r.hq_pad = ta.hq_pad;
   e = launch_absorb_tc(lt, a, r, s);
-  if (e == cudaSuccess && a.ev1) e = record_timing_event(a.ev1, s);
-  return e;
+  return e != cudaSuccess ? e : hook_launched(a.hook, s);
 }
 
 }  // namespace dck

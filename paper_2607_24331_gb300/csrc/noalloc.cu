@@ -51,14 +51,12 @@ extern "C" dck_status dck_decode_attention_noalloc(const dck_layer_desc* desc, c
                                                    const void* B_v, const int64_t* d_seq_start,
                                                    const int32_t* d_seq_len, int32_t batch, float rope_theta,
                                                    void* out, void* stream) {
-  const dck_status st = dck_validate_desc(desc);
-  if (st != DCK_OK) return st;
-  if (batch < 0) return DCK_ERR_INVALID;
-  if (batch == 0)  // nothing to compute; the regular entry point returns DCK_OK without launching
-    return dck_decode_attention(desc, q, kcache, vcache, n_rows, B_k, B_v, d_seq_start, d_seq_len, batch,
-                                rope_theta, out, nullptr, 0, stream);
+  // the regular entry point's argument checks, in its order, before the size test
+  const dck_status st = dck::decode_precheck(desc, q, kcache, vcache, n_rows, B_k, B_v, d_seq_start, d_seq_len,
+                                             batch, rope_theta, out);
+  if (st != DCK_OK || batch == 0) return st;
   const size_t need = dck_decode_workspace_size(desc, batch, n_rows);
-  if (need == 0) return DCK_ERR_CUDA;  // the device could not be queried
+  if (need == 0) return DCK_ERR_CUDA;  // valid arguments: only a failed device query gives 0
   if (need > kNoallocScratchBytes) return DCK_ERR_WORKSPACE;  // beyond the fixed 32 MiB scratch
   void* ws = noalloc_scratch();
   if (!ws) return DCK_ERR_CUDA;

@@ -88,7 +88,7 @@ def lib() -> ctypes.CDLL:
     L.dck_last_launch_count.restype = I32
     L.dck_last_launch_count.argtypes = []
     L.dck_set_timing_events.restype = I32
-    L.dck_set_timing_events.argtypes = [P, P]
+    L.dck_set_timing_events.argtypes = [P, I32]
     L.dck_selftest_bounded_wait.restype = I32
     L.dck_selftest_bounded_wait.argtypes = [I64, P]
     L.dck_synth_gaussian.restype = I32
@@ -198,11 +198,13 @@ def dck_synth_gaussian(dst, n: int, key: int, start: int, scale: float, dtype: i
                                     int(dtype), _stream(stream))
 
 
-def dck_set_timing_events(ev_start, ev_stop) -> int:
-    """ev_* are torch.cuda.Event objects (or None to switch the hook off)."""
-    p0 = None if ev_start is None else ev_start.cuda_event
-    p1 = None if ev_stop is None else ev_stop.cuda_event
-    return lib().dck_set_timing_events(p0, p1)
+def dck_set_timing_events(events) -> int:
+    """``events``: torch.cuda.Event objects (already recorded once, so that the CUDA
+    events exist), or None / [] to switch this thread's hook off."""
+    if not events:
+        return lib().dck_set_timing_events(None, 0)
+    arr = (ctypes.c_void_p * len(events))(*[e.cuda_event for e in events])
+    return lib().dck_set_timing_events(arr, len(events))
 
 
 def dck_selftest_bounded_wait(limit_cycles: int, stream=None) -> int:

@@ -37,3 +37,47 @@ def assert_parity(got, ref, dtype, what=""):
     print(f"{what} max|d|/||o||inf = {err:.3e}")
     assert err <= TOL[dtype], (what, err)
     return err
+
+
+def sm_count():
+    return torch.cuda.get_device_properties(0).multi_processor_count
+
+
+def leftover_sequences(lens, sms):
+    """Sequences with tiles in the finely split leftover range of the tensor-core
+    path: with NT 128-token tiles and fewer than 8 per SM, tiles from
+    floor(NT / sms) * sms on are shared out by groups of heads."""
+    nts = [(int(L) + 127) // 128 for L in lens]
+    NT = sum(nts)
+    NTm = NT // sms * sms if NT // sms < 8 else NT
+    out, pre = [], 0
+    for b, n in enumerate(nts):
+        if n and pre + n > NTm:
+            out.append(b)
+        pre += n
+    return out
+
+
+def plant_needle(di, b, t, j, score=30.0):
+    """Rewrites token t of sequence b so that its key, for query head j, scores
+    `score` (natural-log units, after the 1/sqrt(d) scale) against that head's
+    query: the group latent is the direction that maximises the score,
+    c = alpha w / |w| with w = B_slot RoPE(RoPE(q_j, L - 1), -t), rounded to the
+    storage dtype.  Returns the row written."""
+    spec = di.spec
+    d = spec.head_dim
+    h = oracle.kv_head_of(j, spec.n_q_heads, spec.n_kv_heads)
+    g = next(i for i, hs in enumerate(spec.groups) if h in hs)
+    s = spec.groups[g].index(h)
+    r_g, n_g = spec.ranks[g], len(spec.groups[g])
+    off = spec.bk_offsets()
+    Bg = np.asarray(di.B_k[off[g]:off[g + 1]], dtype=np.float64).reshape(r_g, n_g * d)
+    B_slot = Bg[:, s * d:(s + 1) * d]
+    L = int(di.seq_lens[b])
+    qr = oracle.rope(np.asarray(di.q[b, j], dtype=np.float64), L - 1, spec.rope_theta)
+    w = B_slot @ oracle.rope(qr, -t, spec.rope_theta)
+    c = w * (score * np.sqrt(d) / (w @ w))
+    row = int(di.seq_start[b]) + t
+    r0 = spec.rank_offsets()[g]
+    di.kcache[row, r0:r0 + r_g] = S.round_to(c.astype(np.float32), spec.dtype)
+    return row

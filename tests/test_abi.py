@@ -74,3 +74,40 @@ def test_selftest_rejects_limits_out_of_range_without_launching():
     # checked on the host before any CUDA call (stream handle 0 is never used)
     assert dck.dck_selftest_bounded_wait(10, 0) == dck.DCK_ERR_INVALID
     assert dck.dck_selftest_bounded_wait(5_000_000_000, 0) == dck.DCK_ERR_INVALID
+
+
+def test_decode_entry_points_check_arguments_before_any_cuda_call():
+    """Both decode entry points run the same host-side checks, in the same
+    order, before touching the device: nothing here needs a GPU (stream 0 and
+    fake aligned addresses are never used)."""
+    L = dck.Layer.from_spec(S.workload(1).layer)
+    p = 1 << 20   # aligned, never dereferenced
+    lib = dck.lib()
+    args = dict(q=p, kc=p, vc=p, n_rows=100, bk=p, bv=p, st=p, ln=p, batch=2, theta=1e4, out=p)
+
+    def both(**kw):
+        a = dict(args, **kw)
+        r1 = lib.dck_decode_attention(L.ref, a["q"], a["kc"], a["vc"], a["n_rows"], a["bk"], a["bv"], a["st"],
+                                      a["ln"], a["batch"], a["theta"], a["out"], p, 1 << 30, 0)
+        r2 = lib.dck_decode_attention_noalloc(L.ref, a["q"], a["kc"], a["vc"], a["n_rows"], a["bk"], a["bv"],
+                                              a["st"], a["ln"], a["batch"], a["theta"], a["out"], 0)
+        return r1, r2
+
+    assert both(n_rows=-1) == (dck.DCK_ERR_INVALID,) * 2
+    assert both(q=None) == (dck.DCK_ERR_INVALID,) * 2
+    assert both(theta=-1.0) == (dck.DCK_ERR_INVALID,) * 2
+    assert both(batch=-3) == (dck.DCK_ERR_INVALID,) * 2
+    assert both(batch=5000) == (dck.DCK_ERR_INVALID,) * 2       # beyond the batch limit
+    assert both(q=p + 1) == (dck.DCK_ERR_INVALID,) * 2          # misaligned bf16 pointer
+    assert both(batch=0) == (dck.DCK_OK,) * 2                   # nothing to do, nothing launched
+
+
+def test_timing_hook_arguments():
+    lib = dck.lib()
+    assert lib.dck_set_timing_events(None, 0) == dck.DCK_OK
+    assert lib.dck_set_timing_events(None, 2) == dck.DCK_ERR_INVALID
+    import ctypes
+    one = (ctypes.c_void_p * 1)(1)
+    assert lib.dck_set_timing_events(one, 1) == dck.DCK_ERR_INVALID
+    nulls = (ctypes.c_void_p * 2)(None, None)
+    assert lib.dck_set_timing_events(nulls, 2) == dck.DCK_ERR_INVALID

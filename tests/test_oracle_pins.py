@@ -355,3 +355,53 @@ def test_table1_key_param_counts():
         assert row["recalkv"] % per_rank == 0, name
         r_sum = row["recalkv"] // per_rank
         assert oracle.recalkv_key_params(row["m"], row["n"], row["h"], r_sum) == row["recalkv"]
+
+
+# ---------------------------------------------------------------------------
+# the parity measure itself: max |got - ref| / ||ref||_inf over the entries the
+# reference evaluated (hand-computed cases)
+# ---------------------------------------------------------------------------
+
+def test_max_rel_err_hand_computed():
+    ref = np.array([[1.0, 2.5], [3.0, -5.0]])
+    got = np.array([[1.0, 2.0], [3.0, -4.0]])
+    # |d| = 0, 0.5, 0, 1.0 -> 1.0; ||ref||_inf = 5
+    assert max_rel_err(got, ref) == pytest.approx(0.2, abs=1e-15)
+    assert max_rel_err(ref, ref) == 0.0
+
+
+def test_max_rel_err_normalises_by_the_reference():
+    ref = np.array([2.0, -4.0])
+    got = np.array([2.0, -3.0])
+    assert max_rel_err(got, ref) == pytest.approx(0.25, abs=1e-15)   # 1 / 4, not 1 / 3
+    # scaling `got` alone moves the numerator only
+    assert max_rel_err(10 * got, ref) == pytest.approx(26.0 / 4.0, abs=1e-12)   # |20-2|, |-30+4|
+
+
+def test_max_rel_err_non_finite_got_fails_every_tolerance():
+    ref = np.array([1.0, 2.0, 3.0])
+    for bad in (np.nan, np.inf, -np.inf):
+        got = np.array([1.0, bad, 3.0])
+        e = max_rel_err(got, ref)
+        assert e == math.inf and not e <= 1e30
+
+
+def test_max_rel_err_ignores_entries_the_reference_did_not_evaluate():
+    ref = np.array([[1.0, np.nan], [np.nan, -2.0]])
+    got = np.array([[1.1, 123.0], [np.nan, -2.0]])
+    assert max_rel_err(got, ref) == pytest.approx(0.05, abs=1e-15)   # 0.1 / 2
+    with pytest.raises(ValueError):
+        max_rel_err(got[:1], ref)
+    assert max_rel_err(got, np.full_like(ref, np.nan)) == math.inf
+
+
+def test_oracle_kv_reuse_equals_one_head_at_a_time():
+    """Evaluating all heads at once (keys and values of a KV head reused by its
+    query heads) equals evaluating each head alone."""
+    spec = small_spec(8, 4, 16, ((2, 0), (1,), (3,)), (8, 16, 4), 12)
+    lens = [7, 30]
+    args = random_inputs(spec, lens, seed=13, q_std=2.0)
+    full = decode_attention(spec, *args)
+    for j in range(8):
+        one = decode_attention(spec, *args, heads=[j])
+        np.testing.assert_array_equal(one[:, j], full[:, j])
