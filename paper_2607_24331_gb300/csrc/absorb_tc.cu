@@ -1,12 +1,14 @@
 // Value absorption in latent space on the tensor cores (Sec. III-D: the value
 // up-projection x W^(v) ~ z_v R_v is applied once, after the attention sum):
-//   U_seg[:, j] = sum over the tiles of a sequence segment of C_v[tile]^T P_tile[:, j]
+//   U_seg[:, j] = sum over the 128-token tiles of a segment of C_v[tile]^T P_tile[:, j]
 // with P_tile the bf16 probabilities the scores kernel wrote (already the
 // 128B-swizzled image of the UMMA B operand) and C_v[tile] the tile's value
 // latents [128 tokens x r_v].  The segments and their partial slots are those
-// of the scores kernel (the same split of the flattened tiles over the same
-// number of CTAs: whole main tiles per CTA, every extra tile a segment of its
-// own), which has already written each segment's reference max and row sum.
+// of the scores kernel (the pair-tile plan of tc_common.cuh): CTA c = 2p + h
+// absorbs half h of CTA pair p's main pair tiles, one segment per sequence,
+// and a share of the extra 128-token tiles by r_v chunks, each a segment of
+// its own; the scores kernel has already written each segment's reference max
+// and row sum.
 //
 // The scores kernel's reference max of a head can rise from one tile to the
 // next (it moves only when a tile's max exceeds it by 8); before such a tile
@@ -72,9 +74,73 @@ struct ASmem {
   uint64_t v_full[2 * kNVr], v_empty[2 * kNVr], p_full[kNP], p_empty[kNP];
   uint64_t drain, tile_ok, u_ready, u_free;
   int pneed[kNP];  // P slot's tile raises some head's reference max (set by the producer before the slot fills)
-  int scan[kAThreads];
+  int s256[kAThreads], s128[kAThreads];
   uint32_t tmem_base;
   int abort_flag;
+};
+
+// This CTA's share of the scores kernel's plan (see tc_common.cuh).
+struct AbsPlan {
+  int P, pr, hh, NPm, nc, c_lo, c_hi;
+};
+
+// One absorption segment: n 128-token tiles of one sequence, two tiles apart
+// in the flattened tile list (one half of consecutive pair tiles), r_v chunks
+// [ca, cb) of each, accumulated into partial slot `slot`.
+struct ASeg {
+  int L, n, ca, cb, t00;
+  int64_t slot, x0, row0;
+  __device__ int64_t x(int i) const { return x0 + 2 * (int64_t)i; }
+  __device__ int64_t row(int i) const { return row0 + (int64_t)kPTile * i; }
+  __device__ int nvalid(int i) const { return min(kTile, L - (t00 + kPTile * i)); }
+};
+
+// Segments of this CTA in order: half hh of each main run (the tiles that
+// exist: the odd half of a sequence's last pair tile may hold none), then each
+// extra 128-token tile (e, half) with chunks in [c_lo, c_hi).
+struct AWalk {
+  PairWalker wm, wx;
+  int ph = 0, hx = 2;
+  PSegment sx;
+  __device__ bool next(const DecodeArgs& a, const AbsPlan& pl, ASeg& s) {
+    PSegment sg;
+    while (ph == 0) {
+      if (!wm.next(a, sg)) {
+        ph = 1;
+        break;
+      }
+      const int n = min(sg.ntiles, max(0, (sg.n128 - pl.hh - 2 * sg.i0 + 1) / 2));
+      if (n == 0) continue;
+      s.L = sg.L;
+      s.n = n;
+      s.ca = 0;
+      s.cb = pl.nc;
+      s.t00 = sg.t0(0, pl.hh);
+      s.slot = pair_slot(pl.pr, sg.b, pl.hh);
+      s.x0 = sg.x128(0, pl.hh);
+      s.row0 = sg.row0 + s.t00;
+      return true;
+    }
+    while (true) {
+      if (hx == 2) {
+        if (!wx.next(a, sx)) return false;
+        hx = 0;
+      }
+      const int h2 = hx++;
+      const int e = sx.X0 - pl.NPm, q = 2 * e + h2;
+      const int ca = max(pl.c_lo - q * pl.nc, 0), cb = min(pl.c_hi - q * pl.nc, pl.nc);
+      if (ca >= cb || !sx.has(0, h2)) continue;
+      s.L = sx.L;
+      s.n = 1;
+      s.ca = ca;
+      s.cb = cb;
+      s.t00 = sx.t0(0, h2);
+      s.slot = pair_xslot(pl.P, a.B, e, h2);
+      s.x0 = sx.x128(0, h2);
+      s.row0 = sx.row0 + s.t00;
+      return true;
+    }
+  }
 };
 
 __global__ void __launch_bounds__(kAThreads, 1)
@@ -108,41 +174,36 @@ __global__ void __launch_bounds__(kAThreads, 1)
     tmem_alloc(&sm.tmem_base, kTmemCols);
     tmem_relinquish();
   }
-  // the work split of the scores kernel: main tiles [x0, x1) in segments per
-  // sequence, then whole extra tiles [e0, e1), each a segment of its own
-  const int NT = tile_count(a, sm.scan);
-  const Split sp(NT, a.n_items, a.split_extra != 0);
-  const bool fits = NT <= aa.max_tiles;  // else the scores kernel has reported the input
-  const int x0 = fits ? sp.main_begin(blockIdx.x, a.n_items) : 0;
-  const int x1 = fits ? sp.main_begin(blockIdx.x + 1, a.n_items) : 0;
-  // extra tiles by r_v chunks: chunks [c_lo, c_hi) of the flattened (extra tile, chunk) list
-  const int xc = sp.R * n_chunks;
-  const int c_lo = fits ? (int)((int64_t)blockIdx.x * xc / a.n_items) : 0;
-  const int c_hi = fits ? (int)((int64_t)(blockIdx.x + 1) * xc / a.n_items) : 0;
-  const int xe0 = sp.NTm + (c_lo < c_hi ? c_lo / n_chunks : 0), xe1 = sp.NTm + (c_lo < c_hi ? (c_hi - 1) / n_chunks + 1 : 0);
-  int bm, pm, bx, px;
-  tile_find(a, sm.scan, x0, bm, pm);
-  tile_find(a, sm.scan, xe0, bx, px);
-  const Walker walk_m{bm, pm, x0, x1, false}, walk_x{bx, px, xe0, xe1, true};
-  const bool has_work = x0 < x1 || xe0 < xe1;
-  // r_v chunks [ca, cb) of flattened tile x in phase ph (0: main, every chunk)
-  auto chunks_of = [&](int ph, int64_t x, int& ca, int& cb) {
-    ca = 0;
-    cb = n_chunks;
-    if (ph) {
-      const int e = (int)(x - sp.NTm);
-      ca = max(c_lo - e * n_chunks, 0);
-      cb = min(c_hi - e * n_chunks, n_chunks);
-    }
-  };
+  // the work plan of the scores kernel: half hh of pair pr's main pair tiles
+  // [X0, X1), one segment per sequence; then chunks [c_lo, c_hi) of the
+  // flattened (extra 128-token tile (e, half), r_v chunk) list
+  AbsPlan pl;
+  pl.P = a.n_items / 2;
+  pl.pr = blockIdx.x >> 1;
+  pl.hh = blockIdx.x & 1;
+  pl.nc = n_chunks;
+  const int NP = pair_tile_count(a, sm.s256, sm.s128);
+  const PSplit sp(NP, pl.P);
+  pl.NPm = sp.NPm;
+  const bool fits = sm.s128[kAThreads - 1] <= aa.max_tiles;  // else the scores kernel has reported the input
+  const int X0 = fits ? sp.main_begin(pl.pr, pl.P) : 0;
+  const int X1 = fits ? sp.main_begin(pl.pr + 1, pl.P) : 0;
+  const int xc = 2 * sp.R * n_chunks;
+  pl.c_lo = fits ? (int)((int64_t)blockIdx.x * xc / a.n_items) : 0;
+  pl.c_hi = fits ? (int)((int64_t)(blockIdx.x + 1) * xc / a.n_items) : 0;
+  const int q0 = pl.c_lo < pl.c_hi ? pl.c_lo / n_chunks : 0;
+  const int q1 = pl.c_lo < pl.c_hi ? (pl.c_hi - 1) / n_chunks + 1 : 0;
+  AWalk walk0;
+  walk0.wm = pair_walker_at(a, sm.s256, sm.s128, X0, X1, false);
+  walk0.wx = pair_walker_at(a, sm.s256, sm.s128, sp.NPm + q0 / 2, q0 < q1 ? sp.NPm + (q1 - 1) / 2 + 1 : sp.NPm, true);
+  const bool has_work = X0 < X1 || pl.c_lo < pl.c_hi;
   // the two MMA threads split a tile's chunks [ca, cb) at cm: thread 0 [ca, cm), thread 1 [cm, cb)
   auto chunk_mid = [](int ca, int cb) { return ca + (cb - ca + 1) / 2; };
-  const int64_t xbase = extra_slot_base(a.n_items, a.B);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
-  Segment seg;
+  ASeg seg;
   DCK_AB_TRACE(0);
 
   if (warp == 0) {
@@ -158,17 +219,15 @@ __global__ void __launch_bounds__(kAThreads, 1)
       // reference maxima (lane = head) of the previous tile and, loaded a tile
       // ahead so that their latency hides behind the value loads, of this one
       float m_prev = 0.f, m_pf = 0.f;
-      for (int ph = 0; ph < 2 && ok; ++ph)
-      for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
-        for (int i = 0; i < seg.ntiles && ok; ++i) {
-          const int64_t x = seg.x0 + i;
-          const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
-          int ca, cb;
-          chunks_of(ph, x, ca, cb);
+      for (AWalk walk = walk0; ok && walk.next(a, pl, seg);) {
+        for (int i = 0; i < seg.n && ok; ++i) {
+          const int64_t x = seg.x(i);
+          const int64_t yrow = seg.row(i);
+          const int ca = seg.ca, cb = seg.cb;
           if (lane == 0) {  // this CTA's first tile, then each next tile, toward L2
             for (int q = first ? 0 : 1; q < 2; ++q) {
-              if (q == 1 && i + 1 >= seg.ntiles) break;
-              const int64_t r0 = yrow + kTile * q, nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
+              if (q == 1 && i + 1 >= seg.n) break;
+              const int64_t r0 = seg.row(i + q), nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
               if (nr > 0)
                 prefetch_l2(static_cast<const __nv_bfloat16*>(a.vc) + r0 * lt.rv, (uint32_t)(nr * lt.rv * 2));
             }
@@ -220,7 +279,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
               m_now = m_pf;
               need = __any_sync(0xffffffffu, m_now > m_prev);
             }
-            if (i + 1 < seg.ntiles) m_pf = lane < Hq ? aa.mglob[(x + 1) * Hq + lane] : 0.f;
+            if (i + 1 < seg.n) m_pf = lane < Hq ? aa.mglob[seg.x(i + 1) * Hq + lane] : 0.f;
             m_prev = m_now;
             if (lane == 0) {
               const int sl = p_cnt % kNP;
@@ -251,9 +310,8 @@ __global__ void __launch_bounds__(kAThreads, 1)
       const uint32_t idesc_v = idesc_bf16(128, hq_pad, true, false);
       int vs = 0, vph = 0, p_cnt = 0, rc = 0, sgc = 0;
       bool ok = true;
-      for (int ph = 0; ph < 2 && ok; ++ph)
-      for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
-        for (int i = 0; i < seg.ntiles && ok; ++i) {
+      for (AWalk walk = walk0; ok && walk.next(a, pl, seg);) {
+        for (int i = 0; i < seg.n && ok; ++i) {
           const int psl = p_cnt % kNP;
           if (!(ok = mbar_wait(&sm.p_full[psl], (p_cnt / kNP) & 1, abort_flag))) break;
           if (i > 0) {
@@ -272,13 +330,12 @@ __global__ void __launch_bounds__(kAThreads, 1)
             tc_fence_after();
           }
           DCK_AB_TRACE(11);
-          const int nvalid = i == seg.ntiles - 1 ? seg.t_end - (seg.t_begin + kTile * i) : kTile;
+          const int nvalid = seg.nvalid(i);
           const uint32_t pbase = smem_u32(sm.p[psl]);
           // chunks in pairs: the K = 16 MMAs of one chunk form a dependent chain on
           // its accumulator (about 120 cycles each at N = Hq_pad), so two chunks'
           // chains are interleaved
-          int ca, cb;
-          chunks_of(ph, seg.x0 + i, ca, cb);
+          const int ca = seg.ca, cb = seg.cb;
           const int cm = chunk_mid(ca, cb);
           const int c0 = t ? cm : ca, c1 = t ? cb : cm;
           for (int c = c0; c < c1 && ok; c += 2) {
@@ -333,13 +390,11 @@ __global__ void __launch_bounds__(kAThreads, 1)
     int rc = 0, sgc = 0;
     bool ok = true;
     griddep_wait();  // the maxima come from the scores kernel
-    for (int ph = 0; ph < 2 && ok; ++ph)
-      for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
-      for (int i = 1; i < seg.ntiles && ok; ++i) {
-        const int64_t x = seg.x0 + i;
-        // reference maxima of this tile and the previous one, head = lane
-        const float mn = lane < Hq ? aa.mglob[x * Hq + lane] : 0.f;
-        const float mo = lane < Hq ? aa.mglob[(x - 1) * Hq + lane] : 0.f;
+    for (AWalk walk = walk0; ok && walk.next(a, pl, seg);) {
+      for (int i = 1; i < seg.n && ok; ++i) {
+        // reference maxima of this tile and the segment's previous one, head = lane
+        const float mn = lane < Hq ? aa.mglob[seg.x(i) * Hq + lane] : 0.f;
+        const float mo = lane < Hq ? aa.mglob[seg.x(i - 1) * Hq + lane] : 0.f;
         if (__any_sync(0xffffffffu, mn > mo)) {
           if (!(ok = wwait(&sm.drain, rc & 1, abort_flag))) break;
           tc_fence_after();
@@ -363,14 +418,12 @@ __global__ void __launch_bounds__(kAThreads, 1)
         }
       }
       if (!ok) break;
-      // segment end: U -> partial slot c + b (extra tile e: slot xbase + e)
+      // segment end: U -> the segment's partial slot
       if (!(ok = wwait(&sm.u_ready, sgc & 1, abort_flag))) break;
       tc_fence_after();
       DCK_AB_TRACE(22);
-      const int64_t slot = ph ? xbase + (seg.x0 - sp.NTm) : (int64_t)blockIdx.x + seg.b;
-      float* dst = a.part_u + slot * Hq * lt.rv + tau;
-      int ca, cb;  // the segment's last tile (extra segments have one)
-      chunks_of(ph, seg.x0 + seg.ntiles - 1, ca, cb);
+      float* dst = a.part_u + seg.slot * Hq * lt.rv + tau;
+      const int ca = seg.ca, cb = seg.cb;
       for (int c = ca; c < cb; ++c) {
         float v0[16], v1[16];
         tmem_ld16(tmem + lane_base + c * hq_pad, v0);

@@ -2,9 +2,12 @@
 //
 // Every work item wrote, for each sequence b it touched and each query head j,
 // the un-normalised latent accumulator u = sum_t 2^(s_t - m) v_t, its reference
-// max m (log2 units) and l = sum_t 2^(s_t - m) (the tensor-core path also one
-// such partial per extra tile, see tc_common.cuh).  For sequence b this kernel
-// takes the partials covering b's tiles, merges them with
+// max m (log2 units) and l = sum_t 2^(s_t - m).  CUDA-core path: item c covers
+// a contiguous range of 128-token tiles and writes slot c + b.  Tensor-core
+// path (the pair-tile plan of tc_common.cuh): each half of CTA pair p writes
+// slot 2 (p + b) + half, and each half of an extra pair tile e its own slot;
+// a slot whose half holds no token of b is not read.  For sequence b this
+// kernel takes the partials covering b's tiles, merges them with
 //   M = max m_c,  u = sum_c 2^(m_c - M) u_c,  l = sum_c 2^(m_c - M) l_c
 // and applies the value up-factor once per head (Sec. III-D, x W^(v) ~ z_v R_v):
 //   o_j = (u / l) B_v[:, h d : (h+1) d],  h = KV head of j.
@@ -25,6 +28,7 @@
 #include <cooperative_groups.h>
 
 #include "common.cuh"
+#include "tc_common.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -111,22 +115,25 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
     cp_async_commit();
   }
 
-  const int NT = build_tile_prefix(a.seq_len, a.seq_start, B, a.n_rows, prefix, scan, a.err, false);
-  // Partials of sequence b: the items c whose main tiles (the first NTm, split
-  // evenly in whole tiles) cover b's, in slots c + b; with the tensor-core
-  // split, also one slot per extra tile x >= NTm of b, slot xbase + x - NTm.
-  const int NTm = main_tiles(NT, a.n_items, a.split_extra != 0);
-  const int64_t xbase = (int64_t)a.n_items + B - 1;
-  for (int c = threadIdx.x; c <= a.n_items; c += kThreads) ibeg[c] = item_begin(c, NTm, a.n_items);
+  // tiles: pair tiles (tensor-core path) or 128-token tiles; items: CTA pairs or CTAs
+  const bool pairs = a.split_extra != 0;
+  const int n_it = pairs ? a.n_items / 2 : a.n_items;
+  const int NT = build_tile_prefix(a.seq_len, a.seq_start, B, a.n_rows, prefix, scan, a.err, false,
+                                   pairs ? 2 * kTile : kTile);
+  // Partials of sequence b: the items whose main tiles (the first NTm, split
+  // evenly in whole tiles) cover b's; on the tensor-core path also the extra
+  // pair tiles of b (x >= NTm), two slots (halves) per item and per extra tile.
+  const int NTm = pairs && NT / n_it < kFineSplitBelow ? NT / n_it * n_it : NT;
+  for (int c = threadIdx.x; c <= n_it; c += kThreads) ibeg[c] = item_begin(c, NTm, n_it);
   if (threadIdx.x < nrow) {
     const int b = b0 + threadIdx.x / qpg;
     const int me = min(prefix[b + 1], NTm);  // end of b's main tiles
     const bool any = me > prefix[b];
     int* r = rc + 4 * threadIdx.x;
-    r[0] = any ? item_of_tile(prefix[b], NTm, a.n_items) : 0;           // first main item
-    r[1] = any ? item_of_tile(me - 1, NTm, a.n_items) - r[0] + 1 : 0;  // main items
-    r[2] = max(prefix[b], NTm) - NTm;                                   // first extra tile
-    r[3] = max(prefix[b + 1] - NTm, r[2]) - r[2];                       // extra tiles
+    r[0] = any ? item_of_tile(prefix[b], NTm, n_it) : 0;           // first main item
+    r[1] = any ? item_of_tile(me - 1, NTm, n_it) - r[0] + 1 : 0;  // main items
+    r[2] = max(prefix[b], NTm) - NTm;                              // first extra tile
+    r[3] = max(prefix[b + 1] - NTm, r[2]) - r[2];                  // extra tiles
   }
   __syncthreads();
 
@@ -146,22 +153,41 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
     const int b = b0 + i / qpg, j = h * qpg + i % qpg;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     float M = -INFINITY, l = 0.f;
-    const int c0 = rc[4 * i], nm = rc[4 * i + 1], e0 = rc[4 * i + 2], ns = nm + rc[4 * i + 3];
+    const int c0 = rc[4 * i], nm = rc[4 * i + 1], e0 = rc[4 * i + 2];
+    const int nps = pairs ? 2 : 1;                         // slots per item or extra tile
+    const int ns = nps * (nm + rc[4 * i + 3]);
+    const int n128 = (valid_len(a.seq_len, a.seq_start, b, a.n_rows) + kTile - 1) / kTile;
     if (ns > 0) {
-      const int xb = (int)xbase + e0 - nm;                       // slot of partial q >= nm: xb + q
-      const int s0 = nm > 0 ? c0 + b : xb + nm;                    // a live slot
       for (int vv = 0; vv < ns; vv += kItemBatch) {
         float m[kItemBatch], lv[kItemBatch];
         float4 v[kItemBatch];
 #pragma unroll
         for (int u = 0; u < kItemBatch; ++u) {
-          const int q = vv + u;  // q-th partial of the row: main items, then extra tiles
-          const bool live = q < ns && (q >= nm || ibeg[c0 + q] != ibeg[c0 + q + 1]);
-          const int64_t sl = (int64_t)(live ? (q < nm ? c0 + b + q : xb + q) : s0) * Hq + j;
+          const int q = vv + u;  // q-th partial of the row: main items, then extra tiles; halves innermost
+          const int k = q / nps, hh = q % nps;
+          bool live = q < ns;
+          int64_t slot = 0;
+          if (live && k < nm) {  // item c0 + k
+            const int c = c0 + k;
+            live = ibeg[c] != ibeg[c + 1];
+            if (pairs) {
+              const int i0 = max(ibeg[c], prefix[b]) - prefix[b];  // b's first pair tile in the item
+              live = live && 2 * i0 + hh < n128;
+              slot = tc::pair_slot(c, b, hh);
+            } else {
+              slot = (int64_t)c + b;
+            }
+          } else if (live) {  // extra pair tile e (tensor-core path only)
+            const int e = e0 + k - nm;
+            live = 2 * (NTm + e - prefix[b]) + hh < n128;
+            slot = tc::pair_xslot(n_it, B, e, hh);
+          }
+          const int64_t sl = (live ? slot : 0) * Hq + j;
           const float2 ml = reinterpret_cast<const float2*>(a.part_ml)[sl];
+          const float4 uv = reinterpret_cast<const float4*>(a.part_u + sl * rv + r0)[r4];
           m[u] = live ? ml.x : -INFINITY;
-          lv[u] = ml.y;
-          v[u] = reinterpret_cast<const float4*>(a.part_u + sl * rv + r0)[r4];
+          lv[u] = live ? ml.y : 0.f;
+          v[u] = live ? uv : make_float4(0.f, 0.f, 0.f, 0.f);
         }
         float Mb = M;
 #pragma unroll

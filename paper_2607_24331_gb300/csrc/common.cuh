@@ -47,7 +47,7 @@ struct DecodeArgs {
   int64_t n_rows;
   int32_t B;
   int32_t n_items;
-  int32_t split_extra;  // tensor-core path: extra tiles split finely, each with its own partial slot
+  int32_t split_extra;  // tensor-core path: the pair-tile plan of tc_common.cuh (n_items = 2 x CTA pairs)
   float theta;
   float* part_u;   // [n_slots, Hq, rv]
   float* part_ml;  // [n_slots, Hq, 2]  (running max in log2 units, sum)
@@ -102,14 +102,14 @@ __device__ __forceinline__ float from_f32<float>(float v) { return v; }
 template <>
 __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
 
-// Number of 128-token tiles of every sequence, as an exclusive prefix in
+// Number of `tile`-token tiles of every sequence, as an exclusive prefix in
 // shared memory prefix[0..B].  Sequences whose rows fall outside the cache
 // count as empty and raise kErrBadSeq.  Must be called by the whole block.
 // Returns the total tile count NT.
 __device__ __forceinline__ int build_tile_prefix(const int32_t* __restrict__ seq_len,
                                                  const int64_t* __restrict__ seq_start, int B,
                                                  int64_t n_rows, int* prefix, int* scratch, int* err,
-                                                 bool report) {
+                                                 bool report, int tile = kTile) {
   const int nt = blockDim.x;
   const int per = (B + nt - 1) / nt;
   const int b0 = threadIdx.x * per;
@@ -121,7 +121,7 @@ __device__ __forceinline__ int build_tile_prefix(const int32_t* __restrict__ seq
       if (report) atomicOr(err, kErrBadSeq);
       L = 0;
     }
-    local += (int)((L + kTile - 1) / kTile);
+    local += (int)((L + tile - 1) / tile);
   }
   scratch[threadIdx.x] = local;
   __syncthreads();
@@ -138,7 +138,7 @@ __device__ __forceinline__ int build_tile_prefix(const int32_t* __restrict__ seq
     int64_t L = seq_len[b];
     int64_t st = seq_start[b];
     if (L < 0 || st < 0 || st + L > n_rows) L = 0;
-    run += (int)((L + kTile - 1) / kTile);
+    run += (int)((L + tile - 1) / tile);
   }
   int total = scratch[nt - 1];
   if (threadIdx.x == 0) prefix[B] = total;
@@ -155,7 +155,7 @@ __device__ __forceinline__ int valid_len(const int32_t* seq_len, const int64_t* 
   return (int)L;
 }
 
-__device__ __forceinline__ int item_begin(int c, int NT, int n_items) {
+__host__ __device__ __forceinline__ int item_begin(int c, int NT, int n_items) {
   return (int)(((int64_t)c * NT) / n_items);
 }
 

@@ -7,12 +7,14 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "tc_common.cuh"
 
 namespace dck {
 bool simt_supports(const LayerTable& lt);
 bool combine_supports(const LayerTable& lt);
 bool tc_decode_supports(const LayerTable& lt, int dtype);
 size_t tc_decode_extra_ws(const LayerTable& lt, int batch, int64_t n_rows);
+int tc_decode_pairs(const LayerTable& lt);
 cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s);
 bool tc_append_supports(int D, int Rk, int rv, int dtype);
 size_t tc_append_workspace(int n_tok, int Rk, int rv);
@@ -115,13 +117,14 @@ LayerTable make_table(const dck_layer_desc* d) {
   return lt;
 }
 
-// Partial slots: c + b for work item c and sequence b it touched (n_items + B - 1),
-// then one per extra tile of the tensor-core path: fewer than n_items, and no
-// more than the call's tiles (ceil(n_rows / 128) + B with non-overlapping sequences).
-size_t n_partial_slots(int batch, int n_items, int64_t n_rows) {
-  const int64_t tiles = (n_rows + 127) / 128 + batch;
-  const int64_t extra = std::min<int64_t>(n_items > 0 ? n_items - 1 : 0, tiles);
-  return (size_t)n_items + (batch > 0 ? batch - 1 : 0) + (size_t)extra;
+// Partial slots: CUDA-core path, c + b for work item c (one per SM) and
+// sequence b it touched; tensor-core path, two per (CTA pair, sequence) and two
+// per extra pair tile (tc::pair_slot_count, at most SMs / 2 pairs).  The
+// workspace holds the larger count, so one size query serves both paths.
+size_t n_partial_slots(int batch, int sms, int64_t n_rows) {
+  const int64_t simt = (int64_t)sms + (batch > 0 ? batch - 1 : 0);
+  const int64_t tc = tc::pair_slot_count(sms / 2, batch, n_rows);
+  return (size_t)std::max(simt, tc);
 }
 
 size_t decode_ws_parts(const LayerTable& lt, int batch, int n_items, int64_t n_rows) {
@@ -243,13 +246,16 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const
   a.extra = static_cast<char*>(workspace) + decode_ws_parts(lt, batch, sms, n_rows);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e;
-  const bool use_tc = t_decode_kernel == 0 && n_rows < (int64_t(1) << 31) - 256 &&
-                      tc_decode_supports(lt, desc->dtype);
+  const int pairs = t_decode_kernel == 0 && n_rows < (int64_t(1) << 31) - 256 && tc_decode_supports(lt, desc->dtype)
+                        ? std::min(tc_decode_pairs(lt), sms / 2)
+                        : 0;
+  const bool use_tc = pairs > 0;
   LaunchHook hook;
   hook.ev = t_events;
   hook.n_ev = t_n_events;
   a.hook = &hook;
   a.split_extra = use_tc ? 1 : 0;
+  if (use_tc) a.n_items = 2 * pairs;  // the tensor-core kernels run on the pairs' SMs
   if (use_tc) e = launch_decode_tc(lt, a, s);
   else e = launch_decode_simt(lt, a, desc->dtype, s);
   if (e != cudaSuccess) return DCK_ERR_CUDA;

@@ -1,15 +1,19 @@
 // Tensor-core (tcgen05) decode attention over DynaCalKV latent caches, bf16:
 // the scores kernel (key reconstruction, RoPE, scores, online softmax).
 //
-// One persistent CTA per SM walks its share of 128-token tiles (see
-// DecodeArgs).  For every tile and every key group g (Sec. III-C) the group's
-// latent tile C_g [128 tokens x r_g] meets, on the tensor cores, the factor
-// columns of the group's KV heads, two heads per MMA where the group has them
-// (tcgen05.mma, M = 128 tokens, N = 256 or 128, K = r_g, fp32 accumulator in
-// TMEM).  A pair shares every read of the latent operand: one-head MMAs that
-// read fresh shared-memory operands run the tensor pipe at about half rate.
-// Two 256-column accumulators (all of TMEM) let the epilogue read one unit
-// while the tensor core computes the next.  Per head:
+// The kernel runs as persistent CTA pairs: a cluster of two CTAs on the two
+// SMs of a TPC issues one tcgen05 pair MMA (cta_group::2) over a pair tile of
+// 256 tokens, the even CTA holding the first 128 tokens' latents and the odd
+// CTA the rest (the work plan is in tc_common.cuh).  For every pair tile and
+// every key group g (Sec. III-C) the group's latent tile C_g [256 tokens x r_g]
+// meets the factor columns of the group's KV heads, two heads per MMA where the
+// group has them (M = 256 tokens, N = 256 or 128, K = r_g; each CTA holds the
+// factor columns of one head, or one half of a lone head, and receives the
+// fp32 accumulator rows of its own 128 tokens in its TMEM).  A pair MMA moves
+// each SM's share of the factor operand once per 256 tokens instead of once
+// per 128, and halves the MMA instructions per token.  Two 256-column
+// accumulators (all of TMEM) let the epilogue read one unit while the tensor
+// cores compute the next.  Per head:
 //
 //  * key mode (several query heads per KV head): the factor is B_g[:, slot(h)],
 //    the product is the reconstructed key K^_h = C_g B_g[:, slot(h)]
@@ -28,40 +32,47 @@
 // Factor items (one latent piece's ranks x 128 columns of each head of a
 // unit) are prepared once per call by factor_prep_kernel as the exact
 // 128B-swizzled shared-memory image of the UMMA B operand (heads * ranks * 256
-// bytes each, in consumption order), so each item arrives with one 1-D bulk copy.
+// bytes each, in consumption order); each CTA of a pair loads its half of an
+// item (its head, or its half of a lone head) with one TMA copy.
 //
 // Scores are in log2 units; the online softmax keeps a per-head reference max
 // that moves only when a tile's max exceeds it by 8 (probabilities <= 256).
-// Each tile's probabilities P (bf16, laid out as the B operand of the value
-// absorption) and the reference maxima they were computed with go to the
-// workspace; at the end of each sequence segment the reference max and the
-// row sum (over the rounded P) are written as the segment's split partial.
-// The absorption kernel (absorb_tc.cu) forms U = C_v^T P from them.
+// Each CTA runs the softmax of its own 128-token halves: their probabilities P
+// (bf16, laid out as the B operand of the value absorption) and the reference
+// maxima they were computed with go to the workspace per 128-token tile; at
+// the end of each segment the reference max and the row sum (over the rounded
+// P) are written as the segment's split partial.  The absorption kernel
+// (absorb_tc.cu) forms U = C_v^T P from them.
 //
-// Warp roles (384 threads query-folded, 352 key mode).  Every TMA or
-// bulk-copy instruction costs its issuing thread a long round trip, so loads
-// are issued by two producer warps, each putting several copies (one per lane)
-// into one instruction:
+// Warp roles (384 threads query-folded, 352 key mode), in both CTAs unless
+// noted.  Every TMA instruction costs its issuing thread a long round trip, so
+// loads are issued by two producer warps, each putting several copies (one per
+// lane) into one instruction; the copies of both CTAs complete on the even
+// CTA's barriers, which its MMA threads wait on:
 //   warp 0     latent pieces of C_g (ring A)
 //   warp 10    factor items (ring W; query-folded mode: one ring per MMA thread)
-//   warp 1     TMEM owner; its lane 0 issues MMAs.  On this GPU every barrier
-//              test, commit or fence costs the issuing thread a dependent round
-//              trip of 100-500 cycles, longer than the MMAs of a factor item, so
-//              in query-folded mode lane 0 of warp 11 issues every other unit
-//              into the other accumulator and the two threads' bookkeeping
-//              overlaps the other's MMAs
+//   warp 1     TMEM owner; in the even CTA its lane 0 issues pair MMAs.  On this
+//              GPU every barrier test, commit or fence costs the issuing thread a
+//              dependent round trip of 100-500 cycles, so in query-folded mode
+//              lane 0 of the even CTA's warp 11 issues every other unit into the
+//              other accumulator and the two threads' bookkeeping overlaps the
+//              other's MMAs; the MMA commits arrive on both CTAs' barriers
 //   warps 2-9  epilogue: each TMEM lane quadrant (32 tokens) is served by two
 //              warps that split the 64 RoPE frequency pairs of a head; their
 //              partial scores go to one shared-memory array per frequency
-//              half, summed at the tile end.
+//              half, summed at the tile end.  Both CTAs' epilogues release an
+//              accumulator on the even CTA's barrier.
 // Every wait is bounded (about 2 s); on expiry the CTA stops issuing work,
-// records kErrTimeout, waits for work in flight and still releases TMEM.
+// tells its peer to stop, records kErrTimeout, waits for work in flight and
+// still releases TMEM.
 //
-// Shared-memory operand layouts (128B swizzle unless noted):
+// Shared-memory operand layouts (128B swizzle unless noted), identical in both
+// CTAs (a pair MMA reads the same offsets in each):
 //   A slot  [128 tokens][w ranks] K-major, w in {64, 32, 16} with 128/64/32B
-//           swizzle: UMMA operand A of the reconstruction;
-//   W slot  [nh heads][2 halves][w ranks][64 columns] MN-major: operand B
-//           (N = 128 nh, the 64-column atoms w * 128 bytes apart);
+//           swizzle: this CTA's rows of the UMMA operand A;
+//   W slot  [2 halves][w ranks][64 columns] MN-major (one head), or
+//           [w ranks][64 columns] (half of a lone head): this CTA's columns of
+//           operand B (the 64-column atoms w * 128 bytes apart);
 // P ([2 token atoms][Hq_pad heads][64 tokens] bf16, K-major: the absorption's
 // operand B) is written straight to the workspace by the tile-end owners.
 #include <algorithm>
@@ -73,13 +84,6 @@
 #include "tc_host.h"
 #include "tmap.h"
 
-#ifndef DCK_TC_TRACE
-#define DCK_TC_TRACE(code) ((void)0)
-#endif
-#ifndef DCK_TC_TRACE_FLUSH
-#define DCK_TC_TRACE_FLUSH() ((void)0)
-#endif
-
 namespace dck {
 namespace {
 
@@ -87,15 +91,15 @@ using namespace sm100;
 using namespace tc;
 
 constexpr int kD = 128;
-constexpr int kSlot = 16384;     // latent slots
-constexpr int kSlotW = 32768;    // factor slots: up to 2 heads x 64 ranks x 128 columns
-constexpr int kNA = 4;           // latent-piece ring depth
+constexpr int kSlot = 16384;     // latent slots: 128 tokens x 64 ranks
+constexpr int kSlotW = 16384;    // factor slots: one head (2 x 64 ranks x 64 columns) of an item
 constexpr int kMaxGroupsTc = 16;
 constexpr int kMaxPieces = 5;
 constexpr int kMaxHqTc = 32;
 constexpr int kMaxItems = 256;
 constexpr int kMaxUnits = 32;
 constexpr int kEpiThreads = 256;
+constexpr int kEpiWarps = kEpiThreads / 32;
 constexpr float kRescaleThr = 8.f;  // log2 units: probabilities stay <= 256
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kKCols = 256;    // TMEM columns of one key accumulator
@@ -105,17 +109,22 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 template <bool kFold>
 struct Ring {
-  static constexpr int NW = kFold ? 4 : 3;    // factor-item slots (key mode keeps 16 KB for queries)
+  static constexpr int NA = kFold ? 5 : 4;    // latent-piece slots (16 KB each)
+  static constexpr int NW = kFold ? 6 : 6;    // factor-item slots (half items: 16 KB each)
   // MMA-issuing threads, each with its own factor ring: two in query-folded
   // mode; key mode's units carry up to four items, which one thread's ring of
-  // all four slots streams better
+  // all slots streams better
   static constexpr int kMma = kFold ? 2 : 1;
   static constexpr int NWt = NW / kMma;       // slots of one MMA thread's ring
   static constexpr int kThreads = kFold ? 384 : 352;
 };
 
+// Latent-piece maps (box 64/32/16 ranks x 128 tokens, 128/64/32B swizzle) and
+// factor-image maps (rows of 128 bytes, box 16/32/64/128 rows, no swizzle: the
+// images are stored pre-swizzled).
 struct Maps {
   CUtensorMap kc64, kc32, kc16;
+  CUtensorMap im[4];
 };
 
 // Per-group facts the hot loops need; copied to shared memory at kernel start
@@ -131,13 +140,14 @@ struct GroupSm {
   int16_t u0;            // the group's first unit in the tile's unit order
   int16_t k[kMaxPieces]; // first rank of each piece
   int16_t i0;            // the group's first factor item in the tile's item order
+  int16_t rank;          // r_g
 };
 
 struct TcArgs {
   int hq_pad;
   int n_items;                   // factor items per tile
+  int n_pairs;                   // P
   int64_t fimg_seq_bytes;        // factor image bytes per sequence (query-folded mode)
-  const uint8_t* fimg;           // factor images (workspace)
   uint8_t* pglob;                // per-tile P images (workspace)
   float* mglob;                  // per-tile reference maxima (workspace)
   int64_t max_tiles;
@@ -152,7 +162,7 @@ struct TcArgs {
 
 template <bool kFold>
 struct Smem {
-  uint8_t a[kNA][kSlot];
+  uint8_t a[Ring<kFold>::NA][kSlot];
   uint8_t w[Ring<kFold>::NW][kSlotW];
   // scores [frequency half][query head][token]: each half's partial scores by
   // plain stores, summed at the tile end
@@ -162,12 +172,14 @@ struct Smem {
   // of its 32 tokens' rotated keys [token][32] bf16 (the A operand), 16-byte
   // chunks swizzled by (token / 2) % 4
   __nv_bfloat16 qr[kFold ? 2 : kMaxHqTc * kD];
-  uint8_t kst[kFold ? 1 : kEpiThreads / 32][kFold ? 16 : 32 * 64];
+  uint8_t kst[kFold ? 1 : kEpiWarps][kFold ? 16 : 32 * 64];
   double om64[kD / 2];
   float om32[kD / 2];
   float beta[kD / 2];
-  uint64_t a_full[kNA], a_empty[kNA];
-  uint64_t w_full[Ring<kFold>::NW], w_empty[Ring<kFold>::NW];
+  // latent ring: one full/empty pair per group instance; factor rings: one
+  // pair per unit (batch of items) of each MMA thread (see SlotFifo)
+  uint64_t g_full[kFifoBars], g_empty[kFifoBars];
+  uint64_t u_full[Ring<kFold>::kMma][kFifoBars], u_empty[Ring<kFold>::kMma][kFifoBars];
   uint64_t k_full[2], k_empty[2], epi_bar;
   GroupSm grp[kMaxGroupsTc];
   int16_t order[kMaxHqTc];
@@ -198,6 +210,11 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
+// Rows (of 128 bytes) of a half item of `bytes` bytes -> factor-image map index.
+__device__ __forceinline__ int im_map_of(uint32_t half_rows) {
+  return half_rows == 16 ? 0 : (half_rows == 32 ? 1 : (half_rows == 64 ? 2 : 3));
+}
+
 // ---------------------------------------------------------------------------
 // the scores kernel
 // ---------------------------------------------------------------------------
@@ -206,7 +223,7 @@ template <bool kFold>
 __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     decode_tc_kernel(const __grid_constant__ Maps maps, const LayerTable lt, const DecodeArgs a,
                      const __grid_constant__ TcArgs ta) {
-  constexpr int NW = Ring<kFold>::NW, kMma = Ring<kFold>::kMma, NWt = Ring<kFold>::NWt;
+  constexpr int kMma = Ring<kFold>::kMma, NWt = Ring<kFold>::NWt, kNA = Ring<kFold>::NA;
   constexpr int kThreads = Ring<kFold>::kThreads;
   extern __shared__ uint8_t smem_raw[];
   Smem<kFold>& sm =
@@ -215,29 +232,32 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
   volatile int* abort_flag = &sm.abort_flag;
   const int hq_pad = ta.hq_pad;
   const int Hq = lt.Hq, qpg = lt.qpg;
+  const int hr = (int)cluster_ctarank();  // the half of every pair tile this CTA holds
+  const bool leader = hr == 0;            // the even CTA issues the pair MMAs
+  const int P = ta.n_pairs, pair = blockIdx.x >> 1;
   griddep_launch();  // the absorption kernel may start streaming values as CTAs finish
 
   // ---- setup -------------------------------------------------------------
   if (tid == 0) {
-    for (int i = 0; i < kNA; ++i) {
-      mbar_init(&sm.a_full[i], 1);
-      mbar_init(&sm.a_empty[i], kMma);  // released by every MMA thread
-    }
-    for (int i = 0; i < NW; ++i) {
-      mbar_init(&sm.w_full[i], 1);
-      mbar_init(&sm.w_empty[i], 1);
+    for (int i = 0; i < kFifoBars; ++i) {
+      mbar_init(&sm.g_full[i], 1);      // even CTA: its producer's expect_tx; both CTAs' copies complete on it
+      mbar_init(&sm.g_empty[i], kMma);  // released by every MMA thread (arrivals reach both CTAs)
+      for (int t = 0; t < kMma; ++t) {
+        mbar_init(&sm.u_full[t][i], 1);
+        mbar_init(&sm.u_empty[t][i], 1);
+      }
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sm.k_full[i], 1);
-      mbar_init(&sm.k_empty[i], kEpiThreads / 32);
+      mbar_init(&sm.k_empty[i], 2 * kEpiWarps);  // even CTA: both CTAs' epilogue warps
     }
-    mbar_init(&sm.epi_bar, kEpiThreads / 32);
+    mbar_init(&sm.epi_bar, kEpiWarps);
     sm.abort_flag = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(&sm.tmem_base, kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(&sm.tmem_base, kTmemCols);
+    tmem_relinquish_pair();
   }
   if (tid < lt.G) sm.grp[tid] = ta.grp[tid];
   if (tid < lt.Hkv) sm.order[tid] = ta.order[tid];
@@ -247,107 +267,122 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     sm.om64[tid] = ta.om[tid];
     sm.om32[tid] = (float)ta.om[tid];
   }
-  // Work of this CTA: main tiles [x0, x1) (every unit), then units [u_lo, u_hi)
-  // of the flattened (extra tile, unit) list, every extra tile a segment of its own.
+  // Work of this pair: main pair tiles [X0, X1) (every unit), then units
+  // [u_lo, u_hi) of the flattened (extra tile, unit) list, every extra tile a
+  // segment of its own.
   const int U = ta.n_units;
-  const int NT = tile_count(a, reinterpret_cast<int*>(sm.x));
-  const Split sp(NT, a.n_items, a.split_extra != 0);
+  // block-scan scratch in the latent ring: used only before the first copy is issued
+  int* const s256 = reinterpret_cast<int*>(sm.a[0]);
+  int* const s128 = s256 + kThreads;
+  const int NP = pair_tile_count(a, s256, s128);
+  const int NT128 = s128[kThreads - 1];
+  const PSplit sp(NP, P);
   // the per-tile stores are sized for non-overlapping sequences; more tiles
   // than that is reported as invalid input and nothing is computed
-  const bool fits = NT <= ta.max_tiles;
+  const bool fits = NT128 <= ta.max_tiles;
   if (!fits && tid == 0 && blockIdx.x == 0) atomicOr(a.err, kErrBadSeq);
-  const int x0 = fits ? sp.main_begin(blockIdx.x, a.n_items) : 0;
-  const int x1 = fits ? sp.main_begin(blockIdx.x + 1, a.n_items) : 0;
+  const int X0 = fits ? sp.main_begin(pair, P) : 0;
+  const int X1 = fits ? sp.main_begin(pair + 1, P) : 0;
   const int xu = sp.R * U;
-  const int u_lo = fits ? (int)((int64_t)blockIdx.x * xu / a.n_items) : 0;
-  const int u_hi = fits ? (int)((int64_t)(blockIdx.x + 1) * xu / a.n_items) : 0;
-  const int xe0 = sp.NTm + (u_lo < u_hi ? u_lo / U : 0), xe1 = sp.NTm + (u_lo < u_hi ? (u_hi - 1) / U + 1 : 0);
-  int bm, pm, bx, px;
-  tile_find(a, reinterpret_cast<const int*>(sm.x), x0, bm, pm);
-  tile_find(a, reinterpret_cast<const int*>(sm.x), xe0, bx, px);
-  const Walker walk_m{bm, pm, x0, x1, false}, walk_x{bx, px, xe0, xe1, true};
-  const bool has_work = x0 < x1 || xe0 < xe1;
-  const int64_t xbase = extra_slot_base(a.n_items, a.B);
-  // units [ua, ub) of flattened tile x in phase ph (0: main, 1: extra)
-  auto units_of = [&](int ph, int x, int& ua, int& ub) {
+  const int u_lo = fits ? (int)((int64_t)pair * xu / P) : 0;
+  const int u_hi = fits ? (int)((int64_t)(pair + 1) * xu / P) : 0;
+  const int xe0 = sp.NPm + (u_lo < u_hi ? u_lo / U : 0), xe1 = sp.NPm + (u_lo < u_hi ? (u_hi - 1) / U + 1 : 0);
+  const PairWalker walk_m = pair_walker_at(a, s256, s128, X0, X1, false);
+  const PairWalker walk_x = pair_walker_at(a, s256, s128, xe0, xe1, true);
+  const bool has_work = X0 < X1 || xe0 < xe1;  // the same in both CTAs of the pair
+  // units [ua, ub) of flattened pair tile X in phase ph (0: main, 1: extra)
+  auto units_of = [&](int ph, int X, int& ua, int& ub) {
     ua = 0;
     ub = U;
     if (ph) {
-      const int e = x - sp.NTm;
+      const int e = X - sp.NPm;
       ua = max(u_lo - e * U, 0);
       ub = min(u_hi - e * U, U);
     }
   };
   for (int i = tid; i < (int)(sizeof(sm.x) / sizeof(float)); i += kThreads) sm.x[i] = 0.f;
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();  // both CTAs' barriers initialised and TMEM allocated
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
-  Segment seg;
-  DCK_TC_TRACE(0);
+  // shared::cluster addresses: a barrier of the even CTA, or a word of the peer
+  auto lead = [](const void* p) { return mapa_shared(smem_u32(p), 0); };
+  auto peer = [hr](const void* p) { return mapa_shared(smem_u32(p), (uint32_t)(hr ^ 1)); };
+  // a wait that gave up stops the peer too
+  auto stop_peer = [&]() { st_cluster_u32(peer(&sm.abort_flag), 1u); };
+  PSegment seg;
 
-  // Factor items of one unit into MMA thread rw's ring (query-folded mode): up to
-  // NWt bulk copies per instruction, one per lane, as their slots come free.
-  auto put_unit_items = [&](int rw, int& wc, int n, int np, const uint8_t* img, uint64_t pol) -> bool {
+  // Half items (this CTA's head, or its half of a lone head) of one unit into
+  // MMA thread rw's ring, in batches of at most NWt items: each batch is one
+  // instance of the ring (one full barrier, which the even CTA's lane 0 arms
+  // with the bytes of both CTAs' copies; one TMA copy per lane).
+  auto put_unit = [&](int rw, SlotFifo& f, int n, int np, int64_t img_row0, uint64_t pol) -> bool {
     for (int p0 = 0; p0 < np;) {
-      const int nb = claim_slots(sm.w_empty + rw * NWt, NWt, wc, np - p0, lane, abort_flag);
-      if (nb == 0) return false;
-      DCK_TC_TRACE(30 + nb);
-      if (lane < nb) {
-        const int sl = rw * NWt + (wc + lane) % NWt;
-        const uint32_t it = ta.item[n + p0 + lane];
-        const uint32_t bytes = (it >> 26) << 12;
-        mbar_expect_tx(&sm.w_full[sl], bytes);
-        bulk_load(sm.w[sl], img + (it & 0x03FFFFFFu), bytes, &sm.w_full[sl], pol);
+      const int nb = min(NWt, np - p0);
+      if (!f.claim(nb, NWt, sm.u_empty[rw], lane, abort_flag)) return false;
+      uint64_t* full = &sm.u_full[rw][f.inst % kFifoBars];
+      if (leader && lane == 0) {
+        uint32_t total = 0;
+        for (int q = 0; q < nb; ++q) total += (ta.item[n + p0 + q] >> 26) << 12;
+        mbar_expect_tx(full, total);
       }
       __syncwarp();
-      wc += nb;
+      if (lane < nb) {
+        const int sl = rw * NWt + (f.head + lane) % NWt;
+        const uint32_t it = ta.item[n + p0 + lane];
+        const uint32_t hrows = ((it >> 26) << 12) / 256;
+        const int64_t y = img_row0 + ((it & 0x03FFFFFFu) >> 7) + hr * hrows;
+        tma_load_2d_pair(sm.w[sl], &maps.im[im_map_of(hrows)], lead(full), 0, (int32_t)y, pol);
+      }
+      __syncwarp();
+      f.advance(nb);
       p0 += nb;
     }
     return true;
   };
+  const int64_t img_seq_rows = ta.fimg_seq_bytes >> 7;
 
   if (warp == 0) {
-    // ---- latent pieces, issued as soon as their slots are free; in
-    // query-folded mode also the factor items of MMA thread 1, in the order
-    // that thread consumes them (a group's pieces, then its units' items) ------
+    // ---- latent pieces (this CTA's 128 rows of each), issued as soon as their
+    // slots are free; in query-folded mode also the factor items of MMA thread
+    // 1, in the order that thread consumes them (a group's pieces, then its
+    // units' items) ---------------------------------------------------------
     if (has_work) {
       const uint64_t pol = policy_evict_first();
       const uint64_t pol_w = policy_evict_last();
-      int a_cnt = 0, wc = 0, kc = 0;
+      SlotFifo ga, fw;  // the latent ring; MMA thread 1's factor ring (query-folded mode)
+      int kc = 0;
       bool ok = true, images_ready = false;
       for (int ph = 0; ph < 2 && ok; ++ph)
-        for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
-          const uint8_t* img = ta.fimg + (kFold ? (int64_t)seg.b * ta.fimg_seq_bytes : 0);
+        for (PairWalker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
+          const int64_t img_row0 = kFold ? (int64_t)seg.b * img_seq_rows : 0;
           for (int i = 0; i < seg.ntiles && ok; ++i) {
-            const int64_t yrow = seg.row0 + seg.t_begin + (int64_t)kTile * i;
-            if (lane == 0 && i + 1 < seg.ntiles) {  // next tile's latent rows toward L2
-              const int64_t r0 = yrow + kTile, nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
+            const int64_t yrow = seg.row0 + seg.t0(i, hr);
+            if (lane == 0 && i + 1 < seg.ntiles) {  // the next pair tile's rows of this half toward L2
+              const int64_t r0 = yrow + kPTile, nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
               if (nr > 0)
                 prefetch_l2(static_cast<const __nv_bfloat16*>(a.kc) + r0 * lt.Rk, (uint32_t)(nr * lt.Rk * 2));
             }
             int ua, ub;
-            units_of(ph, seg.x0 + i, ua, ub);
+            units_of(ph, seg.X0 + i, ua, ub);
             for (int g = 0; g < lt.G && ok; ++g) {
               const GroupSm& gs = sm.grp[g];
               const int np = gs.np;
               const int lo = max(ua - gs.u0, 0), hi = min(ub - gs.u0, (int)gs.nu);
               if (lo >= hi) continue;  // none of the group's units in this piece of work
-              for (int p0 = 0; p0 < np && ok;) {
-                const int nb = claim_slots(sm.a_empty, kNA, a_cnt, np - p0, lane, abort_flag);
-                ok = nb > 0;
-                if (!ok) break;
-                if (lane < nb) {
-                  const int sl = (a_cnt + lane) % kNA;
-                  const int w = gs.w[p0 + lane];
-                  const CUtensorMap* m = w == 64 ? &maps.kc64 : (w == 32 ? &maps.kc32 : &maps.kc16);
-                  mbar_expect_tx(&sm.a_full[sl], kTile * w * 2);
-                  tma_load_2d_hint(sm.a[sl], m, &sm.a_full[sl], gs.roff + gs.k[p0 + lane], (int32_t)yrow, pol);
-                }
-                __syncwarp();
-                a_cnt += nb;
-                p0 += nb;
+              // the group's pieces: one instance of the latent ring
+              if (!(ok = ga.claim(np, kNA, sm.g_empty, lane, abort_flag))) break;
+              uint64_t* gfull = &sm.g_full[ga.inst % kFifoBars];
+              if (leader && lane == 0) mbar_expect_tx(gfull, 2 * kTile * 2 * gs.rank);
+              __syncwarp();
+              if (lane < np) {
+                const int sl = (ga.head + lane) % kNA;
+                const int w = gs.w[lane];
+                const CUtensorMap* m = w == 64 ? &maps.kc64 : (w == 32 ? &maps.kc32 : &maps.kc16);
+                tma_load_2d_pair(sm.a[sl], m, lead(gfull), gs.roff + gs.k[lane], (int32_t)yrow, pol);
               }
+              __syncwarp();
+              ga.advance(np);
               if (kMma == 2)
                 for (int u = lo; u < hi && ok; ++u, ++kc) {
                   if ((kc & 1) != 1) continue;  // MMA thread 0's unit
@@ -355,162 +390,129 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
                     griddep_wait();
                     images_ready = true;
                   }
-                  ok = put_unit_items(1, wc, gs.i0 + u * np, np, img, pol_w);
+                  ok = put_unit(1, fw, gs.i0 + u * np, np, img_row0, pol_w);
                 }
             }
           }
         }
+      if (!ok && lane == 0) stop_peer();
     }
   } else if (warp == 10) {
-    // ---- factor items: several bulk copies per instruction (query-folded
+    // ---- factor items: several TMA copies per instruction (query-folded
     // mode: the ring of MMA thread 0 only) --------------------------------------
     if (has_work) {
       const uint64_t pol = policy_evict_last();
       griddep_wait();  // the images are written by the preparation kernel
-      int w_cnt = 0;
+      SlotFifo fw;         // MMA thread 0's factor ring
       bool ok = true;
-      int wc = 0, kc = 0;  // items put into MMA thread 0's ring, units so far
+      int kc = 0;          // units so far
       for (int ph = 0; ph < 2 && ok; ++ph)
-        for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
-          const uint8_t* img = ta.fimg + (kFold ? (int64_t)seg.b * ta.fimg_seq_bytes : 0);
+        for (PairWalker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
+          const int64_t img_row0 = kFold ? (int64_t)seg.b * img_seq_rows : 0;
           for (int i = 0; i < seg.ntiles && ok; ++i) {
             int ua, ub;
-            units_of(ph, seg.x0 + i, ua, ub);
-            if (kMma == 1) {  // one ring: claims may span units (the units' items are contiguous)
-              const int n_end = sm.uitem[ub];
-              for (int n0 = sm.uitem[ua]; n0 < n_end && ok;) {
-                const int nb = claim_slots(sm.w_empty, NW, w_cnt, min(NW, n_end - n0), lane, abort_flag);
-                ok = nb > 0;
-                if (!ok) break;
-                if (lane < nb) {
-                  const int sl = (w_cnt + lane) % NW;
-                  const uint32_t it = ta.item[n0 + lane];
-                  const uint32_t bytes = (it >> 26) << 12;
-                  mbar_expect_tx(&sm.w_full[sl], bytes);
-                  bulk_load(sm.w[sl], img + (it & 0x03FFFFFFu), bytes, &sm.w_full[sl], pol);
-                }
-                __syncwarp();
-                w_cnt += nb;
-                n0 += nb;
-              }
-              continue;
-            }
+            units_of(ph, seg.X0 + i, ua, ub);
             for (int g = 0; g < lt.G && ok; ++g) {
               const GroupSm& gs = sm.grp[g];
               const int np = gs.np;
               const int lo = max(ua - gs.u0, 0), hi = min(ub - gs.u0, (int)gs.nu);
               for (int u = lo; u < hi && ok; ++u, ++kc)
-                if ((kc & 1) == 0) ok = put_unit_items(0, wc, gs.i0 + u * np, np, img, pol);
+                if (kMma == 1 || (kc & 1) == 0) ok = put_unit(0, fw, gs.i0 + u * np, np, img_row0, pol);
             }
           }
         }
+      if (!ok && lane == 0) stop_peer();
     }
   } else if (warp == 1 || (kMma == 2 && warp == 11)) {
-    // ---- MMA issuers: lane 0 of warp 1 (and of warp 11 in query-folded mode)
-    // runs the schedule of every kMma-th unit into its own accumulator, so one
-    // thread's barrier tests and commits overlap the other's MMAs.  Each thread
-    // owns a factor ring (single consumer) and observes every latent piece's
-    // fill in order, releasing the pieces of groups it has no unit in, so no
-    // parity test can see a stale phase. ---------------------------------------
-    if (lane == 0 && has_work) {
+    // ---- MMA issuers (even CTA only): lane 0 of warp 1 (and of warp 11 in
+    // query-folded mode) runs the schedule of every kMma-th unit into its own
+    // accumulator, so one thread's barrier waits and commits overlap the
+    // other's MMAs.  Each thread owns a factor ring (single consumer).  Per
+    // unit: one wait for its items, one for its accumulator, its MMAs, one
+    // commit for the items and one for the accumulator; per key group one
+    // wait for all its latent pieces and one release (commit, or arrivals in
+    // both CTAs when the thread has no unit in the group, after the fill so
+    // that no barrier phase is passed early). ---------------------------------
+    if (leader && lane == 0 && has_work) {
       const int t = warp == 1 ? 0 : 1;
-      uint64_t* wfull = sm.w_full + t * NWt;
-      uint64_t* wempty = sm.w_empty + t * NWt;
-      int a_cnt = 0, w_cnt = 0, kc = 0, own = 0;
+      int gi = 0, ghead = 0;  // latent-ring instances (groups) and slots handed out so far
+      int ui = 0, uhead = 0;  // this thread's factor-ring instances (item batches) and slots
+      int kc = 0, own = 0;    // units of the pair so far, units in this thread's accumulator
       bool ok = true;
       for (int ph = 0; ph < 2 && ok; ++ph)
-      for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
-        for (int i = 0; i < seg.ntiles && ok; ++i) {
-          int ua, ub;
-          units_of(ph, seg.x0 + i, ua, ub);
-          for (int g = 0; g < lt.G && ok; ++g) {
-            const GroupSm& gs = sm.grp[g];
-            const int np = gs.np;
-            const int lo = max(ua - gs.u0, 0), hi = min(ub - gs.u0, (int)gs.nu);  // the group's units here
-            if (lo >= hi) continue;
-            const int a_base = a_cnt;
-            const int uf = lo + (kMma == 2 ? (((kc & 1) == t) ? 0 : 1) : 0);  // this thread's first unit of the group
-            if (uf >= hi)  // none: observe the group's pieces, then release them
-              for (int p = 0; p < np && ok; ++p) {
-                const int sl = (a_base + p) % kNA;
-                if ((ok = mbar_wait(&sm.a_full[sl], ((a_base + p) / kNA) & 1, abort_flag))) mbar_arrive(&sm.a_empty[sl]);
+        for (PairWalker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
+          for (int i = 0; i < seg.ntiles && ok; ++i) {
+            int ua, ub;
+            units_of(ph, seg.X0 + i, ua, ub);
+            for (int g = 0; g < lt.G && ok; ++g) {
+              const GroupSm& gs = sm.grp[g];
+              const int np = gs.np;
+              const int lo = max(ua - gs.u0, 0), hi = min(ub - gs.u0, (int)gs.nu);  // the group's units here
+              if (lo >= hi) continue;
+              const int gb = gi % kFifoBars;
+              const uint32_t gpar = (gi / kFifoBars) & 1;
+              const int uf = lo + (kMma == 2 ? (((kc & 1) == t) ? 0 : 1) : 0);  // this thread's first unit of the group
+              // all the group's latent pieces (both CTAs' rows) are there
+              if (!(ok = mbar_wait(&sm.g_full[gb], gpar, abort_flag))) break;
+              if (uf >= hi) {  // no unit of this thread in the group: release its pieces in both CTAs
+                mbar_arrive(&sm.g_empty[gb]);
+                mbar_arrive_cluster(peer(&sm.g_empty[gb]));
               }
-            for (int u = uf; u < hi && ok; u += kMma) {
-              const int nh = min(2, gs.nh - 2 * u);
-              const uint32_t idesc_k = idesc_bf16(128, kD * nh, false, true);
-              const int kg = kc + (u - lo);                        // unit index of the CTA
-              const int buf = kMma == 2 ? t : (kg & 1);
-              const int use = kMma == 2 ? own : (kg >> 1);         // earlier units in this accumulator
-              // readiness of this unit's factor items (and, at this thread's first
-              // unit of the group, latent pieces): independent tests whose latencies
-              // overlap; blocking waits, in ring order, only for what is not there
-              // yet.  Only items within one turn of the ring are tested: the previous
-              // use of their slot has been consumed, so the parity test cannot see a
-              // stale phase.
-              uint32_t miss = 0;
-#pragma unroll
-              for (int p = 0; p < kMaxPieces; ++p)
-                if (p < np) {
-                  const int c = w_cnt + p;
-                  if (p >= NWt || !mbar_test(&wfull[c % NWt], (c / NWt) & 1)) miss |= 1u << p;
-                  if (u == uf && !mbar_test(&sm.a_full[(a_base + p) % kNA], ((a_base + p) / kNA) & 1))
-                    miss |= 0x100u << p;
+              for (int u = uf; u < hi && ok; u += kMma) {
+                const int nh = min(2, gs.nh - 2 * u);
+                const uint32_t idesc_k = idesc_bf16(256, kD * nh, false, true);
+                const int kg = kc + (u - lo);                        // unit index of the pair
+                const int buf = kMma == 2 ? t : (kg & 1);
+                const int use = kMma == 2 ? own : (kg >> 1);         // earlier units in this accumulator
+                const uint32_t dcol = tmem + buf * kKCols;
+                for (int p0 = 0; p0 < np && ok;) {  // the unit's item batches (ring instances)
+                  const int nb = min(NWt, np - p0);
+                  const int ub_ = ui % kFifoBars;
+                  if (!(ok = mbar_wait(&sm.u_full[t][ub_], (ui / kFifoBars) & 1, abort_flag))) break;
+                  if (p0 == 0 && use >= 1) {  // both CTAs' epilogues have read this accumulator's previous unit
+                    if (!(ok = mbar_wait(&sm.k_empty[buf], (use - 1) & 1, abort_flag))) break;
+                  }
+                  tc_fence_after();
+                  for (int q = 0; q < nb; ++q) {
+                    const int p = p0 + q;
+                    const int w = gs.w[p];
+                    const uint32_t ab0 = smem_u32(sm.a[(ghead + p) % kNA]);
+                    const uint32_t bb = smem_u32(sm.w[t * NWt + (uhead + q) % NWt]);
+                    const uint32_t swz = swz_of(w);
+                    for (int k = 0; k < w / 16; ++k) {
+                      const uint64_t ad = sdesc(ab0 + k * 32, 16, 16 * w, swz);
+                      const uint64_t bd = sdesc(bb + k * 2048, 128 * w, 1024, kSw128);
+                      umma_f16_pair(dcol, ad, bd, idesc_k, (p > 0 || k > 0) ? 1u : 0u);
+                    }
+                  }
+                  umma_commit_pair(&sm.u_empty[t][ub_]);  // the batch's slots, once its MMAs are done
+                  ++ui;
+                  uhead += nb;
+                  p0 += nb;
                 }
-              // the first piece and item before the accumulator: the operand streams do
-              // not depend on the epilogue, so the MMAs can start as soon as it is free
-              if ((miss & 0x100u) && !(ok = mbar_wait(&sm.a_full[a_base % kNA], (a_base / kNA) & 1, abort_flag))) break;
-              if ((miss & 1u) && !(ok = mbar_wait(&wfull[w_cnt % NWt], (w_cnt / NWt) & 1, abort_flag))) break;
-              miss &= ~0x101u;
-              DCK_TC_TRACE(12);
-              if (use >= 1) {  // the epilogue has read this accumulator's previous unit
-                if (!(ok = mbar_wait(&sm.k_empty[buf], (use - 1) & 1, abort_flag))) break;
-                tc_fence_after();
+                if (!ok) break;
+                umma_commit_pair(&sm.k_full[buf]);
+                if (u + kMma >= hi) umma_commit_pair(&sm.g_empty[gb]);  // this thread is done with the pieces
+                ++own;
               }
-              DCK_TC_TRACE(10);
-              const uint32_t dcol = tmem + buf * kKCols;
-              const bool last = u + kMma >= hi;  // this thread's last unit of the group
-              for (int p = 0; p < np; ++p) {
-                const int asl = (a_base + p) % kNA;
-                const int wsl = w_cnt % NWt;
-                if (((miss >> (8 + p)) & 1) && !(ok = mbar_wait(&sm.a_full[asl], ((a_base + p) / kNA) & 1, abort_flag)))
-                  break;
-                if (((miss >> p) & 1) && !(ok = mbar_wait(&wfull[wsl], (w_cnt / NWt) & 1, abort_flag))) break;
-                DCK_TC_TRACE(13);
-                const int w = gs.w[p];
-                const uint32_t ab0 = smem_u32(sm.a[asl]);
-                const uint32_t bb = smem_u32(sm.w[t * NWt + wsl]);
-                const uint32_t swz = swz_of(w);
-                for (int k = 0; k < w / 16; ++k) {
-                  const uint64_t ad = sdesc(ab0 + k * 32, 16, 16 * w, swz);
-                  const uint64_t bd = sdesc(bb + k * 2048, 128 * w, 1024, kSw128);
-                  umma_f16(dcol, ad, bd, idesc_k, (p > 0 || k > 0) ? 1u : 0u);
-                }
-                umma_commit(&wempty[wsl]);
-                if (last) umma_commit(&sm.a_empty[asl]);  // this thread is done with the piece
-                DCK_TC_TRACE(14);
-                ++w_cnt;
-              }
-              if (!ok) break;
-              umma_commit(&sm.k_full[buf]);
-              DCK_TC_TRACE(11);
-              ++own;
+              ++gi;
+              ghead += np;
+              kc += hi - lo;
             }
-            a_cnt += np;
-            kc += hi - lo;
           }
         }
-      }
+      if (!ok) stop_peer();
     }
     __syncwarp();
   } else if (warp >= 2 && warp <= 9) {
-    // ---- epilogue: RoPE, scores, softmax, P -------------------------------
+    // ---- epilogue: RoPE, scores, softmax, P of this CTA's 128-token halves ----
     const int e = tid - 64;              // 0 .. 255
     const int quad = warp & 3;           // TMEM lane quadrant
     const int hf = (warp - 2) >> 2;      // frequency half, then head half
-    const int tau = quad * 32 + lane;    // token row inside the tile
+    const int tau = quad * 32 + lane;    // token row inside the half tile
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     // tile and segment ends: thread e owns head jt and the 16 tokens [16 ct, 16 ct + 16)
-    // of every tile; the 8 owners of a head are adjacent lanes of one warp
+    // of every half tile; the 8 owners of a head are adjacent lanes of one warp
     const int jt = e >> 3, ct = e & 7;
     int kc = 0, round = 0;
     bool ok = true;
@@ -521,248 +523,247 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     ok = wwait(&sm.epi_bar, round & 1, abort_flag); \
     ++round;                                        \
   } while (0)
+    // an accumulator has been read by this warp: release it on the even CTA's barrier
+    auto release_acc = [&](int buf) {
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (leader) mbar_arrive(&sm.k_empty[buf]);
+        else mbar_arrive_cluster(lead(&sm.k_empty[buf]));
+      }
+    };
     for (int ph = 0; ph < 2 && ok; ++ph)
-    for (Walker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
-      if (!kFold) {
-        // rotated queries of this sequence at position L-1, scaled to log2 units
-        // (angle reduced mod 2 pi in fp64, sine and cosine in fp32)
-        const double P = (double)(seg.L - 1);
-        const float qscale = kLog2e * rsqrtf((float)kD);
-        const __nv_bfloat16* qb = static_cast<const __nv_bfloat16*>(a.q) + (int64_t)seg.b * Hq * kD;
-        for (int i = e; i < Hq * (kD / 2); i += kEpiThreads) {
-          const int j = i / (kD / 2), pi = i % (kD / 2);
-          const double ang = P * sm.om64[pi];
-          float sn, cs;
-          sincosf((float)(ang - 6.283185307179586 * rint(ang * 0.15915494309189535)), &sn, &cs);
-          const float x1v = __bfloat162float(qb[j * kD + pi]), x2v = __bfloat162float(qb[j * kD + pi + kD / 2]);
-          sm.qr[j * kD + pi] = __float2bfloat16_rn((x1v * cs - x2v * sn) * qscale);
-          sm.qr[j * kD + pi + kD / 2] = __float2bfloat16_rn((x1v * sn + x2v * cs) * qscale);
-        }
-      }
-      // RoPE angle of token t0+tau and pair p: (t0*w_p mod 2pi, fp64) + tau*w_p (fp32);
-      // the offsets beta of later tiles are written at the previous tile's end
-      if (e < kD / 2) {
-        const double ang = (double)seg.t_begin * sm.om64[e];
-        sm.beta[e] = (float)(ang - 6.283185307179586 * floor(ang * 0.15915494309189535));
-      }
-      EPI_SYNC();
-      if (!ok) break;
-      // head jt's reference max (log2 units; the same in all 8 owners) and this
-      // owner's share of its row sum, rescaled whenever the reference moves
-      float m_run = -INFINITY, l_part = 0.f;
-      int ua = 0, ub = 0;  // units of the current tile
-      for (int i = 0; i < seg.ntiles && ok; ++i) {
-        const int t0 = seg.t_begin + kTile * i;
-        const int64_t x = seg.x0 + i;  // flattened tile index
-        units_of(ph, (int)x, ua, ub);
-        float cs[32], sn[32];
-#pragma unroll
-        for (int ip = 0; ip < 32; ++ip) {
-          const int pi = 32 * hf + ip;
-          float ph = fmaf((float)tau, sm.om32[pi], sm.beta[pi]);
-          ph = fmaf(-kTwoPi, rintf(ph * kInvTwoPi), ph);
-          __sincosf(ph, &sn[ip], &cs[ip]);
-        }
-        // per unit (one or two KV heads), in MMA order: partial scores of this frequency half
-        for (int g = 0; g < lt.G && ok; ++g) {
-          const GroupSm& gs = sm.grp[g];
-          const int lo = max(ua - gs.u0, 0), hi = min(ub - gs.u0, (int)gs.nu);
-          for (int u = lo; u < hi; ++u) {
-            const int nh = min(2, gs.nh - 2 * u);
-            const int buf = kc & 1;
-            if (!(ok = wwait(&sm.k_full[buf], (kc >> 1) & 1, abort_flag))) break;
-            tc_fence_after();
-            DCK_TC_TRACE(20);
-            if (kFold) {
-              // Y columns [64 hf, 64 hf + 64) of both heads: pairs (2i, 2i+1) of my 32
-              // frequencies, in two passes of 16 pairs; each pass loads both heads
-              // before its one wait, so a unit costs two TMEM round trips
-              const uint32_t cb = tmem + lane_base + buf * kKCols + 64 * hf;
-              float pa[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};  // independent chains
-#pragma unroll
-              for (int ps = 0; ps < 2; ++ps) {
-                float y0[32], y1[32];
-                tmem_ld32(cb + 32 * ps, y0);
-                if (nh == 2) tmem_ld32(cb + kD + 32 * ps, y1);
-                tmem_wait_ld();
-                DCK_TC_TRACE(43 + ps);
-                if (ps == 1) {
-                  tc_fence_before();
-                  __syncwarp();
-                  if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
-                }
-#pragma unroll
-                for (int i2 = 0; i2 < 16; ++i2)
-                  pa[0][i2 & 3] = fmaf(cs[16 * ps + i2], y0[2 * i2], fmaf(sn[16 * ps + i2], y0[2 * i2 + 1], pa[0][i2 & 3]));
-                if (nh == 2)
-#pragma unroll
-                  for (int i2 = 0; i2 < 16; ++i2)
-                    pa[1][i2 & 3] =
-                        fmaf(cs[16 * ps + i2], y1[2 * i2], fmaf(sn[16 * ps + i2], y1[2 * i2 + 1], pa[1][i2 & 3]));
-              }
-              float* xh = sm.x + hf * (kMaxHqTc * 128);  // this frequency half's scores
-              xh[sm.order[gs.h0 + 2 * u] * 128 + tau] = (pa[0][0] + pa[0][1]) + (pa[0][2] + pa[0][3]);
-              if (nh == 2) xh[sm.order[gs.h0 + 2 * u + 1] * 128 + tau] = (pa[1][0] + pa[1][1]) + (pa[1][2] + pa[1][3]);
-            } else {
-              // per head: rotate the key's 32 frequency pairs of this half (two
-              // passes of 16), stage them as bf16, and form the scores of the
-              // head's qpg query heads with mma m16n8k16 (rows: the warp's 32
-              // tokens in two m-tiles; k: 16 rotated x-halves, then 16 y-halves
-              // per pass; n: query heads, padded to 8)
-              const int gid = lane >> 2, tig = lane & 3;
-              uint8_t* st = sm.kst[warp - 2];
-              const uint32_t st_addr = smem_u32(st);
-              for (int hh = 0; hh < nh; ++hh) {
-                const int j0 = sm.order[gs.h0 + 2 * u + hh] * qpg;
-                const uint32_t cb = tmem + lane_base + buf * kKCols + hh * kD;
-                const bool last = hh == nh - 1;
-                float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-#pragma unroll
-                for (int ps = 0; ps < 2; ++ps) {
-                  float k1v[16], k2v[16];
-                  tmem_ld16(cb + 32 * hf + 16 * ps, k1v);
-                  tmem_ld16(cb + 64 + 32 * hf + 16 * ps, k2v);
-                  tmem_wait_ld();
-                  if (last && ps == 1) {
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&sm.k_empty[buf]);
-                  }
-                  // this lane's token: rotated x-halves (chunks 0, 1) and y-halves (2, 3)
-                  uint32_t rw[16];
-#pragma unroll
-                  for (int w = 0; w < 8; ++w) {
-                    const int ip = 16 * ps + 2 * w;
-                    const float a0 = fmaf(k1v[2 * w], cs[ip], -k2v[2 * w] * sn[ip]);
-                    const float a1 = fmaf(k1v[2 * w + 1], cs[ip + 1], -k2v[2 * w + 1] * sn[ip + 1]);
-                    const float b0 = fmaf(k1v[2 * w], sn[ip], k2v[2 * w] * cs[ip]);
-                    const float b1 = fmaf(k1v[2 * w + 1], sn[ip + 1], k2v[2 * w + 1] * cs[ip + 1]);
-                    rw[w] = pack_bf16x2(a0, a1);
-                    rw[8 + w] = pack_bf16x2(b0, b1);
-                  }
-                  __syncwarp();  // the previous pass's fragments have been read
-#pragma unroll
-                  for (int c = 0; c < 4; ++c)
-                    *reinterpret_cast<uint4*>(st + lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4)) =
-                        make_uint4(rw[4 * c], rw[4 * c + 1], rw[4 * c + 2], rw[4 * c + 3]);
-                  __syncwarp();
-#pragma unroll
-                  for (int ks = 0; ks < 2; ++ks) {  // x-halves, then y-halves
-                    // B: query head n = gid (zero past qpg), k = 2 tig .. and 2 tig + 8 ..
-                    uint32_t bq0 = 0u, bq1 = 0u;
-                    if (gid < qpg) {
-                      const __nv_bfloat16* qrow = sm.qr + (j0 + gid) * kD + 64 * ks + 32 * hf + 16 * ps;
-                      bq0 = *reinterpret_cast<const uint32_t*>(qrow + 2 * tig);
-                      bq1 = *reinterpret_cast<const uint32_t*>(qrow + 2 * tig + 8);
-                    }
-#pragma unroll
-                    for (int mt = 0; mt < 2; ++mt) {
-                      // A: tokens 16 mt .. +15, k chunks 2 ks and 2 ks + 1 of the staged rows
-                      const int r = 16 * mt + (lane & 7) + 8 * ((lane >> 3) & 1), ch = 2 * ks + (lane >> 4);
-                      uint32_t af[4];
-                      ldmatrix_x4(af, st_addr + r * 64 + ((ch ^ ((r >> 1) & 3)) << 4));
-                      mma_bf16_16816(acc[mt], af, bq0, bq1);
-                    }
-                  }
-                }
-                // scores: token (16 mt + gid [+ 8]) of this quadrant, query heads 2 tig, 2 tig + 1
-                float* xh = sm.x + hf * (kMaxHqTc * 128);  // this frequency half's scores
-#pragma unroll
-                for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-                  for (int q = 0; q < 4; ++q) {
-                    const int jj = 2 * tig + (q & 1), t = quad * 32 + 16 * mt + gid + 8 * (q >> 1);
-                    if (jj < qpg) xh[(j0 + jj) * 128 + t] = acc[mt][q];
-                  }
-              }
-            }
-            DCK_TC_TRACE(21);
-            ++kc;
+      for (PairWalker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
+        if (!kFold) {
+          // rotated queries of this sequence at position L-1, scaled to log2 units
+          // (angle reduced mod 2 pi in fp64, sine and cosine in fp32)
+          const double Pq = (double)(seg.L - 1);
+          const float qscale = kLog2e * rsqrtf((float)kD);
+          const __nv_bfloat16* qb = static_cast<const __nv_bfloat16*>(a.q) + (int64_t)seg.b * Hq * kD;
+          for (int i = e; i < Hq * (kD / 2); i += kEpiThreads) {
+            const int j = i / (kD / 2), pi = i % (kD / 2);
+            const double ang = Pq * sm.om64[pi];
+            float sn, cs;
+            sincosf((float)(ang - 6.283185307179586 * rint(ang * 0.15915494309189535)), &sn, &cs);
+            const float x1v = __bfloat162float(qb[j * kD + pi]), x2v = __bfloat162float(qb[j * kD + pi + kD / 2]);
+            sm.qr[j * kD + pi] = __float2bfloat16_rn((x1v * cs - x2v * sn) * qscale);
+            sm.qr[j * kD + pi + kD / 2] = __float2bfloat16_rn((x1v * sn + x2v * cs) * qscale);
           }
         }
-        if (!ok) break;
-        // ---- tile end: reference max, P ------------------------------------
-        DCK_TC_TRACE(22);
-        EPI_SYNC();  // every partial score of the tile is in x
-        if (!ok) break;
-        {
-          const bool own = jt < Hq && sm.hunit[jt] >= ua && sm.hunit[jt] < ub;  // head computed here
-          const int tb = 16 * ct;  // first token of this owner
-          float sc[16];
-          const float4* xr = reinterpret_cast<const float4*>(&sm.x[jt * 128 + tb]);
-          const float4* xr2 = reinterpret_cast<const float4*>(&sm.x[kMaxHqTc * 128 + jt * 128 + tb]);
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            float4 v = own ? xr[q] : make_float4(0.f, 0.f, 0.f, 0.f);
-            if (own) {  // plus the other frequency half (every score is stored each tile)
-              const float4 w = xr2[q];
-              v = make_float4(v.x + w.x, v.y + w.y, v.z + w.z, v.w + w.w);
-            }
-            sc[4 * q] = v.x;
-            sc[4 * q + 1] = v.y;
-            sc[4 * q + 2] = v.z;
-            sc[4 * q + 3] = v.w;
-          }
-          const int nv = max(0, min(16, seg.t_end - (t0 + tb)));  // tokens inside the sequence
-          float mx = -INFINITY;
-#pragma unroll
-          for (int k = 0; k < 16; ++k) {
-            if (k >= nv || !own) sc[k] = -INFINITY;
-            mx = fmaxf(mx, sc[k]);
-          }
-          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
-          // the reference moves only when the tile's max exceeds it by the threshold
-          if (own && (m_run == -INFINITY || mx > m_run + kRescaleThr)) {
-            l_part *= exp2f(m_run - mx);
-            m_run = mx;
-          }
-          if (own && ct == 0) ta.mglob[x * Hq + jt] = m_run;
-          // probabilities (bf16, the absorption's operand) straight into this tile's
-          // P image; the row sum uses the rounded values
-          uint32_t pk[8];
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const __nv_bfloat162 pv = __floats2bfloat162_rn(own ? exp2f(sc[2 * k] - m_run) : 0.f,
-                                                            own ? exp2f(sc[2 * k + 1] - m_run) : 0.f);
-            const float2 pf = __bfloat1622float2(pv);
-            l_part += pf.x + pf.y;
-            pk[k] = *reinterpret_cast<const uint32_t*>(&pv);
-          }
-          if (own || (jt >= Hq && jt < hq_pad && ua == 0)) {  // padded heads get zero rows
-            // image: [token atom (64)][head row][64 tokens], 128B rows, 16-byte chunks swizzled by row % 8
-            uint8_t* img = ta.pglob + x * (hq_pad * 256) + (tb >> 6) * (hq_pad * 128) + (jt >> 3) * 1024 +
-                           (jt & 7) * 128;
-            const int ch = (tb & 63) >> 3;
-            *reinterpret_cast<uint4*>(img + ((ch ^ (jt & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            *reinterpret_cast<uint4*>(img + (((ch + 1) ^ (jt & 7)) << 4)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-          }
-        }
-        if (e < kD / 2 && i + 1 < seg.ntiles) {  // RoPE phase offsets of the next tile
-          const double ang = (double)(t0 + kTile) * sm.om64[e];
+        // RoPE angle of token t0+tau and pair p: (t0*w_p mod 2pi, fp64) + tau*w_p (fp32);
+        // the offsets beta of later tiles are written at the previous tile's end
+        if (e < kD / 2) {
+          const double ang = (double)seg.t0(0, hr) * sm.om64[e];
           sm.beta[e] = (float)(ang - 6.283185307179586 * floor(ang * 0.15915494309189535));
         }
-        DCK_TC_TRACE(23);
-        EPI_SYNC();  // x is clear and the next tile's phase offsets are in place
+        EPI_SYNC();
         if (!ok) break;
+        // head jt's reference max (log2 units; the same in all 8 owners) and this
+        // owner's share of its row sum, rescaled whenever the reference moves
+        float m_run = -INFINITY, l_part = 0.f;
+        int ua = 0, ub = 0;  // units of the current tile
+        for (int i = 0; i < seg.ntiles && ok; ++i) {
+          const int t0 = seg.t0(i, hr);
+          const bool has = seg.has(i, hr);    // this half holds tokens of the sequence
+          const int64_t x = seg.x128(i, hr);  // its flattened 128-token tile (when it has)
+          units_of(ph, seg.X0 + i, ua, ub);
+          float cs[32], sn[32];
+#pragma unroll
+          for (int ip = 0; ip < 32; ++ip) {
+            const int pi = 32 * hf + ip;
+            float phs = fmaf((float)tau, sm.om32[pi], sm.beta[pi]);
+            phs = fmaf(-kTwoPi, rintf(phs * kInvTwoPi), phs);
+            __sincosf(phs, &sn[ip], &cs[ip]);
+          }
+          // per unit (one or two KV heads), in MMA order: partial scores of this frequency half
+          for (int g = 0; g < lt.G && ok; ++g) {
+            const GroupSm& gs = sm.grp[g];
+            const int lo = max(ua - gs.u0, 0), hi = min(ub - gs.u0, (int)gs.nu);
+            for (int u = lo; u < hi; ++u) {
+              const int nh = min(2, gs.nh - 2 * u);
+              const int buf = kc & 1;
+              if (!(ok = wwait(&sm.k_full[buf], (kc >> 1) & 1, abort_flag))) break;
+              tc_fence_after();
+              if (kFold) {
+                // Y columns [64 hf, 64 hf + 64) of both heads: pairs (2i, 2i+1) of my 32
+                // frequencies, in two passes of 16 pairs; each pass loads both heads
+                // before its one wait, so a unit costs two TMEM round trips
+                const uint32_t cb = tmem + lane_base + buf * kKCols + 64 * hf;
+                float pa[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};  // independent chains
+#pragma unroll
+                for (int ps = 0; ps < 2; ++ps) {
+                  float y0[32], y1[32];
+                  tmem_ld32(cb + 32 * ps, y0);
+                  if (nh == 2) tmem_ld32(cb + kD + 32 * ps, y1);
+                  tmem_wait_ld();
+                  if (ps == 1) release_acc(buf);
+#pragma unroll
+                  for (int i2 = 0; i2 < 16; ++i2)
+                    pa[0][i2 & 3] =
+                        fmaf(cs[16 * ps + i2], y0[2 * i2], fmaf(sn[16 * ps + i2], y0[2 * i2 + 1], pa[0][i2 & 3]));
+                  if (nh == 2)
+#pragma unroll
+                    for (int i2 = 0; i2 < 16; ++i2)
+                      pa[1][i2 & 3] =
+                          fmaf(cs[16 * ps + i2], y1[2 * i2], fmaf(sn[16 * ps + i2], y1[2 * i2 + 1], pa[1][i2 & 3]));
+                }
+                float* xh = sm.x + hf * (kMaxHqTc * 128);  // this frequency half's scores
+                xh[sm.order[gs.h0 + 2 * u] * 128 + tau] = (pa[0][0] + pa[0][1]) + (pa[0][2] + pa[0][3]);
+                if (nh == 2)
+                  xh[sm.order[gs.h0 + 2 * u + 1] * 128 + tau] = (pa[1][0] + pa[1][1]) + (pa[1][2] + pa[1][3]);
+              } else {
+                // per head: rotate the key's 32 frequency pairs of this half (two
+                // passes of 16), stage them as bf16, and form the scores of the
+                // head's qpg query heads with mma m16n8k16 (rows: the warp's 32
+                // tokens in two m-tiles; k: 16 rotated x-halves, then 16 y-halves
+                // per pass; n: query heads, padded to 8)
+                const int gid = lane >> 2, tig = lane & 3;
+                uint8_t* st = sm.kst[warp - 2];
+                const uint32_t st_addr = smem_u32(st);
+                for (int hh = 0; hh < nh; ++hh) {
+                  const int j0 = sm.order[gs.h0 + 2 * u + hh] * qpg;
+                  const uint32_t cb = tmem + lane_base + buf * kKCols + hh * kD;
+                  const bool last = hh == nh - 1;
+                  float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+#pragma unroll
+                  for (int ps = 0; ps < 2; ++ps) {
+                    float k1v[16], k2v[16];
+                    tmem_ld16(cb + 32 * hf + 16 * ps, k1v);
+                    tmem_ld16(cb + 64 + 32 * hf + 16 * ps, k2v);
+                    tmem_wait_ld();
+                    if (last && ps == 1) release_acc(buf);
+                    // this lane's token: rotated x-halves (chunks 0, 1) and y-halves (2, 3)
+                    uint32_t rw[16];
+#pragma unroll
+                    for (int w = 0; w < 8; ++w) {
+                      const int ip = 16 * ps + 2 * w;
+                      const float a0 = fmaf(k1v[2 * w], cs[ip], -k2v[2 * w] * sn[ip]);
+                      const float a1 = fmaf(k1v[2 * w + 1], cs[ip + 1], -k2v[2 * w + 1] * sn[ip + 1]);
+                      const float b0 = fmaf(k1v[2 * w], sn[ip], k2v[2 * w] * cs[ip]);
+                      const float b1 = fmaf(k1v[2 * w + 1], sn[ip + 1], k2v[2 * w + 1] * cs[ip + 1]);
+                      rw[w] = pack_bf16x2(a0, a1);
+                      rw[8 + w] = pack_bf16x2(b0, b1);
+                    }
+                    __syncwarp();  // the previous pass's fragments have been read
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+                      *reinterpret_cast<uint4*>(st + lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4)) =
+                          make_uint4(rw[4 * c], rw[4 * c + 1], rw[4 * c + 2], rw[4 * c + 3]);
+                    __syncwarp();
+#pragma unroll
+                    for (int ks = 0; ks < 2; ++ks) {  // x-halves, then y-halves
+                      // B: query head n = gid (zero past qpg), k = 2 tig .. and 2 tig + 8 ..
+                      uint32_t bq0 = 0u, bq1 = 0u;
+                      if (gid < qpg) {
+                        const __nv_bfloat16* qrow = sm.qr + (j0 + gid) * kD + 64 * ks + 32 * hf + 16 * ps;
+                        bq0 = *reinterpret_cast<const uint32_t*>(qrow + 2 * tig);
+                        bq1 = *reinterpret_cast<const uint32_t*>(qrow + 2 * tig + 8);
+                      }
+#pragma unroll
+                      for (int mt = 0; mt < 2; ++mt) {
+                        // A: tokens 16 mt .. +15, k chunks 2 ks and 2 ks + 1 of the staged rows
+                        const int r = 16 * mt + (lane & 7) + 8 * ((lane >> 3) & 1), ch = 2 * ks + (lane >> 4);
+                        uint32_t af[4];
+                        ldmatrix_x4(af, st_addr + r * 64 + ((ch ^ ((r >> 1) & 3)) << 4));
+                        mma_bf16_16816(acc[mt], af, bq0, bq1);
+                      }
+                    }
+                  }
+                  // scores: token (16 mt + gid [+ 8]) of this quadrant, query heads 2 tig, 2 tig + 1
+                  float* xh = sm.x + hf * (kMaxHqTc * 128);  // this frequency half's scores
+#pragma unroll
+                  for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                      const int jj = 2 * tig + (q & 1), tt = quad * 32 + 16 * mt + gid + 8 * (q >> 1);
+                      if (jj < qpg) xh[(j0 + jj) * 128 + tt] = acc[mt][q];
+                    }
+                }
+              }
+              ++kc;
+            }
+          }
+          if (!ok) break;
+          // ---- tile end: reference max, P ------------------------------------
+          EPI_SYNC();  // every partial score of the tile is in x
+          if (!ok) break;
+          {
+            const bool own = jt < Hq && sm.hunit[jt] >= ua && sm.hunit[jt] < ub;  // head computed here
+            const int tb = 16 * ct;  // first token of this owner
+            float sc[16];
+            const float4* xr = reinterpret_cast<const float4*>(&sm.x[jt * 128 + tb]);
+            const float4* xr2 = reinterpret_cast<const float4*>(&sm.x[kMaxHqTc * 128 + jt * 128 + tb]);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              float4 v = own ? xr[q] : make_float4(0.f, 0.f, 0.f, 0.f);
+              if (own) {  // plus the other frequency half (every score is stored each tile)
+                const float4 w = xr2[q];
+                v = make_float4(v.x + w.x, v.y + w.y, v.z + w.z, v.w + w.w);
+              }
+              sc[4 * q] = v.x;
+              sc[4 * q + 1] = v.y;
+              sc[4 * q + 2] = v.z;
+              sc[4 * q + 3] = v.w;
+            }
+            const int nv = max(0, min(16, seg.L - (t0 + tb)));  // tokens inside the sequence
+            float mx = -INFINITY;
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+              if (k >= nv || !own) sc[k] = -INFINITY;
+              mx = fmaxf(mx, sc[k]);
+            }
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+            // the reference moves only when the tile's max exceeds it by the threshold
+            if (own && (m_run == -INFINITY || mx > m_run + kRescaleThr)) {
+              l_part *= exp2f(m_run - mx);
+              m_run = mx;
+            }
+            if (has && own && ct == 0) ta.mglob[x * Hq + jt] = m_run;
+            // probabilities (bf16, the absorption's operand) straight into this tile's
+            // P image; the row sum uses the rounded values
+            uint32_t pk[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const __nv_bfloat162 pv = __floats2bfloat162_rn(own ? exp2f(sc[2 * k] - m_run) : 0.f,
+                                                              own ? exp2f(sc[2 * k + 1] - m_run) : 0.f);
+              const float2 pf = __bfloat1622float2(pv);
+              l_part += pf.x + pf.y;
+              pk[k] = *reinterpret_cast<const uint32_t*>(&pv);
+            }
+            if (has && (own || (jt >= Hq && jt < hq_pad && ua == 0))) {  // padded heads get zero rows
+              // image: [token atom (64)][head row][64 tokens], 128B rows, 16-byte chunks swizzled by row % 8
+              uint8_t* img = ta.pglob + x * (hq_pad * 256) + (tb >> 6) * (hq_pad * 128) + (jt >> 3) * 1024 +
+                             (jt & 7) * 128;
+              const int ch = (tb & 63) >> 3;
+              *reinterpret_cast<uint4*>(img + ((ch ^ (jt & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+              *reinterpret_cast<uint4*>(img + (((ch + 1) ^ (jt & 7)) << 4)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+            }
+          }
+          if (e < kD / 2 && i + 1 < seg.ntiles) {  // RoPE phase offsets of the next pair tile
+            const double ang = (double)(t0 + kPTile) * sm.om64[e];
+            sm.beta[e] = (float)(ang - 6.283185307179586 * floor(ang * 0.15915494309189535));
+          }
+          EPI_SYNC();  // x is clear and the next tile's phase offsets are in place
+          if (!ok) break;
+        }
+        if (!ok) break;
+        // ---- segment end: reference max and row sum -> this half's partial slot ----
+        l_part += __shfl_xor_sync(0xffffffffu, l_part, 1);
+        l_part += __shfl_xor_sync(0xffffffffu, l_part, 2);
+        l_part += __shfl_xor_sync(0xffffffffu, l_part, 4);
+        if (jt < Hq && ct == 0 && sm.hunit[jt] >= ua && sm.hunit[jt] < ub) {
+          const int64_t slot = ph ? pair_xslot(P, a.B, seg.X0 - sp.NPm, hr) : pair_slot(pair, seg.b, hr);
+          a.part_ml[(slot * Hq + jt) * 2] = m_run;
+          a.part_ml[(slot * Hq + jt) * 2 + 1] = l_part;
+        }
       }
-      if (!ok) break;
-      // ---- segment end: reference max and row sum -> partial slot c + b -------
-      l_part += __shfl_xor_sync(0xffffffffu, l_part, 1);
-      l_part += __shfl_xor_sync(0xffffffffu, l_part, 2);
-      l_part += __shfl_xor_sync(0xffffffffu, l_part, 4);
-      if (jt < Hq && ct == 0 && sm.hunit[jt] >= ua && sm.hunit[jt] < ub) {
-        const int64_t slot = ph ? xbase + (seg.x0 - sp.NTm) : (int64_t)blockIdx.x + seg.b;
-        a.part_ml[(slot * Hq + jt) * 2] = m_run;
-        a.part_ml[(slot * Hq + jt) * 2 + 1] = l_part;
-      }
-    }
 #undef EPI_SYNC
+    if (!ok && lane == 0) stop_peer();
   }
   tc_fence_before();
   __syncthreads();
-  DCK_TC_TRACE_FLUSH();
   if (sm.abort_flag) {
     // let copies and MMAs already in flight land before the memory is released
     const long long c0 = clock64();
@@ -770,10 +771,10 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     }
     if (tid == 0) atomicOr(a.err, kErrTimeout);
   }
-  __syncthreads();
+  cluster_sync();  // the peer no longer reads this CTA's operands or arrives on its barriers
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
+    tmem_dealloc_pair(tmem, kTmemCols);
   }
 }
 
@@ -890,7 +891,11 @@ struct MapsKey {
   const void* kc;
   int64_t n_rows;
   int Rk;
-  bool operator==(const MapsKey& o) const { return kc == o.kc && n_rows == o.n_rows && Rk == o.Rk; }
+  const void* img;
+  int64_t img_rows;
+  bool operator==(const MapsKey& o) const {
+    return kc == o.kc && n_rows == o.n_rows && Rk == o.Rk && img == o.img && img_rows == o.img_rows;
+  }
 };
 constexpr int kMapsCache = 64;
 std::mutex g_maps_mu;
@@ -898,45 +903,92 @@ MapsKey g_maps_key[kMapsCache];
 Maps g_maps_val[kMapsCache];
 int g_maps_n = 0, g_maps_next = 0;
 
-bool build_maps(const LayerTable& lt, const DecodeArgs& a, Maps& maps) {
+bool build_maps(const LayerTable& lt, const DecodeArgs& a, const void* img, int64_t img_rows, Maps& maps) {
   std::memset(&maps, 0, sizeof(maps));
   const uint64_t rows = (uint64_t)std::max<int64_t>(1, a.n_rows);
-  return make_tmap_2d_bf16(&maps.kc64, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 64, kTile, CU_TENSOR_MAP_SWIZZLE_128B) &&
-         make_tmap_2d_bf16(&maps.kc32, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 32, kTile, CU_TENSOR_MAP_SWIZZLE_64B) &&
-         make_tmap_2d_bf16(&maps.kc16, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 16, kTile, CU_TENSOR_MAP_SWIZZLE_32B);
+  if (!(make_tmap_2d_bf16(&maps.kc64, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 64, kTile, CU_TENSOR_MAP_SWIZZLE_128B) &&
+        make_tmap_2d_bf16(&maps.kc32, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 32, kTile, CU_TENSOR_MAP_SWIZZLE_64B) &&
+        make_tmap_2d_bf16(&maps.kc16, a.kc, lt.Rk, rows, (uint64_t)lt.Rk * 2, 16, kTile, CU_TENSOR_MAP_SWIZZLE_32B)))
+    return false;
+  // the factor images as rows of 128 bytes (64 bf16), boxes of 16 .. 128 rows
+  const uint32_t box_rows[4] = {16, 32, 64, 128};
+  for (int i = 0; i < 4; ++i)
+    if (!make_tmap_2d_bf16(&maps.im[i], img, 64, (uint64_t)std::max<int64_t>(img_rows, 128), 128, 64, box_rows[i],
+                           CU_TENSOR_MAP_SWIZZLE_NONE))
+      return false;
+  return true;
 }
 
 static_assert(sizeof(Smem<true>) + 1024 <= 232448, "shared memory of the query-folded kernel");
 static_assert(sizeof(Smem<false>) + 1024 <= 232448, "shared memory of the key-mode kernel");
 
 template <bool kFold>
-cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& maps, const TcArgs& ta,
-                        const PrepArgs& pa, cudaStream_t s) {
-  const size_t smem = sizeof(Smem<kFold>) + 1024;
+cudaError_t set_smem_attr() {
   static int attr_done[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
   const bool dev_ok = dev >= 0 && dev < 64;
-  if (!dev_ok || !attr_done[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kFold>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    if (e != cudaSuccess) return e;
-    if (dev_ok) attr_done[dev] = 1;
-  }
-  factor_prep_kernel<kFold><<<dim3(pa.n_items, kFold ? a.B : 1), 256, 0, s>>>(lt, a, pa,
-                                                                                static_cast<uint8_t*>(a.extra));
-  cudaError_t e = hook_launched(a.hook, s);
-  if (e != cudaSuccess) return e;
+  if (dev_ok && attr_done[dev]) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kFold>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)(sizeof(Smem<kFold>) + 1024));
+  if (e == cudaSuccess && dev_ok) attr_done[dev] = 1;
+  return e;
+}
+
+// CTA pairs that can be resident at once (at most half the SMs): the scores
+// kernel is persistent, so its grid is exactly that many pairs.
+template <bool kFold>
+int pairs_of_device() {
+  static int pairs[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (pairs[dev]) return pairs[dev];
+  int sms = 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  if (set_smem_attr<kFold>() != cudaSuccess) return 0;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.n_items);
+  cfg.gridDim = dim3(2 * (sms / 2));
   cfg.blockDim = dim3(Ring<kFold>::kThreads);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
+  cfg.dynamicSmemBytes = sizeof(Smem<kFold>) + 1024;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, decode_tc_kernel<kFold>, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    return 0;
+  }
+  pairs[dev] = std::min(n, sms / 2);
+  return pairs[dev];
+}
+
+template <bool kFold>
+cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& maps, const TcArgs& ta,
+                        const PrepArgs& pa, cudaStream_t s) {
+  cudaError_t e = set_smem_attr<kFold>();
+  if (e != cudaSuccess) return e;
+  factor_prep_kernel<kFold><<<dim3(pa.n_items, kFold ? a.B : 1), 256, 0, s>>>(lt, a, pa,
+                                                                                static_cast<uint8_t*>(a.extra));
+  e = hook_launched(a.hook, s);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * ta.n_pairs);
+  cfg.blockDim = dim3(Ring<kFold>::kThreads);
+  cfg.dynamicSmemBytes = sizeof(Smem<kFold>) + 1024;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 2;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
   e = cudaLaunchKernelEx(&cfg, decode_tc_kernel<kFold>, maps, lt, a, ta);
   return e != cudaSuccess ? e : hook_launched(a.hook, s);
 }
@@ -951,9 +1003,10 @@ bool build_tables(const LayerTable& lt, TcArgs& ta, PrepArgs& pa) {
   for (int g = 0; g < lt.G; ++g) {
     GroupSm& gs = ta.grp[g];
     gs.roff = lt.grp_roff[g];
+    gs.rank = (int16_t)lt.grp_rank[g];
     int16_t kk[kMaxPieces];
     gs.np = (int8_t)make_pieces(lt.grp_rank[g], gs.w, kk);
-    if (gs.np > kMaxPieces || gs.np > kNA) return false;
+    if (gs.np > kMaxPieces || gs.np > std::min(Ring<true>::NA, Ring<false>::NA)) return false;
     for (int p = 0; p < gs.np; ++p) gs.k[p] = kk[p];
     gs.h0 = (int8_t)pos;
     gs.nh = (int8_t)lt.grp_nh[g];
@@ -1040,9 +1093,12 @@ size_t tc_decode_extra_ws(const LayerTable& lt, int batch, int64_t n_rows) {
   return extra_layout(lt, batch, n_rows).total;
 }
 
+// CTA pairs of the tensor-core path on the current device (0 if it cannot run).
+int tc_decode_pairs(const LayerTable& lt) { return lt.qpg == 1 ? pairs_of_device<true>() : pairs_of_device<false>(); }
+
 cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) {
   const bool fold = lt.qpg == 1;
-  if (!a.extra) return cudaErrorInvalidValue;
+  if (!a.extra || a.n_items < 2 || (a.n_items & 1)) return cudaErrorInvalidValue;
   static thread_local TcArgs ta;
   static thread_local PrepArgs pa;
   if (!build_tables(lt, ta, pa)) return cudaErrorInvalidValue;
@@ -1050,11 +1106,12 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStre
   std::memcpy(pa.om, ta.om, sizeof(ta.om));
   const ExtraLayout xl = extra_layout(lt, a.B, a.n_rows);
   uint8_t* base = static_cast<uint8_t*>(a.extra);
-  ta.fimg = base;
+  ta.n_pairs = a.n_items / 2;
   ta.pglob = base + xl.img;
   ta.mglob = reinterpret_cast<float*>(base + xl.img + xl.p);
   ta.max_tiles = max_tiles(a.n_rows, a.B);
-  const MapsKey key{a.kc, a.n_rows, lt.Rk};
+  const int64_t img_rows = (int64_t)(xl.img >> 7);
+  const MapsKey key{a.kc, a.n_rows, lt.Rk, base, img_rows};
   Maps maps;
   bool have = false;
   {
@@ -1066,7 +1123,7 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStre
       }
   }
   if (!have) {
-    if (!build_maps(lt, a, maps)) return cudaErrorInvalidValue;
+    if (!build_maps(lt, a, base, img_rows, maps)) return cudaErrorInvalidValue;
     std::lock_guard<std::mutex> lk(g_maps_mu);
     g_maps_key[g_maps_next] = key;
     g_maps_val[g_maps_next] = maps;

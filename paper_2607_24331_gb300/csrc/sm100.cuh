@@ -235,9 +235,13 @@ __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
-// Arrive (release at cluster scope) on an mbarrier given by its shared::cluster address.
+// Arrive on an mbarrier given by its shared::cluster address (possibly in the
+// peer CTA), with the default release at CTA scope: the arrivals here order
+// tcgen05 work (with tcgen05.fence::before_thread_sync) and TMA slot reuse, not
+// generic-proxy data; a release at cluster scope would first wait for this
+// thread's earlier global stores (about 1.4k cycles per arrival measured).
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
 // Store of a 32-bit word to a shared::cluster address (a flag in the peer CTA).

@@ -45,14 +45,16 @@ def sm_count():
 
 def leftover_sequences(lens, sms):
     """Sequences with tiles in the finely split leftover range of the tensor-core
-    path: with NT 128-token tiles and fewer than 8 per SM, tiles from
-    floor(NT / sms) * sms on are shared out by groups of heads."""
-    nts = [(int(L) + 127) // 128 for L in lens]
-    NT = sum(nts)
-    NTm = NT // sms * sms if NT // sms < 8 else NT
+    path: sequences are cut into 256-token pair tiles, split over the CTA pairs
+    (sms // 2 of them on a GPU whose TPCs all hold two SMs); with fewer than 8
+    pair tiles per pair, those from floor(NP / P) * P on are shared out by
+    groups of heads."""
+    nts = [(int(L) + 255) // 256 for L in lens]
+    NP, P = sum(nts), sms // 2
+    NPm = NP // P * P if NP // P < 8 else NP
     out, pre = [], 0
     for b, n in enumerate(nts):
-        if n and pre + n > NTm:
+        if n and pre + n > NPm:
             out.append(b)
         pre += n
     return out

@@ -66,7 +66,11 @@ def test_needles_at_a_tile_boundary_and_in_a_leftover_tile(cfg):
     left = leftover_sequences(lens, sms)
     assert 1 in left
     k_left = nt - 64 - 2                          # second-last tile of sequence 1: a leftover tile
-    needles = [(0, 20 * 128, 3), (0, 20 * 128 - 1, spec.n_q_heads - 1), (1, k_left * 128 + 61, 9)]
+    # a pair-tile boundary (2560: the first token of pair tile 10, 2559: the last of
+    # pair tile 9), the boundary between the two halves of pair tile 10 (2688),
+    # and a token inside a leftover tile
+    needles = [(0, 20 * 128, 3), (0, 20 * 128 - 1, spec.n_q_heads - 1), (0, 21 * 128, 17),
+               (1, k_left * 128 + 61, 9)]
     for b, t, j in needles:
         plant_needle(di, b, t, j)
     got, _ = gpu_decode(spec, lens, di=di)

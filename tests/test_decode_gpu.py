@@ -141,20 +141,23 @@ def test_tensor_core_layer_shapes(name):
 
 
 @pytest.mark.parametrize("cfg", [1, 2])
-@pytest.mark.parametrize("extra", [5, -1])
+@pytest.mark.parametrize("extra", [5, -1, 1])
 def test_leftover_tiles_split_finely(cfg, extra):
-    """More 128-token tiles than SMs: whole tiles per SM, then the leftover tiles
-    shared out by groups of heads (scores) and r_v chunks (absorption), each with
-    its own partial slot.  extra = -1: one tile short of two per SM."""
-    sms = torch.cuda.get_device_properties(0).multi_processor_count
-    nt = sms + (extra if extra > 0 else sms - 1)
-    lens = (64 * 128, (nt - 64 - 1) * 128 + 77)
+    """More 256-token pair tiles than CTA pairs: whole pair tiles per pair, then the
+    leftover pair tiles shared out by groups of heads (scores) and their 128-token
+    halves by r_v chunks (absorption), each half with its own partial slot.
+    extra = -1: one pair tile short of two per pair; extra = 1 with an odd last
+    128-token tile: the leftover pair tile's second half is empty."""
+    P = torch.cuda.get_device_properties(0).multi_processor_count // 2
+    npt = P + (extra if extra > 0 else P - 1)
+    tail = 77 if extra != 1 else 256 + 100
+    lens = (32 * 256, (npt - 32 - 2) * 256 + tail)
     spec = S.workload(cfg).layer
     di = S.make_decode_inputs(spec, lens, seed=21 + cfg)
     got, _ = gpu_decode(spec, lens, di=di)
     for b, j in _sample_pairs(2, spec.n_q_heads, 8, cfg + 40):
         ref = oracle_decode(di, heads=[j], batch_ids=[b])
-        assert_parity(got[b:b + 1, j:j + 1], ref[b:b + 1, j:j + 1], "bf16", f"cfg{cfg} nt{nt} b{b} j{j}")
+        assert_parity(got[b:b + 1, j:j + 1], ref[b:b + 1, j:j + 1], "bf16", f"cfg{cfg} npt{npt} b{b} j{j}")
     assert np.isfinite(got).all()
 
 
