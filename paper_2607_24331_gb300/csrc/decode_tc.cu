@@ -100,6 +100,7 @@ constexpr int kMaxItems = 256;
 constexpr int kMaxUnits = 32;
 constexpr int kEpiThreads = 256;
 constexpr int kEpiWarps = kEpiThreads / 32;
+constexpr int kPrefetchAhead = 2;   // latent tiles prefetched toward L2 ahead of their loads
 constexpr float kRescaleThr = 8.f;  // log2 units: probabilities stay <= 256
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kKCols = 256;    // TMEM columns of one key accumulator
@@ -353,16 +354,31 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
       SlotFifo ga, fw;  // the latent ring; MMA thread 1's factor ring (query-folded mode)
       int kc = 0;
       bool ok = true, images_ready = false;
+      // L2 prefetch of this half's latent rows, kPrefetchAhead tiles ahead of the
+      // loads (across segment boundaries): the TMA loads then find them in L2
+      PairWalker pwalk[2] = {walk_m, walk_x};
+      PSegment pseg;
+      int pph = 0, pti = 0;
+      bool pvalid = false;
+      auto prefetch_next = [&]() {
+        if (lane != 0) return;
+        while (!pvalid || pti >= pseg.ntiles) {
+          while (pph < 2 && !pwalk[pph].next(a, pseg)) ++pph;
+          if (pph >= 2) return;
+          pvalid = true;
+          pti = 0;
+        }
+        const int64_t r0 = pseg.row0 + pseg.t0(pti++, hr);
+        const int64_t nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
+        if (nr > 0) prefetch_l2(static_cast<const __nv_bfloat16*>(a.kc) + r0 * lt.Rk, (uint32_t)(nr * lt.Rk * 2));
+      };
+      for (int q = 0; q < kPrefetchAhead; ++q) prefetch_next();
       for (int ph = 0; ph < 2 && ok; ++ph)
         for (PairWalker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
           const int64_t img_row0 = kFold ? (int64_t)seg.b * img_seq_rows : 0;
           for (int i = 0; i < seg.ntiles && ok; ++i) {
             const int64_t yrow = seg.row0 + seg.t0(i, hr);
-            if (lane == 0 && i + 1 < seg.ntiles) {  // the next pair tile's rows of this half toward L2
-              const int64_t r0 = yrow + kPTile, nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
-              if (nr > 0)
-                prefetch_l2(static_cast<const __nv_bfloat16*>(a.kc) + r0 * lt.Rk, (uint32_t)(nr * lt.Rk * 2));
-            }
+            prefetch_next();
             int ua, ub;
             units_of(ph, seg.X0 + i, ua, ub);
             for (int g = 0; g < lt.G && ok; ++g) {
@@ -993,15 +1009,37 @@ cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& m
   return e != cudaSuccess ? e : hook_launched(a.hook, s);
 }
 
-// Units, items and per-group tables of a layer.  Returns false when the layer
-// does not fit the tables.
+// Order in which a tile's key groups are processed: the latent ring holds the
+// pieces of the group in use while it fills with the next group's, so groups
+// with many pieces are interleaved with groups with few (largest first, then
+// smallest, ...), which keeps the piece counts of neighbours (cyclically: the
+// last group is followed by the next tile's first) within the ring.
+void group_order(const LayerTable& lt, int* order) {
+  int idx[kMaxGroupsTc];
+  int8_t w[kMaxPieces];
+  int16_t k[kMaxPieces];
+  int np[kMaxGroupsTc];
+  for (int g = 0; g < lt.G; ++g) {
+    idx[g] = g;
+    np[g] = make_pieces(lt.grp_rank[g], w, k);
+  }
+  std::stable_sort(idx, idx + lt.G, [&](int x, int y) { return np[x] > np[y]; });
+  for (int i = 0, lo = 0, hi = lt.G - 1; lo <= hi; ++i) order[i] = (i & 1) ? idx[hi--] : idx[lo++];
+}
+
+// Units, items and per-group tables of a layer (groups in processing order).
+// Returns false when the layer does not fit the tables.
 bool build_tables(const LayerTable& lt, TcArgs& ta, PrepArgs& pa) {
   std::memset(&ta, 0, sizeof(ta));
   std::memset(&pa, 0, sizeof(pa));
   ta.hq_pad = hq_pad_of(lt.Hq);
+  if (lt.G > kMaxGroupsTc) return false;
+  int gorder[kMaxGroupsTc];
+  group_order(lt, gorder);
   int pos = 0, item = 0, off = 0, unit = 0;
-  for (int g = 0; g < lt.G; ++g) {
-    GroupSm& gs = ta.grp[g];
+  for (int gi = 0; gi < lt.G; ++gi) {
+    const int g = gorder[gi];
+    GroupSm& gs = ta.grp[gi];
     gs.roff = lt.grp_roff[g];
     gs.rank = (int16_t)lt.grp_rank[g];
     int16_t kk[kMaxPieces];
