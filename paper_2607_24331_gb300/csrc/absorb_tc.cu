@@ -72,7 +72,7 @@ struct ASmem {
   uint8_t v[2 * kNVr][kVSlot];  // ring of MMA thread t: slots [t kNVr, (t + 1) kNVr)
   uint8_t p[kNP][kPSlot];
   uint64_t v_full[2 * kNVr], v_empty[2 * kNVr], p_full[kNP], p_empty[kNP];
-  uint64_t drain, tile_ok, u_ready, u_free;
+  uint64_t drain, tile_ok, u_ready[2], u_free[2];
   int pneed[kNP];  // P slot's tile raises some head's reference max (set by the producer before the slot fills)
   int s256[kAThreads], s128[kAThreads];
   uint32_t tmem_base;
@@ -165,8 +165,10 @@ __global__ void __launch_bounds__(kAThreads, 1)
     }
     mbar_init(&sm.drain, 2);
     mbar_init(&sm.tile_ok, 4);
-    mbar_init(&sm.u_ready, 2);
-    mbar_init(&sm.u_free, 4);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.u_ready[i], 2);
+      mbar_init(&sm.u_free[i], 4);
+    }
     sm.abort_flag = 0;
     fence_mbar_init();
   }
@@ -203,6 +205,10 @@ __global__ void __launch_bounds__(kAThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
+  // U is double-buffered in TMEM where two copies fit: segment s accumulates in
+  // buffer s % nub while the epilogue reads out segment s - 1
+  const uint32_t ucols = (uint32_t)(n_chunks * hq_pad);
+  const int nub = 2 * ucols <= kTmemCols ? 2 : 1;
   ASeg seg;
   DCK_AB_TRACE(0);
 
@@ -219,19 +225,30 @@ __global__ void __launch_bounds__(kAThreads, 1)
       // reference maxima (lane = head) of the previous tile and, loaded a tile
       // ahead so that their latency hides behind the value loads, of this one
       float m_prev = 0.f, m_pf = 0.f;
+      // L2 prefetch of the value rows two tiles ahead of their loads, across
+      // segments (the first two at once)
+      AWalk pwalk = walk0;
+      ASeg pseg;
+      int pti = 0;
+      bool pvalid = false;
+      auto prefetch_next = [&]() {
+        if (lane != 0) return;
+        while (!pvalid || pti >= pseg.n) {
+          if (!pwalk.next(a, pl, pseg)) return;
+          pvalid = true;
+          pti = 0;
+        }
+        const int64_t r0 = pseg.row(pti++), nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
+        if (nr > 0) prefetch_l2(static_cast<const __nv_bfloat16*>(a.vc) + r0 * lt.rv, (uint32_t)(nr * lt.rv * 2));
+      };
+      prefetch_next();
+      prefetch_next();
       for (AWalk walk = walk0; ok && walk.next(a, pl, seg);) {
         for (int i = 0; i < seg.n && ok; ++i) {
           const int64_t x = seg.x(i);
           const int64_t yrow = seg.row(i);
           const int ca = seg.ca, cb = seg.cb;
-          if (lane == 0) {  // this CTA's first tile, then each next tile, toward L2
-            for (int q = first ? 0 : 1; q < 2; ++q) {
-              if (q == 1 && i + 1 >= seg.n) break;
-              const int64_t r0 = seg.row(i + q), nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
-              if (nr > 0)
-                prefetch_l2(static_cast<const __nv_bfloat16*>(a.vc) + r0 * lt.rv, (uint32_t)(nr * lt.rv * 2));
-            }
-          }
+          prefetch_next();
           // chunks go to the two MMA threads' rings alternately (thread 0: [ca, cm),
           // thread 1: [cm, cb)), each chunk one slot filled by two boxes (lanes 0, 1)
           const int cm = chunk_mid(ca, cb), nch = cb - ca;
@@ -325,8 +342,8 @@ __global__ void __launch_bounds__(kAThreads, 1)
               DCK_AB_TRACE(10);
               ++rc;
             }
-          } else if (sgc > 0) {  // the epilogue has read the previous segment's U
-            if (!(ok = mbar_wait(&sm.u_free, (sgc - 1) & 1, abort_flag))) break;
+          } else if (sgc >= nub) {  // the epilogue has read out this buffer's previous segment
+            if (!(ok = mbar_wait(&sm.u_free[sgc % nub], (sgc / nub - 1) & 1, abort_flag))) break;
             tc_fence_after();
           }
           DCK_AB_TRACE(11);
@@ -365,7 +382,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
             for (int k = 0; k < 8; ++k) {
               const uint64_t bd = sdesc(pbase + (k >> 2) * (hq_pad * 128) + (k & 3) * 32, 16, 1024, kSw128);
               for (int q = 0; q < nc; ++q)
-                umma_f16(tmem + (c + q) * hq_pad, sdesc(vb[q] + k * 2048, kVSlot / 2, 1024, kSw128), bd, idesc_v,
+                umma_f16(tmem + (sgc % nub) * ucols + (c + q) * hq_pad, sdesc(vb[q] + k * 2048, kVSlot / 2, 1024, kSw128), bd, idesc_v,
                          (i == 0 && k == 0) ? 0u : 1u);
             }
             for (int q = 0; q < nc; ++q) umma_commit(&sm.v_empty[sl[q]]);
@@ -376,7 +393,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
           ++p_cnt;
         }
         if (!ok) break;
-        umma_commit(&sm.u_ready);
+        umma_commit(&sm.u_ready[sgc % nub]);
         DCK_AB_TRACE(13);
         ++sgc;
       }
@@ -402,7 +419,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
           for (int c = 0; c < n_chunks; ++c)
             for (int cb = 0; cb < hq_pad / 16; ++cb) {
               float v[16];
-              const uint32_t tad = tmem + lane_base + c * hq_pad + 16 * cb;
+              const uint32_t tad = tmem + (sgc % nub) * ucols + lane_base + c * hq_pad + 16 * cb;
               tmem_ld16(tad, v);
               tmem_wait_ld();
 #pragma unroll
@@ -419,15 +436,16 @@ __global__ void __launch_bounds__(kAThreads, 1)
       }
       if (!ok) break;
       // segment end: U -> the segment's partial slot
-      if (!(ok = wwait(&sm.u_ready, sgc & 1, abort_flag))) break;
+      if (!(ok = wwait(&sm.u_ready[sgc % nub], (sgc / nub) & 1, abort_flag))) break;
       tc_fence_after();
       DCK_AB_TRACE(22);
       float* dst = a.part_u + seg.slot * Hq * lt.rv + tau;
       const int ca = seg.ca, cb = seg.cb;
       for (int c = ca; c < cb; ++c) {
         float v0[16], v1[16];
-        tmem_ld16(tmem + lane_base + c * hq_pad, v0);
-        if (hq_pad > 16) tmem_ld16(tmem + lane_base + c * hq_pad + 16, v1);
+        const uint32_t ub = tmem + (sgc % nub) * ucols + lane_base + c * hq_pad;
+        tmem_ld16(ub, v0);
+        if (hq_pad > 16) tmem_ld16(ub + 16, v1);
         tmem_wait_ld();
 #pragma unroll
         for (int i2 = 0; i2 < 16; ++i2) {
@@ -437,7 +455,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.u_free);
+      if (lane == 0) mbar_arrive(&sm.u_free[sgc % nub]);
       ++sgc;
     }
   }

@@ -16,11 +16,13 @@
 // (8 where r_v allows, else 4); a chunk holds as many (sequence, query head)
 // rows as fit kMaxRows, so each head's B_v block is staged about once.
 // CTA `rank` of a cluster owns rows [rank*rv/split, (rank+1)*rv/split) of u
-// and of B_v's column block: it merges those rows of every (sequence, query
-// head) row of its chunk in one pass with a running max (twelve partials' loads in
-// flight at a time), stages its B_v rows in shared memory with cp.async (all
-// issued up front), and forms the partial product over its rows, each output
-// owned by one thread.  The cluster adds the partial outputs through
+// and of B_v's column block.  It stages its B_v rows in shared memory with
+// cp.async (all issued up front), lists each (sequence, query head) row's live
+// partial slots with their maxima and sums in shared memory, forms every row's
+// merged maximum M, weights 2^(m_c - M) and 1/l, then sums its rows of u with
+// those weights (the loads of a row are independent, so they are all in
+// flight together), and forms the partial product over its rows of B_v, each
+// output owned by one thread.  The cluster adds the partial outputs through
 // distributed shared memory, every rank reducing and writing a share of o.
 #include <algorithm>
 #include <type_traits>
@@ -38,7 +40,6 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kMaxSplit = 8;    // CTAs per cluster (r_v split), portable cluster size
 constexpr int kMaxRows = 16;    // (sequence, query head) rows per cluster
-constexpr int kItemBatch = 12;  // partials whose loads are in flight together
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)),
@@ -91,15 +92,20 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   const int r0 = rank * rr;
 
   // shared layout: B_v rows [rr][ldb] T | u rows [kMaxRows][rr + 4] | received partial o [split][kMaxRows * D / split]
-  // | 1/l | row slot ranges [kMaxRows][4] | scan | prefix | item starts [n_items + 1]
+  // | 1/l | per row: partial weights [kMaxRows][cap] f32, sums [kMaxRows][cap] f32, slots [kMaxRows][cap] i32,
+  // partial counts [kMaxRows] | row slot ranges [kMaxRows][4] | prefix [B + 1] | item starts [n_items + 1]
+  const int cap = 2 * a.n_items;  // partials a row can have, on either work plan
   T* sbv = reinterpret_cast<T*>(smem_c);
   float* su = reinterpret_cast<float*>(smem_c + (size_t)rr * ldb<T, D>() * sizeof(T));
   const int ldu = rr + 4;  // padded u rows: the tensor-core fragments read 8 rows at one column
   float* so = su + (size_t)kMaxRows * ldu;
   float* sinv = so + kMaxRows * D;
-  int* rc = reinterpret_cast<int*>(sinv + kMaxRows);
-  int* scan = rc + 4 * kMaxRows;
-  int* prefix = scan + kThreads;
+  float* pw = sinv + kMaxRows;
+  float* pl = pw + (size_t)kMaxRows * cap;
+  int* ps = reinterpret_cast<int*>(pl + (size_t)kMaxRows * cap);
+  int* pn = ps + (size_t)kMaxRows * cap;
+  int* rc = pn + kMaxRows;
+  int* prefix = rc + 4 * kMaxRows;
   int* ibeg = prefix + B + 1;
 
   // stage this CTA's B_v rows (all copies in flight at once)
@@ -118,8 +124,28 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   // tiles: pair tiles (tensor-core path) or 128-token tiles; items: CTA pairs or CTAs
   const bool pairs = a.split_extra != 0;
   const int n_it = pairs ? a.n_items / 2 : a.n_items;
-  const int NT = build_tile_prefix(a.seq_len, a.seq_start, B, a.n_rows, prefix, scan, a.err, false,
-                                   pairs ? 2 * kTile : kTile);
+  // tiles per sequence (every thread a share), then an exclusive prefix by warp 0
+  const int tile = pairs ? 2 * kTile : kTile;
+  for (int b = threadIdx.x; b < B; b += kThreads)
+    prefix[b + 1] = (valid_len(a.seq_len, a.seq_start, b, a.n_rows) + tile - 1) / tile;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    int run = 0;
+    for (int b0s = 0; b0s < B; b0s += 32) {
+      int v = b0s + lane < B ? prefix[b0s + lane + 1] : 0;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += y;
+      }
+      if (b0s + lane < B) prefix[b0s + lane + 1] = run + v;
+      run += __shfl_sync(0xffffffffu, v, 31);
+    }
+    if (lane == 0) prefix[0] = 0;
+  }
+  __syncthreads();
+  const int NT = prefix[B];
   // Partials of sequence b: the items whose main tiles (the first NTm, split
   // evenly in whole tiles) cover b's; on the tensor-core path also the extra
   // pair tiles of b (x >= NTm), two slots (halves) per item and per extra tile.
@@ -142,77 +168,110 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   // preceding grid is.
   asm volatile("griddepcontrol.wait;" ::: "memory");
 
-  // u rows restricted to [r0, r0 + rr), merged over the items in one pass with
-  // a running reference max: each thread owns float4 columns of whole rows and
-  // keeps kItemBatch items' loads in flight.  Every thread of a row sees the
-  // same maxima in the same order, so they agree on M; the thread of column 0
-  // also merges l.
+  // (1) every row's partials: slot, reference max m (log2 units) and sum l of
+  // each live one; (2) per row M = max m, weights 2^(m - M), 1/l; (3) this
+  // CTA's rows of u as the weighted sum, all of a row's loads independent.
+  for (int idx = threadIdx.x; idx < nrow * cap; idx += kThreads) {
+    const int i = idx / cap, q = idx % cap;
+    const int b = b0 + i / qpg, j = h * qpg + i % qpg;
+    const int c0 = rc[4 * i], nm = rc[4 * i + 1], e0 = rc[4 * i + 2];
+    const int nps = pairs ? 2 : 1;  // slots per item or extra tile
+    const int ns = nps * (nm + rc[4 * i + 3]);
+    if (q >= ns) continue;
+    const int k = q / nps, hh = q % nps;
+    bool live;
+    int64_t slot;
+    if (k < nm) {  // item c0 + k
+      const int c = c0 + k;
+      live = ibeg[c] != ibeg[c + 1];
+      if (pairs) {
+        const int n128 = (valid_len(a.seq_len, a.seq_start, b, a.n_rows) + kTile - 1) / kTile;
+        const int i0 = max(ibeg[c], prefix[b]) - prefix[b];  // b's first pair tile in the item
+        live = live && 2 * i0 + hh < n128;
+        slot = tc::pair_slot(c, b, hh);
+      } else {
+        slot = (int64_t)c + b;
+      }
+    } else {  // extra pair tile e (tensor-core path only)
+      const int n128 = (valid_len(a.seq_len, a.seq_start, b, a.n_rows) + kTile - 1) / kTile;
+      const int e = e0 + k - nm;
+      live = 2 * (NTm + e - prefix[b]) + hh < n128;
+      slot = tc::pair_xslot(n_it, B, e, hh);
+    }
+    float m = -INFINITY, l = 0.f;
+    if (live) {
+      const float2 ml = reinterpret_cast<const float2*>(a.part_ml)[slot * Hq + j];
+      m = ml.x;
+      l = ml.y;
+    }
+    pw[(size_t)i * cap + q] = m;
+    pl[(size_t)i * cap + q] = l;
+    ps[(size_t)i * cap + q] = live ? (int)slot : -1;
+  }
+  if (threadIdx.x < nrow) {
+    const int i = threadIdx.x;
+    pn[i] = (pairs ? 2 : 1) * (rc[4 * i + 1] + rc[4 * i + 3]);
+  }
+  __syncthreads();
+  {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int i = warp; i < nrow; i += kThreads / 32) {  // one warp per row
+      const int n = pn[i];
+      float M = -INFINITY;
+      for (int q = lane; q < n; q += 32) M = fmaxf(M, pw[(size_t)i * cap + q]);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+      float l = 0.f;
+      for (int q = lane; q < n; q += 32) {
+        const float wq = M == -INFINITY ? 0.f : exp2f(pw[(size_t)i * cap + q] - M);  // 0 for slots not live
+        pw[(size_t)i * cap + q] = wq;
+        l = fmaf(wq, pl[(size_t)i * cap + q], l);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+      if (lane == 0) sinv[i] = l > 0.f ? 1.f / l : 0.f;
+    }
+  }
+  __syncthreads();
   const int rr4 = rr / 4;
   for (int idx = threadIdx.x; idx < nrow * rr4; idx += kThreads) {
     const int i = idx / rr4, r4 = idx % rr4;
-    const int b = b0 + i / qpg, j = h * qpg + i % qpg;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    float M = -INFINITY, l = 0.f;
-    const int c0 = rc[4 * i], nm = rc[4 * i + 1], e0 = rc[4 * i + 2];
-    const int nps = pairs ? 2 : 1;                         // slots per item or extra tile
-    const int ns = nps * (nm + rc[4 * i + 3]);
-    const int n128 = (valid_len(a.seq_len, a.seq_start, b, a.n_rows) + kTile - 1) / kTile;
-    if (ns > 0) {
-      for (int vv = 0; vv < ns; vv += kItemBatch) {
-        float m[kItemBatch], lv[kItemBatch];
-        float4 v[kItemBatch];
+    const int j = h * qpg + i % qpg;
+    const int n = pn[i];
+    const float* wrow = pw + (size_t)i * cap;
+    const int* srow = ps + (size_t)i * cap;
+    float4 acc0 = make_float4(0.f, 0.f, 0.f, 0.f), acc1 = acc0;
+    int q = 0;
+    for (; q + 8 <= n; q += 8) {
+      float4 v[8];
 #pragma unroll
-        for (int u = 0; u < kItemBatch; ++u) {
-          const int q = vv + u;  // q-th partial of the row: main items, then extra tiles; halves innermost
-          const int k = q / nps, hh = q % nps;
-          bool live = q < ns;
-          int64_t slot = 0;
-          if (live && k < nm) {  // item c0 + k
-            const int c = c0 + k;
-            live = ibeg[c] != ibeg[c + 1];
-            if (pairs) {
-              const int i0 = max(ibeg[c], prefix[b]) - prefix[b];  // b's first pair tile in the item
-              live = live && 2 * i0 + hh < n128;
-              slot = tc::pair_slot(c, b, hh);
-            } else {
-              slot = (int64_t)c + b;
-            }
-          } else if (live) {  // extra pair tile e (tensor-core path only)
-            const int e = e0 + k - nm;
-            live = 2 * (NTm + e - prefix[b]) + hh < n128;
-            slot = tc::pair_xslot(n_it, B, e, hh);
-          }
-          const int64_t sl = (live ? slot : 0) * Hq + j;
-          const float2 ml = reinterpret_cast<const float2*>(a.part_ml)[sl];
-          const float4 uv = reinterpret_cast<const float4*>(a.part_u + sl * rv + r0)[r4];
-          m[u] = live ? ml.x : -INFINITY;
-          lv[u] = live ? ml.y : 0.f;
-          v[u] = live ? uv : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-        float Mb = M;
+      for (int u = 0; u < 8; ++u) {
+        const int sl = srow[q + u];
+        v[u] = sl >= 0 ? reinterpret_cast<const float4*>(a.part_u + ((int64_t)sl * Hq + j) * rv + r0)[r4]
+                       : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
 #pragma unroll
-        for (int u = 0; u < kItemBatch; ++u) Mb = fmaxf(Mb, m[u]);
-        if (Mb == -INFINITY) continue;  // nothing live yet
-        const float sc = exp2f(M - Mb);
-        acc.x *= sc;
-        acc.y *= sc;
-        acc.z *= sc;
-        acc.w *= sc;
-        l *= sc;
-#pragma unroll
-        for (int u = 0; u < kItemBatch; ++u) {
-          const float w = exp2f(m[u] - Mb);  // 0 for items that are not live
-          acc.x = fmaf(w, v[u].x, acc.x);
-          acc.y = fmaf(w, v[u].y, acc.y);
-          acc.z = fmaf(w, v[u].z, acc.z);
-          acc.w = fmaf(w, v[u].w, acc.w);
-          l = fmaf(w, lv[u], l);
-        }
-        M = Mb;
+      for (int u = 0; u < 8; ++u) {
+        float4& ac = (u & 1) ? acc1 : acc0;
+        const float wq = wrow[q + u];
+        ac.x = fmaf(wq, v[u].x, ac.x);
+        ac.y = fmaf(wq, v[u].y, ac.y);
+        ac.z = fmaf(wq, v[u].z, ac.z);
+        ac.w = fmaf(wq, v[u].w, ac.w);
       }
     }
-    reinterpret_cast<float4*>(su + (size_t)i * ldu)[r4] = acc;
-    if (r4 == 0) sinv[i] = l > 0.f ? 1.f / l : 0.f;
+    for (; q < n; ++q) {
+      const int sl = srow[q];
+      if (sl < 0) continue;
+      const float4 v = reinterpret_cast<const float4*>(a.part_u + ((int64_t)sl * Hq + j) * rv + r0)[r4];
+      const float wq = wrow[q];
+      acc0.x = fmaf(wq, v.x, acc0.x);
+      acc0.y = fmaf(wq, v.y, acc0.y);
+      acc0.z = fmaf(wq, v.z, acc0.z);
+      acc0.w = fmaf(wq, v.w, acc0.w);
+    }
+    reinterpret_cast<float4*>(su + (size_t)i * ldu)[r4] =
+        make_float4(acc0.x + acc1.x, acc0.y + acc1.y, acc0.z + acc1.z, acc0.w + acc1.w);
   }
   cp_async_wait_all();
   __syncthreads();
@@ -313,9 +372,10 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   // as many sequences per cluster as its rows allow: each head's B_v block is staged once per chunk
   const int bchunk = std::max(1, std::min(a.B, kMaxRows / lt.qpg));
   const int rr = lt.rv / split;
+  const int cap = 2 * a.n_items;
   const size_t smem = (size_t)rr * ldb<T, D>() * sizeof(T) +
-                      sizeof(float) * ((size_t)kMaxRows * (rr + 4) + kMaxRows * D + kMaxRows) +
-                      sizeof(int) * (4 * kMaxRows + kThreads + a.B + 1 + a.n_items + 1);
+                      sizeof(float) * ((size_t)kMaxRows * (rr + 4) + kMaxRows * D + kMaxRows + 2 * (size_t)kMaxRows * cap) +
+                      sizeof(int) * ((size_t)kMaxRows * cap + kMaxRows + 4 * kMaxRows + a.B + 1 + a.n_items + 1);
   auto k = combine_kernel<T, D>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;

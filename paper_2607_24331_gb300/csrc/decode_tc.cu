@@ -815,67 +815,77 @@ struct PrepArgs {
 // One block writes one factor item: [nh heads][2 halves][ws rank rows]
 // [64 columns] bf16, 128B-swizzled (16-byte chunk c of row r stored at chunk
 // c ^ (r % 8); every half starts on a 1024-byte swizzle atom).
-// Key mode: columns of B_g[:, slot].  Query-folded mode (one block row per
-// sequence b): columns 2i and 2i+1 are
+// Key mode: columns of B_g[:, slot].  Query-folded mode (the block's row of
+// the grid covers kPrepSeqs sequences b): columns 2i and 2i+1 are
 //   a_i B[:, i] + b_i B[:, i+64]  and  b_i B[:, i] - a_i B[:, i+64]
-// with (a, b) the halves of RoPE(q_{b,h}, L_b - 1) * log2(e)/sqrt(d).
+// with (a, b) the halves of RoPE(q_{b,h}, L_b - 1) * log2(e)/sqrt(d); each
+// thread loads its B_g values once and writes them folded for every sequence.
+constexpr int kPrepSeqs = 4;
 template <bool kFold>
 __global__ void __launch_bounds__(256) factor_prep_kernel(const LayerTable lt, const DecodeArgs a, const PrepArgs pa,
                                                           uint8_t* __restrict__ img) {
   griddep_launch();
-  const int n = blockIdx.x, b = blockIdx.y;
+  const int n = blockIdx.x, bs0 = blockIdx.y * kPrepSeqs;
+  const int nbs = kFold ? min(kPrepSeqs, a.B - bs0) : 1;
   const PrepItem it = pa.item[n];
   const int g = it.g, ws = it.ws, nh = it.nh;
-  __shared__ float qa[2][kD / 2], qb[2][kD / 2];
+  __shared__ float qa[kPrepSeqs][2][kD / 2], qb[kPrepSeqs][2][kD / 2];
+  __shared__ int live[kPrepSeqs];
   if (kFold) {
-    const int L = valid_len(a.seq_len, a.seq_start, b, a.n_rows);
-    if (L == 0) return;  // no tile of this sequence is ever processed
-    if (threadIdx.x < nh * (kD / 2)) {
-      const int hh = threadIdx.x / (kD / 2), i = threadIdx.x % (kD / 2);
+    for (int e = threadIdx.x; e < nbs * nh * (kD / 2); e += blockDim.x) {
+      const int sb = e / (nh * (kD / 2)), hh = (e / (kD / 2)) % nh, i = e % (kD / 2);
+      const int b = bs0 + sb;
+      const int L = valid_len(a.seq_len, a.seq_start, b, a.n_rows);
+      if (hh == 0 && i == 0) live[sb] = L > 0;  // no tile of an empty sequence is ever processed
       const int kv = it.kv[hh];
       // angle (L-1) w_i reduced mod 2 pi in fp64, sine and cosine in fp32
-      const double ang = (double)(L - 1) * pa.om[i];
+      const double ang = (double)max(L - 1, 0) * pa.om[i];
       float sn, cs;
       sincosf((float)(ang - 6.283185307179586 * rint(ang * 0.15915494309189535)), &sn, &cs);
       const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(a.q) + ((int64_t)b * lt.Hq + kv) * kD;
       const float x1 = __bfloat162float(q[i]), x2 = __bfloat162float(q[i + kD / 2]);
       const float sc = kLog2e * rsqrtf((float)kD);
-      qa[hh][i] = (x1 * cs - x2 * sn) * sc;
-      qb[hh][i] = (x1 * sn + x2 * cs) * sc;
+      qa[sb][hh][i] = (x1 * cs - x2 * sn) * sc;
+      qb[sb][hh][i] = (x1 * sn + x2 * cs) * sc;
     }
     __syncthreads();
   }
   const int64_t ld = (int64_t)lt.grp_nh[g] * kD;
-  uint8_t* dst = img + (kFold ? (int64_t)b * pa.seq_bytes : 0) + it.off;
   // thread -> (head, row, 8-column chunk): nh x ws rows x 16 chunks (2 halves x 8)
   for (int idx = threadIdx.x; idx < nh * ws * 16; idx += blockDim.x) {
     const int hh = idx / (ws * 16), r = (idx >> 4) % ws, ch = idx & 15;
     const int half = ch >> 3, c8 = ch & 7;
     const __nv_bfloat16* __restrict__ Bs =
-        static_cast<const __nv_bfloat16*>(a.Bk) + lt.grp_boff[g] + (it.s0 + hh) * kD;
-    const int k = it.k0 + r;
-    float v[8];
+        static_cast<const __nv_bfloat16*>(a.Bk) + lt.grp_boff[g] + (it.s0 + hh) * kD + (int64_t)(it.k0 + r) * ld;
+    const int64_t doff = it.off + (hh * 2 + half) * (ws * 128) + r * 128 + ((c8 ^ (r & 7)) << 4);
     if (kFold) {
-      // output columns col = 64*half + 8*c8 + t, t even/odd -> pair i = col/2
+      // output columns col = 64*half + 8*c8 + t, t even/odd -> pair i = col/2 = 32*half + 4*c8 + t/2:
+      // the x-halves B[:, i] and y-halves B[:, i+64] of four pairs, one 8-byte load each
+      const int i0 = 32 * half + 4 * c8;
+      const uint2 xr = *reinterpret_cast<const uint2*>(Bs + i0);
+      const uint2 yr = *reinterpret_cast<const uint2*>(Bs + kD / 2 + i0);
+      const __nv_bfloat16* xh = reinterpret_cast<const __nv_bfloat16*>(&xr);
+      const __nv_bfloat16* yh = reinterpret_cast<const __nv_bfloat16*>(&yr);
+      float x[4], y[4];
 #pragma unroll
-      for (int t = 0; t < 8; t += 2) {
-        const int i = (64 * half + 8 * c8 + t) >> 1;
-        const float x = __bfloat162float(Bs[k * ld + i]);
-        const float y = __bfloat162float(Bs[k * ld + kD / 2 + i]);
-        v[t] = fmaf(qa[hh][i], x, qb[hh][i] * y);
-        v[t + 1] = fmaf(qb[hh][i], x, -qa[hh][i] * y);
+      for (int t = 0; t < 4; ++t) {
+        x[t] = __bfloat162float(xh[t]);
+        y[t] = __bfloat162float(yh[t]);
+      }
+      for (int sb = 0; sb < nbs; ++sb) {
+        if (!live[sb]) continue;
+        uint4 out;
+        __nv_bfloat162* o2 = reinterpret_cast<__nv_bfloat162*>(&out);
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const float qa_ = qa[sb][hh][i0 + t], qb_ = qb[sb][hh][i0 + t];
+          o2[t] = __floats2bfloat162_rn(fmaf(qa_, x[t], qb_ * y[t]), fmaf(qb_, x[t], -qa_ * y[t]));
+        }
+        *reinterpret_cast<uint4*>(img + (int64_t)(bs0 + sb) * pa.seq_bytes + doff) = out;
       }
     } else {
-      const uint4 raw = *reinterpret_cast<const uint4*>(Bs + k * ld + 64 * half + 8 * c8);
-      const __nv_bfloat16* h8 = reinterpret_cast<const __nv_bfloat16*>(&raw);
-#pragma unroll
-      for (int t = 0; t < 8; ++t) v[t] = __bfloat162float(h8[t]);
+      *reinterpret_cast<uint4*>(img + doff) = *reinterpret_cast<const uint4*>(Bs + 64 * half + 8 * c8);
     }
-    uint4 out;
-    __nv_bfloat162* o2 = reinterpret_cast<__nv_bfloat162*>(&out);
-#pragma unroll
-    for (int t = 0; t < 4; ++t) o2[t] = __floats2bfloat162_rn(v[2 * t], v[2 * t + 1]);
-    *reinterpret_cast<uint4*>(dst + (hh * 2 + half) * (ws * 128) + r * 128 + ((c8 ^ (r & 7)) << 4)) = out;
   }
 }
 
@@ -987,8 +997,8 @@ cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& m
                         const PrepArgs& pa, cudaStream_t s) {
   cudaError_t e = set_smem_attr<kFold>();
   if (e != cudaSuccess) return e;
-  factor_prep_kernel<kFold><<<dim3(pa.n_items, kFold ? a.B : 1), 256, 0, s>>>(lt, a, pa,
-                                                                                static_cast<uint8_t*>(a.extra));
+  factor_prep_kernel<kFold><<<dim3(pa.n_items, kFold ? (a.B + kPrepSeqs - 1) / kPrepSeqs : 1), 256, 0, s>>>(
+      lt, a, pa, static_cast<uint8_t*>(a.extra));
   e = hook_launched(a.hook, s);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
