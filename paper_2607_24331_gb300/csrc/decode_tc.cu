@@ -116,7 +116,6 @@ struct Ring {
   // mode; key mode's units carry up to four items, which one thread's ring of
   // all slots streams better
   static constexpr int kMma = kFold ? 2 : 1;
-  static constexpr int NWt = NW / kMma;       // slots of one MMA thread's ring
   static constexpr int kThreads = kFold ? 384 : 352;
 };
 
@@ -180,7 +179,7 @@ struct Smem {
   // latent ring: one full/empty pair per group instance; factor rings: one
   // pair per unit (batch of items) of each MMA thread (see SlotFifo)
   uint64_t g_full[kFifoBars], g_empty[kFifoBars];
-  uint64_t u_full[Ring<kFold>::kMma][kFifoBars], u_empty[Ring<kFold>::kMma][kFifoBars];
+  uint64_t u_full[kFifoBars], u_empty[kFifoBars];
   uint64_t k_full[2], k_empty[2], epi_bar;
   GroupSm grp[kMaxGroupsTc];
   int16_t order[kMaxHqTc];
@@ -224,7 +223,7 @@ template <bool kFold>
 __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     decode_tc_kernel(const __grid_constant__ Maps maps, const LayerTable lt, const DecodeArgs a,
                      const __grid_constant__ TcArgs ta) {
-  constexpr int kMma = Ring<kFold>::kMma, NWt = Ring<kFold>::NWt, kNA = Ring<kFold>::NA;
+  constexpr int kMma = Ring<kFold>::kMma, NW = Ring<kFold>::NW, kNA = Ring<kFold>::NA;
   constexpr int kThreads = Ring<kFold>::kThreads;
   extern __shared__ uint8_t smem_raw[];
   Smem<kFold>& sm =
@@ -243,10 +242,8 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     for (int i = 0; i < kFifoBars; ++i) {
       mbar_init(&sm.g_full[i], 1);      // even CTA: its producer's expect_tx; both CTAs' copies complete on it
       mbar_init(&sm.g_empty[i], kMma);  // released by every MMA thread (arrivals reach both CTAs)
-      for (int t = 0; t < kMma; ++t) {
-        mbar_init(&sm.u_full[t][i], 1);
-        mbar_init(&sm.u_empty[t][i], 1);
-      }
+      mbar_init(&sm.u_full[i], 1);
+      mbar_init(&sm.u_empty[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sm.k_full[i], 1);
@@ -314,14 +311,15 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
   PSegment seg;
 
   // Half items (this CTA's head, or its half of a lone head) of one unit into
-  // MMA thread rw's ring, in batches of at most NWt items: each batch is one
+  // the factor ring, in batches of at most NW items: each batch is one
   // instance of the ring (one full barrier, which the even CTA's lane 0 arms
-  // with the bytes of both CTAs' copies; one TMA copy per lane).
-  auto put_unit = [&](int rw, SlotFifo& f, int n, int np, int64_t img_row0, uint64_t pol) -> bool {
+  // with the bytes of both CTAs' copies; one TMA copy per lane).  The units of
+  // both MMA threads share the ring, in unit order.
+  auto put_unit = [&](SlotFifo& f, int n, int np, int64_t img_row0, uint64_t pol) -> bool {
     for (int p0 = 0; p0 < np;) {
-      const int nb = min(NWt, np - p0);
-      if (!f.claim(nb, NWt, sm.u_empty[rw], lane, abort_flag)) return false;
-      uint64_t* full = &sm.u_full[rw][f.inst % kFifoBars];
+      const int nb = min(NW, np - p0);
+      if (!f.claim(nb, NW, sm.u_empty, lane, abort_flag)) return false;
+      uint64_t* full = &sm.u_full[f.inst % kFifoBars];
       if (leader && lane == 0) {
         uint32_t total = 0;
         for (int q = 0; q < nb; ++q) total += (ta.item[n + p0 + q] >> 26) << 12;
@@ -329,7 +327,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
       }
       __syncwarp();
       if (lane < nb) {
-        const int sl = rw * NWt + (f.head + lane) % NWt;
+        const int sl = (f.head + lane) % NW;
         const uint32_t it = ta.item[n + p0 + lane];
         const uint32_t hrows = ((it >> 26) << 12) / 256;
         const int64_t y = img_row0 + ((it & 0x03FFFFFFu) >> 7) + hr * hrows;
@@ -350,10 +348,8 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     // units' items) ---------------------------------------------------------
     if (has_work) {
       const uint64_t pol = policy_evict_first();
-      const uint64_t pol_w = policy_evict_last();
-      SlotFifo ga, fw;  // the latent ring; MMA thread 1's factor ring (query-folded mode)
-      int kc = 0;
-      bool ok = true, images_ready = false;
+      SlotFifo ga;  // the latent ring
+      bool ok = true;
       // L2 prefetch of this half's latent rows, kPrefetchAhead tiles ahead of the
       // loads (across segment boundaries): the TMA loads then find them in L2
       PairWalker pwalk[2] = {walk_m, walk_x};
@@ -399,15 +395,6 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
               }
               __syncwarp();
               ga.advance(np);
-              if (kMma == 2)
-                for (int u = lo; u < hi && ok; ++u, ++kc) {
-                  if ((kc & 1) != 1) continue;  // MMA thread 0's unit
-                  if (!images_ready) {          // the images are written by the preparation kernel
-                    griddep_wait();
-                    images_ready = true;
-                  }
-                  ok = put_unit(1, fw, gs.i0 + u * np, np, img_row0, pol_w);
-                }
             }
           }
         }
@@ -419,9 +406,8 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     if (has_work) {
       const uint64_t pol = policy_evict_last();
       griddep_wait();  // the images are written by the preparation kernel
-      SlotFifo fw;         // MMA thread 0's factor ring
+      SlotFifo fw;         // the factor ring
       bool ok = true;
-      int kc = 0;          // units so far
       for (int ph = 0; ph < 2 && ok; ++ph)
         for (PairWalker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
           const int64_t img_row0 = kFold ? (int64_t)seg.b * img_seq_rows : 0;
@@ -432,8 +418,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
               const GroupSm& gs = sm.grp[g];
               const int np = gs.np;
               const int lo = max(ua - gs.u0, 0), hi = min(ub - gs.u0, (int)gs.nu);
-              for (int u = lo; u < hi && ok; ++u, ++kc)
-                if (kMma == 1 || (kc & 1) == 0) ok = put_unit(0, fw, gs.i0 + u * np, np, img_row0, pol);
+              for (int u = lo; u < hi && ok; ++u) ok = put_unit(fw, gs.i0 + u * np, np, img_row0, pol);
             }
           }
         }
@@ -452,7 +437,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     if (leader && lane == 0 && has_work) {
       const int t = warp == 1 ? 0 : 1;
       int gi = 0, ghead = 0;  // latent-ring instances (groups) and slots handed out so far
-      int ui = 0, uhead = 0;  // this thread's factor-ring instances (item batches) and slots
+      int ui = 0, uhead = 0;  // factor-ring instances (item batches of every unit) and slots
       int kc = 0, own = 0;    // units of the pair so far, units in this thread's accumulator
       bool ok = true;
       for (int ph = 0; ph < 2 && ok; ++ph)
@@ -474,7 +459,12 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
                 mbar_arrive(&sm.g_empty[gb]);
                 mbar_arrive_cluster(peer(&sm.g_empty[gb]));
               }
-              for (int u = uf; u < hi && ok; u += kMma) {
+              for (int u = lo; u < hi && ok; ++u) {
+                if (u < uf || (u - uf) % kMma != 0) {  // the other thread's unit: skip its item batches
+                  ui += (np + NW - 1) / NW;
+                  uhead += np;
+                  continue;
+                }
                 const int nh = min(2, gs.nh - 2 * u);
                 const uint32_t idesc_k = idesc_bf16(256, kD * nh, false, true);
                 const int kg = kc + (u - lo);                        // unit index of the pair
@@ -482,9 +472,9 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
                 const int use = kMma == 2 ? own : (kg >> 1);         // earlier units in this accumulator
                 const uint32_t dcol = tmem + buf * kKCols;
                 for (int p0 = 0; p0 < np && ok;) {  // the unit's item batches (ring instances)
-                  const int nb = min(NWt, np - p0);
+                  const int nb = min(NW, np - p0);
                   const int ub_ = ui % kFifoBars;
-                  if (!(ok = mbar_wait(&sm.u_full[t][ub_], (ui / kFifoBars) & 1, abort_flag))) break;
+                  if (!(ok = mbar_wait(&sm.u_full[ub_], (ui / kFifoBars) & 1, abort_flag))) break;
                   if (p0 == 0 && use >= 1) {  // both CTAs' epilogues have read this accumulator's previous unit
                     if (!(ok = mbar_wait(&sm.k_empty[buf], (use - 1) & 1, abort_flag))) break;
                   }
@@ -493,7 +483,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
                     const int p = p0 + q;
                     const int w = gs.w[p];
                     const uint32_t ab0 = smem_u32(sm.a[(ghead + p) % kNA]);
-                    const uint32_t bb = smem_u32(sm.w[t * NWt + (uhead + q) % NWt]);
+                    const uint32_t bb = smem_u32(sm.w[(uhead + q) % NW]);
                     const uint32_t swz = swz_of(w);
                     for (int k = 0; k < w / 16; ++k) {
                       const uint64_t ad = sdesc(ab0 + k * 32, 16, 16 * w, swz);
@@ -501,7 +491,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
                       umma_f16_pair(dcol, ad, bd, idesc_k, (p > 0 || k > 0) ? 1u : 0u);
                     }
                   }
-                  umma_commit_pair(&sm.u_empty[t][ub_]);  // the batch's slots, once its MMAs are done
+                  umma_commit_pair(&sm.u_empty[ub_]);  // the batch's slots, once its MMAs are done
                   ++ui;
                   uhead += nb;
                   p0 += nb;
