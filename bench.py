@@ -149,7 +149,7 @@ def workload_config(w, world: int) -> dict:
     ctx = (sorted(int(x) for x in set(w.seq_lens))[:4] if w.n_layers == 1
            else f"ragged U[1024,16384], mean {sum(w.seq_lens) / len(w.seq_lens):.0f}")
     return {"workload": w.name, "batch": w.batch, "context": ctx, "layers": w.n_layers,
-            "step": "latent append of B tokens + decode attention, per layer",
+            "step": "latent append of B tokens + decode attention, per layer (one dck_decode_step call)",
             "l2": "flushed between steps (512 MB write outside the timed events)",
             "parallelism": f"replicas x{world}"}
 
@@ -256,14 +256,16 @@ def job_throughput(world: int, batch: int, steps: int, t_ms: float) -> float:
 # per-kernel breakdown of one decode call
 # ---------------------------------------------------------------------------
 
-def decode_kernel_names(dck, buf):
-    """Kernels of one decode call, in launch order (from the launch count of a plain call)."""
-    dck.check(buf.run(), "decode")
+def decode_kernel_names(dck, step_fn):
+    """Kernels of one decode step call, in launch order (from the launch count of a plain step)."""
+    step_fn()
     n = dck.dck_last_launch_count()
     if n == 4:
-        return ["factor_prep", "scores", "absorb", "combine"]
+        return ["factor_prep+append", "scores", "absorb", "combine"]
     if n == 2:
         return ["decode_simt", "combine"]
+    if n >= 3:
+        return ["append"] * (n - 2) + ["decode_simt", "combine"]
     return [f"kernel{i}" for i in range(n)]
 
 
@@ -283,8 +285,9 @@ def kernel_work(buf, name):
         return buf.n_rows * s.rank_v * el, val_flops
     if name == "combine":
         return bv + qo, 0
-    if name == "factor_prep":
-        return bk + qo, 0
+    if name == "factor_prep+append":
+        app = s.hidden * (s.rank_k + s.rank_v) * el + buf.B * (s.hidden + s.rank_k + s.rank_v) * el
+        return bk + qo + app, 2 * buf.B * s.hidden * (s.rank_k + s.rank_v)
     if name == "decode_simt":
         return buf.n_rows * (s.rank_k + s.rank_v) * el + bk + qo, 0
     return 0, 0
@@ -372,24 +375,23 @@ def main():
         x = torch.empty((B, spec.hidden), dtype=dt, device=dev)
         device.synth_fill(x, S.stream_key(w.seed, l, S.TID["x_step"]), 1.0)
         rows = (buf.seq_start + buf.seq_len.to(torch.int64) - 1).contiguous()
-        ws_a = dck.dck_latent_append_workspace_size(buf.layer, B)
-        wsa = torch.empty(max(ws_a, 256), dtype=torch.uint8, device=dev)
-        layers.append((buf, A_k, A_v, x, rows, wsa, ws_a))
+        ws_s = dck.dck_decode_step_workspace_size(buf.layer, B, buf.n_rows)
+        wss = torch.empty(max(ws_s, 256), dtype=torch.uint8, device=dev)
+        layers.append((buf, A_k, A_v, x, rows, wss, ws_s))
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
     launches = [0]
 
     def step(q_src=None, x_src=None, st=None):
+        """One decode step per layer: latent append of the batch's new tokens and decode
+        attention over the caches that now hold them, one dck_decode_step call."""
         st = torch.cuda.current_stream(dev) if st is None else st
-        for l, (buf, A_k, A_v, x, rows, wsa, ws_a) in enumerate(layers):
+        for l, (buf, A_k, A_v, x, rows, wss, ws_s) in enumerate(layers):
             xx = x if x_src is None else x_src[l]
-            dck.check(dck.dck_latent_append(buf.layer, xx, B, A_k, A_v, rows, buf.kcache, buf.vcache, buf.n_rows,
-                                            wsa, ws_a, st), "append")
-            launches[0] += dck.dck_last_launch_count()
             qq = buf.q if q_src is None else q_src[l]
-            dck.check(dck.dck_decode_attention(buf.layer, qq, buf.kcache, buf.vcache, buf.n_rows, buf.B_k, buf.B_v,
-                                               buf.seq_start, buf.seq_len, B, spec.rope_theta, buf.out,
-                                               buf.workspace, buf.ws_bytes, st), "decode")
+            dck.check(dck.dck_decode_step(buf.layer, xx, A_k, A_v, rows, qq, buf.kcache, buf.vcache, buf.n_rows,
+                                          buf.B_k, buf.B_v, buf.seq_start, buf.seq_len, B, spec.rope_theta,
+                                          buf.out, wss, ws_s, st), "decode step")
             launches[0] += dck.dck_last_launch_count()
 
     for _ in range(args.warmup):
@@ -413,7 +415,7 @@ def main():
         step()
     per_step_launches = launches[0]
     dck.check(dck.dck_set_timing_events(None), "timing events")
-    decode_kernels = decode_kernel_names(dck, layers[-1][0])
+    decode_kernels = decode_kernel_names(dck, step)
     for _ in range(args.warmup):
         flush.fill_(1)
         graph.replay()
@@ -486,20 +488,21 @@ def main():
     e2e_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in eev), world, dev)
     e2e_value = job_throughput(world, B, K, e2e_ms)
 
-    # ---- roofline of one whole decode call (every kernel between the two hook events;
-    # one call = one layer), then a per-kernel breakdown from a separate capture ----
+    # ---- roofline of one whole decode-step call (append + decode attention: every kernel
+    # between the two hook events; one call = one layer), then a per-kernel breakdown ----
     peaks = load_peaks()
     buf0 = layers[-1][0]
-    alg_bytes = buf0.algorithmic_bytes()
-    flops = buf0.tensor_flops()
+    el0 = 2 if spec.dtype == "bf16" else 4
+    app_bytes = (spec.hidden * (spec.rank_k + spec.rank_v) + B * (spec.hidden + spec.rank_k + spec.rank_v)) * el0
+    alg_bytes = buf0.algorithmic_bytes() + app_bytes
+    flops = buf0.tensor_flops() + 2 * B * spec.hidden * (spec.rank_k + spec.rank_v)
     k_avg_s = statistics.mean(kern_ms) / 1e3
     achieved_gbs = alg_bytes / k_avg_s / 1e9
     tflops = flops / k_avg_s / 1e12
-    step_alg_bytes = sum(b.algorithmic_bytes() for (b, *_r) in layers) + \
-        sum((a.numel() + v.numel()) * a.element_size() for (_b, a, v, *_r) in layers)
+    step_alg_bytes = len(layers) * alg_bytes
     roof = {"bound": "hbm", "achieved": achieved_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
             "frac": achieved_gbs / peaks["hbm_gbs"], "traffic": profiled_traffic(args.config),
-            "kernel": "one whole decode call: " + " + ".join(decode_kernels), "kernel_us": 1e6 * k_avg_s,
+            "kernel": "one whole decode-step call: " + " + ".join(decode_kernels), "kernel_us": 1e6 * k_avg_s,
             "alg_bytes_per_launch": alg_bytes, "peak_source": peaks["source"],
             "tensor_tflops": tflops, "tensor_frac": tflops / peaks["bf16_tflops"],
             "roofline_us": 1e6 * max(alg_bytes / (peaks["hbm_gbs"] * 1e9), flops / (peaks["bf16_tflops"] * 1e12)),

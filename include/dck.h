@@ -151,6 +151,34 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q,
                                 void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * One decode step of a layer: the latent append of the batch's new tokens
+ * (Sec. III-A z = x L) followed by decode attention over the caches that now
+ * hold them (the formula at the top of this file).
+ *   x           [B, D] the new tokens' hidden states, one per sequence
+ *   A_k, A_v    as for dck_latent_append
+ *   d_rows      device int64 [B]: cache row that receives sequence b's new
+ *               token, normally d_seq_start[b] + d_seq_len[b] - 1 (its
+ *               position L_b - 1, where its own query attends)
+ *   the rest    as for dck_decode_attention; kcache and vcache are written
+ *   workspace   at least dck_decode_step_workspace_size(desc, B, n_rows)
+ *               bytes, 256-byte aligned
+ * On the bf16 tensor-core path with B <= 64 and D a multiple of 128 the
+ * append is computed by extra blocks of the call's first kernel (fp32
+ * accumulation, one read of A_k and A_v) and the attention kernels read the
+ * caches only after it; otherwise the call runs dck_latent_append and then
+ * dck_decode_attention on the same stream.  Results equal those of the two
+ * calls made one after the other (the appended rows are rounded to the cache
+ * dtype in both).  Errors as for the two calls (rows outside the cache are
+ * skipped and recorded in the device error word).
+ */
+size_t dck_decode_step_workspace_size(const dck_layer_desc* desc, int32_t batch, int64_t n_rows);
+dck_status dck_decode_step(const dck_layer_desc* desc, const void* x, const void* A_k, const void* A_v,
+                           const int64_t* d_rows, const void* q, void* kcache, void* vcache, int64_t n_rows,
+                           const void* B_k, const void* B_v, const int64_t* d_seq_start,
+                           const int32_t* d_seq_len, int32_t batch, float rope_theta, void* out,
+                           void* workspace, size_t ws_bytes, void* stream);
+
+/*
  * Decode attention for callers that cannot allocate device memory (the paper
  * has no counterpart: this is a deployment convenience of the library).
  * A runtime whose device memory is fully reserved by its own pool, a plug-in

@@ -66,6 +66,7 @@ struct AbsArgs {
   const uint8_t* pglob;
   const float* mglob;
   int64_t max_tiles;
+  int early_values;  // value loads may start before the scores kernel completes
 };
 
 struct ASmem {
@@ -275,7 +276,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
             ++v_cnt[r];
           };
           if (first) {  // the chunks that fit the empty rings, ahead of the wait
-            for (; done < nch; ++done) {
+            for (; done < nch && aa.early_values; ++done) {
               int c, r;
               chunk_at(done, c, r);
               if (v_cnt[r] >= kNVr) break;
@@ -519,6 +520,7 @@ cudaError_t launch_absorb_tc(const LayerTable& lt, const DecodeArgs& a, const Tc
   aa.pglob = r.pglob;
   aa.mglob = r.mglob;
   aa.max_tiles = r.max_tiles;
+  aa.early_values = r.early_values ? 1 : 0;
   const size_t smem = sizeof(ASmem) + 1024;
   static int attr_done[64] = {};
   int dev = 0;

@@ -8,6 +8,7 @@
 
 #include "common.cuh"
 #include "tc_common.cuh"
+#include "tc_host.h"
 
 namespace dck {
 bool simt_supports(const LayerTable& lt);
@@ -15,7 +16,8 @@ bool combine_supports(const LayerTable& lt);
 bool tc_decode_supports(const LayerTable& lt, int dtype);
 size_t tc_decode_extra_ws(const LayerTable& lt, int batch, int64_t n_rows);
 int tc_decode_pairs(const LayerTable& lt);
-cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s);
+cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, const TcStepAppend* app, cudaStream_t s);
+bool tc_step_append_supports(const LayerTable& lt, int D, int batch);
 bool tc_append_supports(int D, int Rk, int rv, int dtype);
 size_t tc_append_workspace(int n_tok, int Rk, int rv);
 cudaError_t launch_bounded_wait_selftest(long long limit_cycles, int* err, cudaStream_t s);
@@ -209,10 +211,16 @@ dck_status decode_precheck(const dck_layer_desc* desc, const void* q, const void
 
 extern "C" {
 
-dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const void* kcache, const void* vcache,
-                                int64_t n_rows, const void* B_k, const void* B_v, const int64_t* d_seq_start,
-                                const int32_t* d_seq_len, int32_t batch, float rope_theta, void* out,
-                                void* workspace, size_t ws_bytes, void* stream) {
+}  // extern "C"
+
+namespace {
+// The decode call, optionally with the decode step's latent append fused into
+// its first launch (app != nullptr: the caller has checked that the fused
+// append applies).
+dck_status decode_call(const dck_layer_desc* desc, const void* q, const void* kcache, const void* vcache,
+                       int64_t n_rows, const void* B_k, const void* B_v, const int64_t* d_seq_start,
+                       const int32_t* d_seq_len, int32_t batch, float rope_theta, void* out, void* workspace,
+                       size_t ws_bytes, const TcStepAppend* app, void* stream) {
   t_last_launches = 0;
   const dck_status st =
       decode_precheck(desc, q, kcache, vcache, n_rows, B_k, B_v, d_seq_start, d_seq_len, batch, rope_theta, out);
@@ -250,19 +258,82 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const
                         ? std::min(tc_decode_pairs(lt), sms / 2)
                         : 0;
   const bool use_tc = pairs > 0;
+  if (app && !use_tc) return DCK_ERR_UNSUPPORTED;
   LaunchHook hook;
   hook.ev = t_events;
   hook.n_ev = t_n_events;
   a.hook = &hook;
   a.split_extra = use_tc ? 1 : 0;
   if (use_tc) a.n_items = 2 * pairs;  // the tensor-core kernels run on the pairs' SMs
-  if (use_tc) e = launch_decode_tc(lt, a, s);
+  if (use_tc) e = launch_decode_tc(lt, a, app, s);
   else e = launch_decode_simt(lt, a, desc->dtype, s);
   if (e != cudaSuccess) return DCK_ERR_CUDA;
   e = launch_combine(lt, a, desc->dtype, s);
   t_last_launches = hook.count;
   if (e != cudaSuccess) return DCK_ERR_CUDA;
   return DCK_OK;
+}
+
+// Whether dck_decode_step can fuse the append into the decode call.
+bool step_fuses(const dck_layer_desc* desc, int32_t batch, int64_t n_rows) {
+  if (check_desc(desc) != DCK_OK || desc->dtype != DCK_BF16 || batch < 1) return false;
+  const LayerTable lt = make_table(desc);
+  int sms = 0;
+  if (!device_state(nullptr, &sms)) return false;
+  return t_decode_kernel == 0 && n_rows < (int64_t(1) << 31) - 256 && tc_decode_supports(lt, desc->dtype) &&
+         tc_step_append_supports(lt, desc->hidden, batch) && std::min(tc_decode_pairs(lt), sms / 2) > 0;
+}
+}  // namespace
+
+extern "C" {
+
+dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q, const void* kcache, const void* vcache,
+                                int64_t n_rows, const void* B_k, const void* B_v, const int64_t* d_seq_start,
+                                const int32_t* d_seq_len, int32_t batch, float rope_theta, void* out,
+                                void* workspace, size_t ws_bytes, void* stream) {
+  return decode_call(desc, q, kcache, vcache, n_rows, B_k, B_v, d_seq_start, d_seq_len, batch, rope_theta, out,
+                     workspace, ws_bytes, nullptr, stream);
+}
+
+size_t dck_decode_step_workspace_size(const dck_layer_desc* desc, int32_t batch, int64_t n_rows) {
+  const size_t dw = dck_decode_workspace_size(desc, batch, n_rows);
+  if (dw == 0) return 0;
+  // the separate append (when the fused one does not apply) uses the space after the decode workspace
+  return align_up(dw, 256) + align_up(dck_latent_append_workspace_size(desc, batch), 256);
+}
+
+dck_status dck_decode_step(const dck_layer_desc* desc, const void* x, const void* A_k, const void* A_v,
+                           const int64_t* d_rows, const void* q, void* kcache, void* vcache, int64_t n_rows,
+                           const void* B_k, const void* B_v, const int64_t* d_seq_start, const int32_t* d_seq_len,
+                           int32_t batch, float rope_theta, void* out, void* workspace, size_t ws_bytes,
+                           void* stream) {
+  t_last_launches = 0;
+  const dck_status st =
+      decode_precheck(desc, q, kcache, vcache, n_rows, B_k, B_v, d_seq_start, d_seq_len, batch, rope_theta, out);
+  if (st != DCK_OK || batch == 0) return st;
+  if (!x || !A_k || !A_v || !d_rows || !aligned(x, 16) || !aligned(A_k, 16) || !aligned(A_v, 16))
+    return DCK_ERR_INVALID;
+  if (step_fuses(desc, batch, n_rows)) {
+    TcStepAppend app;
+    app.x = x;
+    app.A_k = A_k;
+    app.A_v = A_v;
+    app.rows = d_rows;
+    app.D = desc->hidden;
+    return decode_call(desc, q, kcache, vcache, n_rows, B_k, B_v, d_seq_start, d_seq_len, batch, rope_theta, out,
+                       workspace, ws_bytes, &app, stream);
+  }
+  // separate append, then the decode call (the append's scratch after the decode workspace)
+  const size_t dw = align_up(dck_decode_workspace_size(desc, batch, n_rows), 256);
+  if (!workspace || ws_bytes < dw) return DCK_ERR_WORKSPACE;
+  dck_status r = dck_latent_append(desc, x, batch, A_k, A_v, d_rows, kcache, vcache, n_rows,
+                                   static_cast<char*>(workspace) + dw, ws_bytes - dw, stream);
+  if (r != DCK_OK) return r;
+  const int appended = t_last_launches;
+  r = dck_decode_attention(desc, q, kcache, vcache, n_rows, B_k, B_v, d_seq_start, d_seq_len, batch, rope_theta,
+                           out, workspace, dw, stream);
+  t_last_launches += appended;
+  return r;
 }
 
 size_t dck_latent_append_workspace_size(const dck_layer_desc* desc, int32_t n_tok) {

@@ -369,6 +369,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
         if (nr > 0) prefetch_l2(static_cast<const __nv_bfloat16*>(a.kc) + r0 * lt.Rk, (uint32_t)(nr * lt.Rk * 2));
       };
       for (int q = 0; q < kPrefetchAhead; ++q) prefetch_next();
+      griddep_wait();  // the preparation launch may append the step's own latents
       for (int ph = 0; ph < 2 && ok; ++ph)
         for (PairWalker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
           const int64_t img_row0 = kFold ? (int64_t)seg.b * img_seq_rows : 0;
@@ -795,12 +796,166 @@ struct PrepItem {
   int32_t off;           // byte offset in a sequence's image
 };
 
+// The decode step's latent append, done by extra blocks of the preparation
+// launch: z_b = x_b [A_k | A_v] for the batch's new tokens, written to cache
+// row rows[b] (Sec. III-A z = x L; Sec. III-C L_g side by side; Sec. III-D L_v).
+struct StepAppend {
+  const __nv_bfloat16* x;   // [B, D]
+  const __nv_bfloat16* Ak;  // [D, Rk]
+  const __nv_bfloat16* Av;  // [D, rv]
+  const int64_t* rows;      // [B]
+  int D;
+  int n_blocks;             // GEMV blocks: one per 16 output columns
+};
+
 struct PrepArgs {
   int n_items;
   int64_t seq_bytes;
   double om[kD / 2];  // RoPE frequencies, fp64
   PrepItem item[kMaxItems];
+  StepAppend app;
 };
+
+constexpr int kAppCols = 16;     // output columns of one GEMV block
+constexpr int kAppMaxTok = 64;   // tokens of a fused append
+constexpr int kAppWarps = 8;     // warps of a GEMV block, each a K range of D / 8
+
+// d += a b for one 16 x 8 x 16 tile, bf16 inputs, fp32 accumulators (row.col).
+__device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                          uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Four 8x8 b16 matrices from shared memory, transposed.
+__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+
+// 16-byte global -> shared copies tracked per thread (cp.async groups).
+__device__ __forceinline__ void cp_async16_cg(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit_group() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Four 8x8 b16 matrices from shared memory.
+__device__ __forceinline__ void ldmatrix_x4_plain(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+
+constexpr int kAppStages = 6;    // k-steps of a warp in flight
+// Dynamic shared memory of the append blocks: per warp kAppStages stages of a
+// factor tile (512 B) and an x tile (16 tokens x 16 k per token m-tile), then
+// the warps' partial sums.
+__host__ __device__ inline int app_stage_bytes(int batch) { return 512 + ((batch + 15) / 16) * 512; }
+__host__ __device__ inline size_t app_smem_bytes(int batch) {
+  return (size_t)kAppWarps * kAppStages * app_stage_bytes(batch) + (size_t)kAppWarps * batch * kAppCols * 4;
+}
+
+// One GEMV block: output columns [c0, c0 + 16) of [A_k | A_v] for B <= 64
+// tokens.  Warp w accumulates K range [w D / 8, (w + 1) D / 8) with mma
+// m16n8k16 (tokens x K) . (K x 16 columns).  Each k-step's factor tile
+// [16 k][16 columns] and x tile [tokens][16 k] go through a per-warp ring of
+// cp.async stages, kAppStages k-steps ahead, so the factor stream (read once)
+// keeps enough bytes in flight; ldmatrix reads the operands (.trans for the
+// column-major factor).  The eight warps' partial sums are added in shared
+// memory, rounded to bf16 and written to the cache rows.
+__device__ __forceinline__ void step_append_block(const LayerTable& lt, const DecodeArgs& a, const StepAppend& ap,
+                                                  int blk) {
+  extern __shared__ __align__(128) uint8_t app_dyn[];
+  const int sb = app_stage_bytes(a.B);
+  float* red = reinterpret_cast<float*>(app_dyn + (size_t)kAppWarps * kAppStages * sb);  // [warp][B * 16]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gid = lane >> 2, tig = lane & 3;
+  const int c0 = blk * kAppCols;
+  const bool is_k = c0 < lt.Rk;
+  const int N = is_k ? lt.Rk : lt.rv;
+  const __nv_bfloat16* A = (is_k ? ap.Ak : ap.Av) + (is_k ? c0 : c0 - lt.Rk);
+  const int B = a.B, D = ap.D;
+  const int mt = (B + 15) / 16;  // token m-tiles
+  const int kr = D / kAppWarps, kbeg = warp * kr, nks = kr / 16;
+  float acc[kAppMaxTok / 16][2][4];
+#pragma unroll
+  for (int m = 0; m < kAppMaxTok / 16; ++m)
+#pragma unroll
+    for (int n = 0; n < 2; ++n)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) acc[m][n][q] = 0.f;
+  const uint32_t rbase = smem_u32(app_dyn + (size_t)warp * kAppStages * sb);
+  // stage kk: factor rows k (lane / 2), columns 8 (lane & 1) ..; x rows t, 16-byte halves h (two per row)
+  auto issue = [&](int kk) {
+    const uint32_t st = rbase + (uint32_t)((kk % kAppStages) * sb);
+    if (kk < nks) {
+      const int k0 = kbeg + 16 * kk;
+      cp_async16_cg(st + (uint32_t)(((lane >> 1) * 16 + 8 * (lane & 1)) * 2),
+                    A + (int64_t)(k0 + (lane >> 1)) * N + 8 * (lane & 1));
+      for (int e = lane; e < 2 * 16 * mt; e += 32) {  // x rows of the token m-tiles (zero rows past B)
+        const int t = e >> 1, h = e & 1;
+        const uint32_t dst = st + 512 + (uint32_t)((t * 16 + 8 * h) * 2);
+        if (t < B) cp_async16_cg(dst, ap.x + (int64_t)t * D + k0 + 8 * h);
+        else asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" ::"r"(dst), "r"(0u) : "memory");
+      }
+    }
+    cp_async_commit_group();
+  };
+#pragma unroll
+  for (int q = 0; q < kAppStages - 1; ++q) issue(q);
+  for (int kk = 0; kk < nks; ++kk) {
+    issue(kk + kAppStages - 1);
+    cp_async_wait_group<kAppStages - 1>();  // stage kk has landed (this thread's copies)
+    __syncwarp();
+    const uint32_t st = rbase + (uint32_t)((kk % kAppStages) * sb);
+    // B fragments: matrix m = lane / 8 covers k rows 8 (m & 1) .., n columns 8 (m >> 1) ..
+    uint32_t bf[4];
+    const int m8 = lane >> 3, r8 = lane & 7;
+    ldmatrix_x4_trans(bf, st + (uint32_t)(((8 * (m8 & 1) + r8) * 16 + 8 * (m8 >> 1)) * 2));
+#pragma unroll
+    for (int m = 0; m < kAppMaxTok / 16; ++m) {
+      if (m >= mt) break;
+      // A fragments (tokens 16 m .., k 0..15): matrix q = lane / 8 covers rows 8 (q & 1) .., k 8 (q >> 1) ..
+      uint32_t af[4];
+      ldmatrix_x4_plain(af, st + 512 + (uint32_t)(((16 * m + 8 * (m8 & 1) + r8) * 16 + 8 * (m8 >> 1)) * 2));
+      mma_16816(acc[m][0], af[0], af[1], af[2], af[3], bf[0], bf[1]);
+      mma_16816(acc[m][1], af[0], af[1], af[2], af[3], bf[2], bf[3]);
+    }
+    __syncwarp();  // every lane is done with the stage before it is refilled
+  }
+  cp_async_wait_group<0>();
+  // partial sums -> shared memory: token 16 m + gid (+8), column 8 n + 2 tig (+1)
+#pragma unroll
+  for (int m = 0; m < kAppMaxTok / 16; ++m)
+#pragma unroll
+    for (int n = 0; n < 2; ++n)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int t = 16 * m + gid + 8 * (q >> 1), c = 8 * n + 2 * tig + (q & 1);
+        if (t < B) red[warp * B * kAppCols + t * kAppCols + c] = acc[m][n][q];
+      }
+  __syncthreads();
+  __nv_bfloat16* cache = static_cast<__nv_bfloat16*>(const_cast<void*>(is_k ? a.kc : a.vc));
+  for (int e = threadIdx.x; e < B * kAppCols; e += blockDim.x) {
+    const int t = e / kAppCols, c = e % kAppCols;
+    float v = 0.f;
+#pragma unroll
+    for (int w = 0; w < kAppWarps; ++w) v += red[w * B * kAppCols + e];
+    const int64_t row = ap.rows[t];
+    if (row < 0 || row >= a.n_rows) {
+      if (c == 0) atomicOr(a.err, kErrBadRow);
+      continue;
+    }
+    cache[row * N + (is_k ? c0 : c0 - lt.Rk) + c] = __float2bfloat16_rn(v);
+  }
+}
 
 // One block writes one factor item: [nh heads][2 halves][ws rank rows]
 // [64 columns] bf16, 128B-swizzled (16-byte chunk c of row r stored at chunk
@@ -810,11 +965,19 @@ struct PrepArgs {
 //   a_i B[:, i] + b_i B[:, i+64]  and  b_i B[:, i] - a_i B[:, i+64]
 // with (a, b) the halves of RoPE(q_{b,h}, L_b - 1) * log2(e)/sqrt(d); each
 // thread loads its B_g values once and writes them folded for every sequence.
+// Blocks in rows after the preparation rows do the decode step's latent
+// append (step_append_block), when the call has one.
 constexpr int kPrepSeqs = 4;
 template <bool kFold>
 __global__ void __launch_bounds__(256) factor_prep_kernel(const LayerTable lt, const DecodeArgs a, const PrepArgs pa,
                                                           uint8_t* __restrict__ img) {
   griddep_launch();
+  const int prep_rows = kFold ? (a.B + kPrepSeqs - 1) / kPrepSeqs : 1;
+  if ((int)blockIdx.y >= prep_rows) {  // a block of the fused decode-step append
+    const int blk = (blockIdx.y - prep_rows) * gridDim.x + blockIdx.x;
+    if (blk < pa.app.n_blocks) step_append_block(lt, a, pa.app, blk);
+    return;
+  }
   const int n = blockIdx.x, bs0 = blockIdx.y * kPrepSeqs;
   const int nbs = kFold ? min(kPrepSeqs, a.B - bs0) : 1;
   const PrepItem it = pa.item[n];
@@ -987,7 +1150,14 @@ cudaError_t launch_mode(const LayerTable& lt, const DecodeArgs& a, const Maps& m
                         const PrepArgs& pa, cudaStream_t s) {
   cudaError_t e = set_smem_attr<kFold>();
   if (e != cudaSuccess) return e;
-  factor_prep_kernel<kFold><<<dim3(pa.n_items, kFold ? (a.B + kPrepSeqs - 1) / kPrepSeqs : 1), 256, 0, s>>>(
+  const int prep_rows = kFold ? (a.B + kPrepSeqs - 1) / kPrepSeqs : 1;
+  const int app_rows = (pa.app.n_blocks + pa.n_items - 1) / pa.n_items;
+  const size_t app_smem = pa.app.n_blocks ? app_smem_bytes(a.B) : 0;
+  if (app_smem) {
+    e = cudaFuncSetAttribute(factor_prep_kernel<kFold>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)app_smem);
+    if (e != cudaSuccess) return e;
+  }
+  factor_prep_kernel<kFold><<<dim3(pa.n_items, prep_rows + app_rows), 256, app_smem, s>>>(
       lt, a, pa, static_cast<uint8_t*>(a.extra));
   e = hook_launched(a.hook, s);
   if (e != cudaSuccess) return e;
@@ -1131,15 +1301,31 @@ size_t tc_decode_extra_ws(const LayerTable& lt, int batch, int64_t n_rows) {
   return extra_layout(lt, batch, n_rows).total;
 }
 
+// The fused decode-step append takes up to 64 tokens and widths D that split
+// into eight warp ranges of 16-wide k-steps.
+bool tc_step_append_supports(const LayerTable& lt, int D, int batch) {
+  return batch >= 1 && batch <= kAppMaxTok && D % (kAppWarps * 16) == 0 && lt.Rk % kAppCols == 0 &&
+         lt.rv % kAppCols == 0;
+}
+
 // CTA pairs of the tensor-core path on the current device (0 if it cannot run).
 int tc_decode_pairs(const LayerTable& lt) { return lt.qpg == 1 ? pairs_of_device<true>() : pairs_of_device<false>(); }
 
-cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) {
+cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, const TcStepAppend* app, cudaStream_t s) {
   const bool fold = lt.qpg == 1;
   if (!a.extra || a.n_items < 2 || (a.n_items & 1)) return cudaErrorInvalidValue;
   static thread_local TcArgs ta;
   static thread_local PrepArgs pa;
   if (!build_tables(lt, ta, pa)) return cudaErrorInvalidValue;
+  if (app) {
+    if (!tc_step_append_supports(lt, app->D, a.B)) return cudaErrorInvalidValue;
+    pa.app.x = static_cast<const __nv_bfloat16*>(app->x);
+    pa.app.Ak = static_cast<const __nv_bfloat16*>(app->A_k);
+    pa.app.Av = static_cast<const __nv_bfloat16*>(app->A_v);
+    pa.app.rows = app->rows;
+    pa.app.D = app->D;
+    pa.app.n_blocks = (lt.Rk + lt.rv) / kAppCols;
+  }
   rope_freqs(a.theta, ta.om);
   std::memcpy(pa.om, ta.om, sizeof(ta.om));
   const ExtraLayout xl = extra_layout(lt, a.B, a.n_rows);
@@ -1177,6 +1363,7 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, cudaStre
   r.mglob = ta.mglob;
   r.max_tiles = ta.max_tiles;
   r.hq_pad = ta.hq_pad;
+  r.early_values = app == nullptr;
   e = launch_absorb_tc(lt, a, r, s);
   return e != cudaSuccess ? e : hook_launched(a.hook, s);
 }

@@ -15,6 +15,17 @@ struct TcRegions {
   const float* mglob;    // [max_tiles][Hq]: reference max (log2 units) P of tile x was computed with
   int64_t max_tiles;
   int hq_pad;
+  bool early_values;     // value loads may start before the scores kernel completes (false when the
+                         // call's first launch also appends latents, which those loads could read)
+};
+
+// A decode step's latent append fused into the decode call (dck_decode_step).
+struct TcStepAppend {
+  const void* x;        // [B, D] bf16
+  const void* A_k;      // [D, R_k]
+  const void* A_v;      // [D, r_v]
+  const int64_t* rows;  // [B] cache row of each sequence's new token
+  int D;
 };
 
 // Launches the absorption kernel for the tiles the scores kernel just processed.

@@ -28,7 +28,7 @@ EXPORTED = (
     "dck_status_string", "dck_validate_desc", "dck_latent_append_workspace_size", "dck_latent_append",
     "dck_decode_workspace_size", "dck_decode_attention", "dck_last_device_error", "dck_set_decode_kernel",
     "dck_last_launch_count", "dck_synth_gaussian", "dck_set_timing_events", "dck_decode_attention_noalloc",
-    "dck_selftest_bounded_wait",
+    "dck_selftest_bounded_wait", "dck_decode_step", "dck_decode_step_workspace_size",
 )
 
 
@@ -79,6 +79,10 @@ def lib() -> ctypes.CDLL:
     L.dck_decode_workspace_size.argtypes = [D, I32, I64]
     L.dck_decode_attention.restype = I32
     L.dck_decode_attention.argtypes = [D, P, P, P, I64, P, P, P, P, I32, F32, P, P, SZ, P]
+    L.dck_decode_step_workspace_size.restype = SZ
+    L.dck_decode_step_workspace_size.argtypes = [D, I32, I64]
+    L.dck_decode_step.restype = I32
+    L.dck_decode_step.argtypes = [D, P, P, P, P, P, P, P, I64, P, P, P, P, I32, F32, P, P, SZ, P]
     L.dck_decode_attention_noalloc.restype = I32
     L.dck_decode_attention_noalloc.argtypes = [D, P, P, P, I64, P, P, P, P, I32, F32, P, P]
     L.dck_last_device_error.restype = I32
@@ -165,6 +169,19 @@ def dck_decode_attention(layer: Layer, q, kcache, vcache, n_rows: int, B_k, B_v,
     return lib().dck_decode_attention(layer.ref, _ptr(q), _ptr(kcache), _ptr(vcache), int(n_rows), _ptr(B_k),
                                       _ptr(B_v), _ptr(seq_start), _ptr(seq_len), int(batch), float(rope_theta),
                                       _ptr(out), _ptr(workspace), int(ws_bytes), _stream(stream))
+
+
+def dck_decode_step_workspace_size(layer: Layer, batch: int, n_rows: int) -> int:
+    return lib().dck_decode_step_workspace_size(layer.ref, batch, n_rows)
+
+
+def dck_decode_step(layer: Layer, x, A_k, A_v, rows, q, kcache, vcache, n_rows: int, B_k, B_v, seq_start, seq_len,
+                    batch: int, rope_theta: float, out, workspace, ws_bytes: int, stream=None) -> int:
+    """Latent append of the batch's new tokens, then decode attention (one call)."""
+    return lib().dck_decode_step(layer.ref, _ptr(x), _ptr(A_k), _ptr(A_v), _ptr(rows), _ptr(q), _ptr(kcache),
+                                 _ptr(vcache), int(n_rows), _ptr(B_k), _ptr(B_v), _ptr(seq_start), _ptr(seq_len),
+                                 int(batch), float(rope_theta), _ptr(out), _ptr(workspace), int(ws_bytes),
+                                 _stream(stream))
 
 
 def dck_decode_attention_noalloc(layer: Layer, q, kcache, vcache, n_rows: int, B_k, B_v, seq_start, seq_len,
