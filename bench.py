@@ -326,6 +326,174 @@ def kernel_breakdown(dck, torch, stream, flush, buf, step_fn, names, peaks, K):
 
 
 # ---------------------------------------------------------------------------
+# --sweep: the measurement matrix (decode vs context length, the 32-layer step
+# vs batch, every workload's call, the long-context prefill append)
+# ---------------------------------------------------------------------------
+
+def time_decode_steps(w, steps, warmup, dev, flush):
+    """Decode steps (one dck_decode_step per layer) of workload w, as a CUDA graph replayed with
+    L2 flushed between steps; CUDA-event times of the step and of the last layer's call."""
+    import torch
+    from paper_2607_24331_gb300 import dck, device
+    from paper_2607_24331_gb300 import synth as S
+    spec = w.layer
+    B = w.batch
+    dt = device.TORCH_DTYPE[spec.dtype]
+    layers = []
+    for l in range(w.n_layers):
+        buf = device.DecodeBuffers(spec, w.seq_lens, device=dev).synth(seed=w.seed, layer=l)
+        A_k = torch.empty((spec.hidden, spec.rank_k), dtype=dt, device=dev)
+        A_v = torch.empty((spec.hidden, spec.rank_v), dtype=dt, device=dev)
+        device.synth_fill(A_k, S.stream_key(w.seed, l, S.TID["A_k"]), 1.0 / math.sqrt(spec.hidden))
+        device.synth_fill(A_v, S.stream_key(w.seed, l, S.TID["A_v"]), 1.0 / math.sqrt(spec.hidden))
+        x = torch.empty((B, spec.hidden), dtype=dt, device=dev)
+        device.synth_fill(x, S.stream_key(w.seed, l, S.TID["x_step"]), 1.0)
+        rows = (buf.seq_start + buf.seq_len.to(torch.int64) - 1).contiguous()
+        ws_s = dck.dck_decode_step_workspace_size(buf.layer, B, buf.n_rows)
+        wss = torch.empty(max(ws_s, 256), dtype=torch.uint8, device=dev)
+        layers.append((buf, A_k, A_v, x, rows, wss, ws_s))
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        for buf, A_k, A_v, x, rows, wss, ws_s in layers:
+            dck.check(dck.dck_decode_step(buf.layer, x, A_k, A_v, rows, buf.q, buf.kcache, buf.vcache, buf.n_rows,
+                                          buf.B_k, buf.B_v, buf.seq_start, buf.seq_len, B, spec.rope_theta,
+                                          buf.out, wss, ws_s, stream), "decode step")
+
+    for _ in range(warmup):
+        flush.fill_(1)
+        step()
+    torch.cuda.synchronize()
+    assert dck.dck_last_device_error(stream) == dck.DCK_OK
+    kev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    for e_ in kev:
+        e_.record(stream)
+    torch.cuda.synchronize()
+    dck.check(dck.dck_set_timing_events(kev), "timing events")
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step()
+    dck.check(dck.dck_set_timing_events(None), "timing events")
+    graph.replay()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    call_ms = []
+    for k in range(steps):
+        flush.fill_(k & 0xFF)
+        ev[k][0].record(stream)
+        graph.replay()
+        ev[k][1].record(stream)
+        ev[k][1].synchronize()
+        call_ms.append(kev[0].elapsed_time(kev[1]))
+    step_ms = statistics.median(a.elapsed_time(b) for a, b in ev)
+    call_ms = statistics.median(call_ms)
+    buf0 = layers[-1][0]
+    el = 2 if spec.dtype == "bf16" else 4
+    app_bytes = (spec.hidden * (spec.rank_k + spec.rank_v) + B * (spec.hidden + spec.rank_k + spec.rank_v)) * el
+    call_bytes = buf0.algorithmic_bytes() + app_bytes
+    call_flops = buf0.tensor_flops() + 2 * B * spec.hidden * (spec.rank_k + spec.rank_v)
+    del graph, layers
+    torch.cuda.empty_cache()
+    return step_ms, call_ms, call_bytes, call_flops
+
+
+def time_prefill_append(w, steps, warmup, dev, flush):
+    """Latent append of w.append_tokens new tokens per sequence (dck_latent_append, rows at the end of
+    each sequence), CUDA events around each call, L2 flushed between calls."""
+    import numpy as np
+    import torch
+    from paper_2607_24331_gb300 import dck, device
+    from paper_2607_24331_gb300 import synth as S
+    spec = w.layer
+    dt = device.TORCH_DTYPE[spec.dtype]
+    n_tok = w.append_tokens * w.batch
+    n_rows = sum(w.seq_lens)
+    starts = S.seq_starts(w.seq_lens)
+    rows_h = np.concatenate([np.arange(int(st) + L - w.append_tokens, int(st) + L) for st, L in zip(starts, w.seq_lens)])
+    rows = torch.from_numpy(rows_h.astype(np.int64)).to(dev)
+    x = torch.empty((n_tok, spec.hidden), dtype=dt, device=dev)
+    A_k = torch.empty((spec.hidden, spec.rank_k), dtype=dt, device=dev)
+    A_v = torch.empty((spec.hidden, spec.rank_v), dtype=dt, device=dev)
+    kc = torch.empty((n_rows, spec.rank_k), dtype=dt, device=dev)
+    vc = torch.empty((n_rows, spec.rank_v), dtype=dt, device=dev)
+    device.synth_fill(x, S.stream_key(w.seed, 0, S.TID["x"]), 1.0)
+    device.synth_fill(A_k, S.stream_key(w.seed, 0, S.TID["A_k"]), 1.0 / math.sqrt(spec.hidden))
+    device.synth_fill(A_v, S.stream_key(w.seed, 0, S.TID["A_v"]), 1.0 / math.sqrt(spec.hidden))
+    L = dck.Layer.from_spec(spec)
+    wsb = dck.dck_latent_append_workspace_size(L, n_tok)
+    ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def call():
+        dck.check(dck.dck_latent_append(L, x, n_tok, A_k, A_v, rows, kc, vc, n_rows, ws, wsb, stream), "append")
+
+    for _ in range(warmup):
+        flush.fill_(1)
+        call()
+    torch.cuda.synchronize()
+    assert dck.dck_last_device_error(stream) == dck.DCK_OK
+    ms = []
+    for k in range(steps):
+        flush.fill_(k & 0xFF)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        call()
+        e1.record(stream)
+        e1.synchronize()
+        ms.append(e0.elapsed_time(e1))
+    el = 2
+    bytes_ = (n_tok * spec.hidden + spec.hidden * (spec.rank_k + spec.rank_v) + n_tok * (spec.rank_k + spec.rank_v)) * el
+    flops = 2 * n_tok * spec.hidden * (spec.rank_k + spec.rank_v)
+    del x, kc, vc
+    torch.cuda.empty_cache()
+    return statistics.median(ms), bytes_, flops
+
+
+def run_sweep(args):
+    import torch
+    from paper_2607_24331_gb300 import synth as S
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    peaks = load_peaks()
+    steps, warmup = max(args.steps, 3), max(args.warmup, 3)
+    out = {"sweep": [], "peaks": peaks}
+
+    def line(kind, w, step_ms, call_ms, bytes_, flops, extra=None):
+        ctx = sum(w.seq_lens)
+        d = {"kind": kind, "workload": w.name, "batch": w.batch, "layers": w.n_layers,
+             "mean_context": ctx / max(1, w.batch), "ms_per_step": step_ms, "call_us": 1e3 * call_ms,
+             "decode_tokens_per_s": w.batch / (step_ms / 1e3),
+             "context_tokens_per_s": ctx * w.n_layers / (step_ms / 1e3),
+             "call_alg_gbs": bytes_ / (call_ms / 1e3) / 1e9,
+             "hbm_frac_of_measured": bytes_ / (call_ms / 1e3) / 1e9 / peaks["hbm_gbs"],
+             "tensor_frac_of_measured": flops / (call_ms / 1e3) / 1e12 / peaks["bf16_tflops"],
+             "roofline_call_us": 1e6 * max(bytes_ / (peaks["hbm_gbs"] * 1e9), flops / (peaks["bf16_tflops"] * 1e12))}
+        if extra:
+            d.update(extra)
+        out["sweep"].append(d)
+        print(json.dumps(d), file=sys.stderr, flush=True)
+
+    base = S.workload(1)
+    for T in (1024, 4096, 16384, 65536):   # decode vs context length on the 7B MHA layer, B16
+        w = S.Workload(f"llama2-7b-mha B16 T{T}", base.layer, (T,) * 16)
+        line("context", w, *time_decode_steps(w, steps, warmup, dev, flush))
+    for cfg in (0, 2, 3, 5):
+        w = S.workload(cfg)
+        line("workload", w, *time_decode_steps(w, steps, warmup, dev, flush))
+    for b in (1, 8, 32, 64):               # the 32-layer step vs batch
+        w = S.workload(4, b)
+        line("32-layer step", w, *time_decode_steps(w, 3, 3, dev, flush))
+    w3 = S.workload(3)
+    ms, by, fl = time_prefill_append(w3, steps, warmup, dev, flush)
+    out["sweep"].append({"kind": "prefill append", "workload": f"{w3.name}: latent append of 2 x {w3.append_tokens} tokens",
+                         "us": 1e3 * ms, "tensor_tflops": fl / (ms / 1e3) / 1e12,
+                         "tensor_frac_of_measured": fl / (ms / 1e3) / 1e12 / peaks["bf16_tflops"],
+                         "roofline_us": 1e6 * max(by / (peaks["hbm_gbs"] * 1e9), fl / (peaks["bf16_tflops"] * 1e12))})
+    print(json.dumps(out), flush=True)
+
+
+# ---------------------------------------------------------------------------
 # the GPU arm
 # ---------------------------------------------------------------------------
 
@@ -339,11 +507,16 @@ def main():
     ap.add_argument("--batch", type=int, default=None, help="batch of the 32-layer workload (config 4)")
     ap.add_argument("--impl", default="dck", choices=["dck", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time for cpu_baseline")
+    ap.add_argument("--sweep", action="store_true",
+                    help="measurement matrix (context lengths, workloads, 32-layer batch sweep, prefill append)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
     if args.impl == "reference":
         run_reference(args)
+        return
+    if args.sweep:
+        run_sweep(args)
         return
 
     import numpy as np
