@@ -58,7 +58,8 @@ def kernel_source_sha():
     comment edit does not retire DRAM counters taken on the same code."""
     import re
     h = hashlib.sha256()
-    for fn in ("decode_tc.cu", "absorb_tc.cu", "tc_common.cuh", "sm100.cuh", "decode_simt.cu", "common.cuh"):
+    for fn in ("decode_tc.cu", "absorb_tc.cu", "combine.cu", "tc_common.cuh", "tc_host.h", "sm100.cuh",
+               "decode_simt.cu", "common.cuh"):
         p = os.path.join(ROOT, "paper_2607_24331_gb300", "csrc", fn)
         if os.path.exists(p):
             txt = open(p).read()
@@ -70,8 +71,8 @@ def kernel_source_sha():
 
 
 def profiled_traffic(cfg):
-    """DRAM bytes per call of the attention kernels (factor preparation, scores, absorption) from the
-    committed ncu summary, if it was taken on the current sources."""
+    """DRAM bytes of one whole decode-step call (every kernel of it) from the committed ncu summary,
+    if it was taken on the current kernel sources (their hash is stored beside the bytes)."""
     p = os.path.join(ROOT, "profiles", "decode_main_traffic.json")
     if not os.path.exists(p):
         return None
@@ -355,10 +356,11 @@ def time_decode_steps(w, steps, warmup, dev, flush):
     stream = torch.cuda.current_stream(dev)
 
     def step():
+        st = torch.cuda.current_stream(dev)  # the capture stream while a graph is captured
         for buf, A_k, A_v, x, rows, wss, ws_s in layers:
             dck.check(dck.dck_decode_step(buf.layer, x, A_k, A_v, rows, buf.q, buf.kcache, buf.vcache, buf.n_rows,
                                           buf.B_k, buf.B_v, buf.seq_start, buf.seq_len, B, spec.rope_theta,
-                                          buf.out, wss, ws_s, stream), "decode step")
+                                          buf.out, wss, ws_s, st), "decode step")
 
     for _ in range(warmup):
         flush.fill_(1)

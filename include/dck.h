@@ -151,6 +151,47 @@ dck_status dck_decode_attention(const dck_layer_desc* desc, const void* q,
                                 void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * Prefill attention: many new tokens per sequence, each attending causally to
+ * its prefix, over the same latent caches (Sec. III-A x W ~ z R, Sec. III-C
+ * grouped key factors, Sec. III-D value factor; keys and values are rebuilt
+ * as for decode, once per cache row for all of a sequence's queries).  The
+ * paper describes neither prefill nor a causal mask; the library's reading:
+ * the Q_b new tokens of sequence b are the LAST Q_b rows of its cache (their
+ * latents appended before the call), query i (0 <= i < Q_b) sits at position
+ * p_i = L_b - Q_b + i, rotated there, and attends to the keys at positions
+ * 0 .. p_i:
+ *   o_ij = sum_{t <= p_i} softmax_t(<q_ij', k_t'> / sqrt(d)) v_t B_v[:, h*d:(h+1)*d]
+ * with k_t', q_ij', h and the RoPE convention of the decode formula above.
+ *   q            [B, q_max, Hq, d] queries before RoPE; row i of sequence b is
+ *                its i-th new token for i < Q_b (later rows are ignored)
+ *   d_q_len      device int32 [B]: Q_b, 0 <= Q_b <= min(L_b, q_max); Q_b = 0
+ *                writes nothing for sequence b
+ *   q_max        the second dimension of q and out, 1 .. 2^24
+ *   max_seq_len  an upper bound on every L_b, 1 .. 2^24 (sizes the launch)
+ *   kcache .. d_seq_len, rope_theta: as for dck_decode_attention
+ *   out          [B, q_max, Hq, d]; rows i < Q_b of each sequence written
+ *   workspace    at least dck_prefill_workspace_size(desc, n_rows) bytes,
+ *                256-byte aligned: the rebuilt keys (after RoPE) and values,
+ *                [n_rows][Hkv][d] bf16 each, written and then read by the call
+ * bf16 only, head_dim 128, Hq / Hkv in {1, 2, 4, 8}, at most 16 key groups
+ * (DCK_ERR_UNSUPPORTED otherwise; the workspace size query returns 0).  q
+ * and out must be 16-byte aligned; n_rows < 2^31 - 256.  Accumulation is
+ * fp32 in the tensor cores' accumulators; probabilities are rounded to bf16
+ * before the value product and the softmax denominator sums the rounded
+ * values.  A sequence with Q_b < 0, Q_b > L_b, Q_b > q_max, L_b > max_seq_len
+ * or rows outside the cache is recorded as a device error (DCK_ERR_INVALID
+ * from dck_last_device_error) and all q_max of its output rows are zero.
+ * Two launches on `stream`: the reconstruction, then the attention.
+ */
+size_t dck_prefill_workspace_size(const dck_layer_desc* desc, int64_t n_rows);
+dck_status dck_prefill_attention(const dck_layer_desc* desc, const void* q, const int32_t* d_q_len,
+                                 int32_t q_max, const void* kcache, const void* vcache, int64_t n_rows,
+                                 const void* B_k, const void* B_v, const int64_t* d_seq_start,
+                                 const int32_t* d_seq_len, int32_t batch, int32_t max_seq_len,
+                                 float rope_theta, void* out, void* workspace, size_t ws_bytes,
+                                 void* stream);
+
+/*
  * One decode step of a layer: the latent append of the batch's new tokens
  * (Sec. III-A z = x L) followed by decode attention over the caches that now
  * hold them (the formula at the top of this file).

@@ -14,6 +14,7 @@ constexpr int kMaxGroups = 128;
 constexpr int kMaxQPerKv = 8;     // query heads per KV head handled by the kernels
 constexpr int kMaxRankV = 2048;
 constexpr int kMaxBatch = 4096;
+constexpr int kMaxPrefillLen = 1 << 24;  // bound on a prefill call's q_max and max_seq_len
 constexpr int kTile = 128;        // tokens per work tile (one UMMA M block)
 
 // Device error word values (bit flags).

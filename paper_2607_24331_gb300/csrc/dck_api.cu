@@ -20,6 +20,12 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, const Tc
 bool tc_step_append_supports(const LayerTable& lt, int D, int batch);
 bool tc_append_supports(int D, int Rk, int rv, int dtype);
 size_t tc_append_workspace(int n_tok, int Rk, int rv);
+bool tc_prefill_supports(const LayerTable& lt, int dtype);
+size_t tc_prefill_workspace(const LayerTable& lt, int64_t n_rows);
+cudaError_t launch_prefill_tc(const LayerTable& lt, const void* q, const int32_t* q_len, int qmax, const void* kc,
+                              const void* vc, int64_t n_rows, const void* Bk, const void* Bv,
+                              const int64_t* seq_start, const int32_t* seq_len, int B, int max_len, float theta,
+                              void* out, void* ws, int* err, LaunchHook* hook, cudaStream_t s);
 cudaError_t launch_bounded_wait_selftest(long long limit_cycles, int* err, cudaStream_t s);
 cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, const void* A_v, int Rk, int rv,
                              const int64_t* rows, void* kc, void* vc, int64_t n_rows, void* ws, size_t ws_bytes,
@@ -210,6 +216,40 @@ dck_status decode_precheck(const dck_layer_desc* desc, const void* q, const void
 }  // namespace dck
 
 extern "C" {
+
+size_t dck_prefill_workspace_size(const dck_layer_desc* desc, int64_t n_rows) {
+  if (check_desc(desc) != DCK_OK || n_rows < 0) return 0;
+  const LayerTable lt = make_table(desc);
+  if (!tc_prefill_supports(lt, desc->dtype)) return 0;
+  return tc_prefill_workspace(lt, n_rows);
+}
+
+dck_status dck_prefill_attention(const dck_layer_desc* desc, const void* q, const int32_t* d_q_len, int32_t q_max,
+                                 const void* kcache, const void* vcache, int64_t n_rows, const void* B_k,
+                                 const void* B_v, const int64_t* d_seq_start, const int32_t* d_seq_len,
+                                 int32_t batch, int32_t max_seq_len, float rope_theta, void* out, void* workspace,
+                                 size_t ws_bytes, void* stream) {
+  t_last_launches = 0;
+  dck_status st =
+      decode_precheck(desc, q, kcache, vcache, n_rows, B_k, B_v, d_seq_start, d_seq_len, batch, rope_theta, out);
+  if (st != DCK_OK) return st;
+  if (q_max < 1 || q_max > kMaxPrefillLen || max_seq_len < 1 || max_seq_len > kMaxPrefillLen) return DCK_ERR_INVALID;
+  if (batch == 0) return DCK_OK;
+  if (!d_q_len || !aligned(q, 16) || !aligned(out, 16)) return DCK_ERR_INVALID;
+  const LayerTable lt = make_table(desc);
+  if (!tc_prefill_supports(lt, desc->dtype) || n_rows >= (int64_t(1) << 31) - 256) return DCK_ERR_UNSUPPORTED;
+  if (!workspace || ws_bytes < tc_prefill_workspace(lt, n_rows) || !aligned(workspace, 256)) return DCK_ERR_WORKSPACE;
+  int* err = nullptr;
+  if (!device_state(&err, nullptr)) return DCK_ERR_CUDA;
+  LaunchHook hook;
+  hook.ev = t_events;
+  hook.n_ev = t_n_events;
+  const cudaError_t e = launch_prefill_tc(lt, q, d_q_len, q_max, kcache, vcache, n_rows, B_k, B_v, d_seq_start,
+                                          d_seq_len, batch, max_seq_len, rope_theta, out, workspace, err, &hook,
+                                          static_cast<cudaStream_t>(stream));
+  t_last_launches = hook.count;
+  return e == cudaSuccess ? DCK_OK : DCK_ERR_CUDA;
+}
 
 }  // extern "C"
 

@@ -29,6 +29,7 @@ EXPORTED = (
     "dck_decode_workspace_size", "dck_decode_attention", "dck_last_device_error", "dck_set_decode_kernel",
     "dck_last_launch_count", "dck_synth_gaussian", "dck_set_timing_events", "dck_decode_attention_noalloc",
     "dck_selftest_bounded_wait", "dck_decode_step", "dck_decode_step_workspace_size",
+    "dck_prefill_workspace_size", "dck_prefill_attention",
 )
 
 
@@ -79,6 +80,10 @@ def lib() -> ctypes.CDLL:
     L.dck_decode_workspace_size.argtypes = [D, I32, I64]
     L.dck_decode_attention.restype = I32
     L.dck_decode_attention.argtypes = [D, P, P, P, I64, P, P, P, P, I32, F32, P, P, SZ, P]
+    L.dck_prefill_workspace_size.restype = SZ
+    L.dck_prefill_workspace_size.argtypes = [D, I64]
+    L.dck_prefill_attention.restype = I32
+    L.dck_prefill_attention.argtypes = [D, P, P, I32, P, P, I64, P, P, P, P, I32, I32, F32, P, P, SZ, P]
     L.dck_decode_step_workspace_size.restype = SZ
     L.dck_decode_step_workspace_size.argtypes = [D, I32, I64]
     L.dck_decode_step.restype = I32
@@ -182,6 +187,19 @@ def dck_decode_step(layer: Layer, x, A_k, A_v, rows, q, kcache, vcache, n_rows: 
                                  _ptr(vcache), int(n_rows), _ptr(B_k), _ptr(B_v), _ptr(seq_start), _ptr(seq_len),
                                  int(batch), float(rope_theta), _ptr(out), _ptr(workspace), int(ws_bytes),
                                  _stream(stream))
+
+
+def dck_prefill_workspace_size(layer: Layer, n_rows: int) -> int:
+    return lib().dck_prefill_workspace_size(layer.ref, int(n_rows))
+
+
+def dck_prefill_attention(layer: Layer, q, q_len, q_max: int, kcache, vcache, n_rows: int, B_k, B_v, seq_start,
+                          seq_len, batch: int, max_seq_len: int, rope_theta: float, out, workspace, ws_bytes: int,
+                          stream=None) -> int:
+    return lib().dck_prefill_attention(layer.ref, _ptr(q), _ptr(q_len), int(q_max), _ptr(kcache), _ptr(vcache),
+                                       int(n_rows), _ptr(B_k), _ptr(B_v), _ptr(seq_start), _ptr(seq_len), int(batch),
+                                       int(max_seq_len), float(rope_theta), _ptr(out), _ptr(workspace),
+                                       int(ws_bytes), _stream(stream))
 
 
 def dck_decode_attention_noalloc(layer: Layer, q, kcache, vcache, n_rows: int, B_k, B_v, seq_start, seq_len,

@@ -49,7 +49,7 @@ MIX_C2 = 0x94D049BB133111EB
 # 64-bit key, so these ids live here alone.
 TID = {
     "q": 1, "kcache": 2, "vcache": 3, "B_k": 4, "B_v": 5, "x": 6,
-    "A_k": 7, "A_v": 8, "perm": 9, "lens": 10, "x_step": 11,
+    "A_k": 7, "A_v": 8, "perm": 9, "lens": 10, "x_step": 11, "q_prefill": 12,
 }
 
 
@@ -394,6 +394,13 @@ def make_decode_inputs(spec: LayerSpec, seq_lens: Sequence[int], seed: int = 0, 
     vc = gaussian(stream_key(seed, layer, TID["vcache"]), (n_rows, spec.rank_v), 1.0, spec.dtype)
     return DecodeInputs(spec, q, kc, vc, make_bk(spec, seed, layer), make_bv(spec, seed, layer),
                         seq_starts(lens), lens)
+
+
+def make_prefill_q(spec: LayerSpec, batch: int, q_max: int, seed: int = 0, layer: int = 0,
+                   q_std: float = 1.0) -> np.ndarray:
+    """Prefill queries [B, q_max, Hq, d] before RoPE, ~ N(0, q_std^2), storage dtype."""
+    return gaussian(stream_key(seed, layer, TID["q_prefill"]), (batch, q_max, spec.n_q_heads, spec.head_dim),
+                    q_std, spec.dtype)
 
 
 def cache_rows(spec: LayerSpec, seed: int, layer: int, which: str, row0: int, n: int) -> np.ndarray:
