@@ -496,6 +496,44 @@ def run_sweep(args):
 
 
 # ---------------------------------------------------------------------------
+# --calls: a plain driver for profilers (no timing, no JSON line)
+# ---------------------------------------------------------------------------
+
+def run_calls(args):
+    """N decode-step calls (latent append + decode attention) of the first layer of the workload, L2
+    flushed before each, then a check of the device error word.  ncu captures in profiles/ use it with
+    `-s` to skip the first calls' kernels."""
+    import torch
+    from paper_2607_24331_gb300 import dck, device
+    from paper_2607_24331_gb300 import synth as S
+    dev = torch.device("cuda", 0)
+    w = S.workload(args.config, args.batch)
+    spec = w.layer
+    B = w.batch
+    dt = device.TORCH_DTYPE[spec.dtype]
+    buf = device.DecodeBuffers(spec, w.seq_lens, device=dev).synth(seed=w.seed, layer=0)
+    A_k = torch.empty((spec.hidden, spec.rank_k), dtype=dt, device=dev)
+    A_v = torch.empty((spec.hidden, spec.rank_v), dtype=dt, device=dev)
+    device.synth_fill(A_k, S.stream_key(w.seed, 0, S.TID["A_k"]), 1.0 / math.sqrt(spec.hidden))
+    device.synth_fill(A_v, S.stream_key(w.seed, 0, S.TID["A_v"]), 1.0 / math.sqrt(spec.hidden))
+    x = torch.empty((B, spec.hidden), dtype=dt, device=dev)
+    device.synth_fill(x, S.stream_key(w.seed, 0, S.TID["x_step"]), 1.0)
+    rows = (buf.seq_start + buf.seq_len.to(torch.int64) - 1).contiguous()
+    ws_s = dck.dck_decode_step_workspace_size(buf.layer, B, buf.n_rows)
+    wss = torch.empty(max(ws_s, 256), dtype=torch.uint8, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    for _ in range(args.calls):
+        flush.fill_(1)
+        dck.check(dck.dck_decode_step(buf.layer, x, A_k, A_v, rows, buf.q, buf.kcache, buf.vcache, buf.n_rows,
+                                      buf.B_k, buf.B_v, buf.seq_start, buf.seq_len, B, spec.rope_theta, buf.out,
+                                      wss, ws_s), "decode step")
+    torch.cuda.synchronize()
+    if dck.dck_last_device_error() != dck.DCK_OK:
+        raise SystemExit("device error word set")
+    print(f"{args.calls} decode-step calls of {w.name}: ok", flush=True)
+
+
+# ---------------------------------------------------------------------------
 # the GPU arm
 # ---------------------------------------------------------------------------
 
@@ -511,8 +549,13 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--sweep", action="store_true",
                     help="measurement matrix (context lengths, workloads, 32-layer batch sweep, prefill append)")
+    ap.add_argument("--calls", type=int, default=0,
+                    help="profiling driver: this many plain decode-step calls, no timing and no JSON line")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    if args.calls > 0:
+        run_calls(args)
+        return
 
     if args.impl == "reference":
         run_reference(args)

@@ -40,6 +40,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kMaxSplit = 8;    // CTAs per cluster (r_v split), portable cluster size
 constexpr int kMaxRows = 16;    // (sequence, query head) rows per cluster
+constexpr int kMergeBatch = 16; // partial loads of a row in flight together
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)),
@@ -149,7 +150,7 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   // Partials of sequence b: the items whose main tiles (the first NTm, split
   // evenly in whole tiles) cover b's; on the tensor-core path also the extra
   // pair tiles of b (x >= NTm), two slots (halves) per item and per extra tile.
-  const int NTm = pairs && NT / n_it < kFineSplitBelow ? NT / n_it * n_it : NT;
+  const int NTm = main_tiles(NT, n_it, pairs);
   for (int c = threadIdx.x; c <= n_it; c += kThreads) ibeg[c] = item_begin(c, NTm, n_it);
   if (threadIdx.x < nrow) {
     const int b = b0 + threadIdx.x / qpg;
@@ -241,34 +242,26 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
     const float* wrow = pw + (size_t)i * cap;
     const int* srow = ps + (size_t)i * cap;
     float4 acc0 = make_float4(0.f, 0.f, 0.f, 0.f), acc1 = acc0;
-    int q = 0;
-    for (; q + 8 <= n; q += 8) {
-      float4 v[8];
+    // batches of kMergeBatch partials, every load of a batch in flight before
+    // the first is used (a row has up to a few tens of partials: one or two
+    // L2 round trips per row instead of one per partial)
+    for (int q0 = 0; q0 < n; q0 += kMergeBatch) {
+      float4 v[kMergeBatch];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int sl = srow[q + u];
-        v[u] = sl >= 0 ? reinterpret_cast<const float4*>(a.part_u + ((int64_t)sl * Hq + j) * rv + r0)[r4]
+      for (int u = 0; u < kMergeBatch; ++u) {
+        const int sl = q0 + u < n ? srow[q0 + u] : -1;
+        v[u] = sl >= 0 ? __ldcg(reinterpret_cast<const float4*>(a.part_u + ((int64_t)sl * Hq + j) * rv + r0) + r4)
                        : make_float4(0.f, 0.f, 0.f, 0.f);
       }
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
+      for (int u = 0; u < kMergeBatch; ++u) {
         float4& ac = (u & 1) ? acc1 : acc0;
-        const float wq = wrow[q + u];
+        const float wq = q0 + u < n ? wrow[q0 + u] : 0.f;
         ac.x = fmaf(wq, v[u].x, ac.x);
         ac.y = fmaf(wq, v[u].y, ac.y);
         ac.z = fmaf(wq, v[u].z, ac.z);
         ac.w = fmaf(wq, v[u].w, ac.w);
       }
-    }
-    for (; q < n; ++q) {
-      const int sl = srow[q];
-      if (sl < 0) continue;
-      const float4 v = reinterpret_cast<const float4*>(a.part_u + ((int64_t)sl * Hq + j) * rv + r0)[r4];
-      const float wq = wrow[q];
-      acc0.x = fmaf(wq, v.x, acc0.x);
-      acc0.y = fmaf(wq, v.y, acc0.y);
-      acc0.z = fmaf(wq, v.z, acc0.z);
-      acc0.w = fmaf(wq, v.w, acc0.w);
     }
     reinterpret_cast<float4*>(su + (size_t)i * ldu)[r4] =
         make_float4(acc0.x + acc1.x, acc0.y + acc1.y, acc0.z + acc1.z, acc0.w + acc1.w);
