@@ -197,10 +197,42 @@ def host_cores():
         return os.cpu_count() or 1
 
 
-def cpu_baseline(w, budget_s=12.0):
+def cpu_baseline(w, budget_s=12.0, config=None, batch=None):
     pairs, secs, desc = oracle_sample_seconds(w, budget_s)
     tok_s = (pairs / w.layer.n_q_heads) / secs / w.n_layers
-    return {"value": tok_s, "unit": UNIT, "cores": host_cores(), "kind": "oracle", "sample": desc}
+    out = {"value": tok_s, "unit": UNIT, "cores": host_cores(), "kind": "oracle", "sample": desc}
+    if config is not None:
+        one = oracle_one_core(config, batch, max(1.0, budget_s / 4))
+        if one:
+            out["single_core"] = one
+    return out
+
+
+def oracle_one_core(config, batch, budget_s):
+    """The same oracle timing on one host core: a child process pinned to one CPU with its BLAS and
+    OpenMP pools at one thread (the pools size themselves at import, hence the separate process)."""
+    env = dict(os.environ)
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
+        env[k] = "1"
+    cmd = [sys.executable, os.path.abspath(__file__), "--oracle-one-core", "--config", str(config),
+           "--cpu-budget", str(budget_s)] + (["--batch", str(batch)] if batch else [])
+    try:
+        cpu = sorted(os.sched_getaffinity(0))[0]
+        r = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=max(60.0, 8 * budget_s),
+                           preexec_fn=lambda: os.sched_setaffinity(0, {cpu}))
+        return json.loads(r.stdout.strip().splitlines()[-1]) if r.returncode == 0 else None
+    except Exception:
+        return None
+
+
+def run_oracle_one_core(args):
+    """Child side of oracle_one_core: prints {"value", "unit", "cores", "sample"}."""
+    from paper_2607_24331_gb300 import synth as S
+    w = S.workload(args.config, args.batch)
+    pairs, secs, desc = oracle_sample_seconds(w, args.cpu_budget)
+    cores = host_cores()
+    print(json.dumps({"value": (pairs / w.layer.n_q_heads) / secs / w.n_layers, "unit": UNIT, "cores": cores,
+                      "sample": desc.replace("BLAS threads = host cores", "one core, BLAS threads = 1")}), flush=True)
 
 
 def run_reference(args):
@@ -451,6 +483,54 @@ def time_prefill_append(w, steps, warmup, dev, flush):
     return statistics.median(ms), bytes_, flops
 
 
+def time_prefill_attention(spec, B, L, steps, warmup, dev, flush, seed=0):
+    """Prefill attention (dck_prefill_attention) of B sequences whose whole L-token prompt is new
+    (Q = L): CUDA events around each call, L2 flushed between calls.  Returns the median ms, the
+    algorithmic bytes and the tensor flops of one call."""
+    import torch
+    from paper_2607_24331_gb300 import dck, device
+    from paper_2607_24331_gb300 import synth as S
+    dt = device.TORCH_DTYPE[spec.dtype]
+    buf = device.DecodeBuffers(spec, (L,) * B, device=dev).synth(seed=seed)
+    q = torch.empty((B, L, spec.n_q_heads, spec.head_dim), dtype=dt, device=dev)
+    device.synth_fill(q, S.stream_key(seed, 0, S.TID["q_prefill"]), 1.0)
+    ql = torch.full((B,), L, dtype=torch.int32, device=dev)
+    out = torch.empty_like(q)
+    wsb = dck.dck_prefill_workspace_size(buf.layer, buf.n_rows)
+    ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def call():
+        dck.check(dck.dck_prefill_attention(buf.layer, q, ql, L, buf.kcache, buf.vcache, buf.n_rows, buf.B_k,
+                                            buf.B_v, buf.seq_start, buf.seq_len, B, L, spec.rope_theta, out, ws,
+                                            wsb, stream), "prefill attention")
+
+    for _ in range(warmup):
+        flush.fill_(1)
+        call()
+    torch.cuda.synchronize()
+    assert dck.dck_last_device_error(stream) == dck.DCK_OK
+    ms = []
+    for k in range(steps):
+        flush.fill_(k & 0xFF)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        call()
+        e1.record(stream)
+        e1.synchronize()
+        ms.append(e0.elapsed_time(e1))
+    d, el = spec.head_dim, 2
+    n = B * L
+    recon = 2 * n * d * (sum(r * len(g) for g, r in zip(spec.groups, spec.ranks)) + spec.rank_v * spec.n_kv_heads)
+    pairs = B * L * (L + 1) // 2                      # causal (query, key) pairs per head
+    attn = 2 * 2 * pairs * d * spec.n_q_heads          # S = Q K^T and O = P V
+    bytes_ = (n * (spec.rank_k + spec.rank_v) + spec.bk_offsets()[-1] + spec.rank_v * spec.n_kv_heads * d
+              + 2 * n * spec.n_q_heads * d) * el
+    del buf, q, out, ws
+    torch.cuda.empty_cache()
+    return statistics.median(ms), bytes_, recon + attn
+
+
 def run_sweep(args):
     import torch
     from paper_2607_24331_gb300 import synth as S
@@ -486,6 +566,16 @@ def run_sweep(args):
     for b in (1, 8, 32, 64):               # the 32-layer step vs batch
         w = S.workload(4, b)
         line("32-layer step", w, *time_decode_steps(w, 3, 3, dev, flush))
+    for cfg, B, L in ((1, 2, 4096), (2, 1, 8192), (3, 1, 8192)):   # prefill attention, whole prompt new
+        spec = S.workload(cfg).layer
+        ms, by, fl = time_prefill_attention(spec, B, L, steps, warmup, dev, flush)
+        name = S.workload(cfg).name.split(" B")[0]
+        out["sweep"].append({"kind": "prefill attention", "workload": f"{name}: prefill of B{B} x {L} new tokens",
+                             "us": 1e3 * ms, "prompt_tokens_per_s": B * L / (ms / 1e3),
+                             "tensor_tflops": fl / (ms / 1e3) / 1e12,
+                             "tensor_frac_of_measured": fl / (ms / 1e3) / 1e12 / peaks["bf16_tflops"],
+                             "roofline_us": 1e6 * max(by / (peaks["hbm_gbs"] * 1e9), fl / (peaks["bf16_tflops"] * 1e12))})
+        print(json.dumps(out["sweep"][-1]), file=sys.stderr, flush=True)
     w3 = S.workload(3)
     ms, by, fl = time_prefill_append(w3, steps, warmup, dev, flush)
     out["sweep"].append({"kind": "prefill append", "workload": f"{w3.name}: latent append of 2 x {w3.append_tokens} tokens",
@@ -549,10 +639,14 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--sweep", action="store_true",
                     help="measurement matrix (context lengths, workloads, 32-layer batch sweep, prefill append)")
+    ap.add_argument("--oracle-one-core", action="store_true", help=argparse.SUPPRESS)
     ap.add_argument("--calls", type=int, default=0,
                     help="profiling driver: this many plain decode-step calls, no timing and no JSON line")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    if args.oracle_one_core:
+        run_oracle_one_core(args)
+        return
     if args.calls > 0:
         run_calls(args)
         return
@@ -738,7 +832,7 @@ def main():
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": gpu_launches}
     if rank == 0 and world == 1:
-        line["cpu_baseline"] = cpu_baseline(w, args.cpu_budget)
+        line["cpu_baseline"] = cpu_baseline(w, args.cpu_budget, args.config, args.batch)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
