@@ -94,7 +94,8 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
 
   // shared layout: B_v rows [rr][ldb] T | u rows [kMaxRows][rr + 4] | received partial o [split][kMaxRows * D / split]
   // | 1/l | per row: partial weights [kMaxRows][cap] f32, sums [kMaxRows][cap] f32, slots [kMaxRows][cap] i32,
-  // partial counts [kMaxRows] | row slot ranges [kMaxRows][4] | prefix [B + 1] | item starts [n_items + 1]
+  // partial counts [kMaxRows] | row slot ranges [kMaxRows][4] | row 128-token tiles [kMaxRows] | prefix [B + 1]
+  // | item starts [n_items + 1]
   const int cap = 2 * a.n_items;  // partials a row can have, on either work plan
   T* sbv = reinterpret_cast<T*>(smem_c);
   float* su = reinterpret_cast<float*>(smem_c + (size_t)rr * ldb<T, D>() * sizeof(T));
@@ -106,7 +107,8 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   int* ps = reinterpret_cast<int*>(pl + (size_t)kMaxRows * cap);
   int* pn = ps + (size_t)kMaxRows * cap;
   int* rc = pn + kMaxRows;
-  int* prefix = rc + 4 * kMaxRows;
+  int* rn128 = rc + 4 * kMaxRows;
+  int* prefix = rn128 + kMaxRows;
   int* ibeg = prefix + B + 1;
 
   // stage this CTA's B_v rows (all copies in flight at once)
@@ -157,6 +159,7 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
     const int me = min(prefix[b + 1], NTm);  // end of b's main tiles
     const bool any = me > prefix[b];
     int* r = rc + 4 * threadIdx.x;
+    rn128[threadIdx.x] = (valid_len(a.seq_len, a.seq_start, b, a.n_rows) + kTile - 1) / kTile;
     r[0] = any ? item_of_tile(prefix[b], NTm, n_it) : 0;           // first main item
     r[1] = any ? item_of_tile(me - 1, NTm, n_it) - r[0] + 1 : 0;  // main items
     r[2] = max(prefix[b], NTm) - NTm;                              // first extra tile
@@ -169,68 +172,63 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   // preceding grid is.
   asm volatile("griddepcontrol.wait;" ::: "memory");
 
-  // (1) every row's partials: slot, reference max m (log2 units) and sum l of
-  // each live one; (2) per row M = max m, weights 2^(m - M), 1/l; (3) this
-  // CTA's rows of u as the weighted sum, all of a row's loads independent.
-  for (int idx = threadIdx.x; idx < nrow * cap; idx += kThreads) {
-    const int i = idx / cap, q = idx % cap;
-    const int b = b0 + i / qpg, j = h * qpg + i % qpg;
-    const int c0 = rc[4 * i], nm = rc[4 * i + 1], e0 = rc[4 * i + 2];
-    const int nps = pairs ? 2 : 1;  // slots per item or extra tile
-    const int ns = nps * (nm + rc[4 * i + 3]);
-    if (q >= ns) continue;
-    const int k = q / nps, hh = q % nps;
-    bool live;
-    int64_t slot;
-    if (k < nm) {  // item c0 + k
-      const int c = c0 + k;
-      live = ibeg[c] != ibeg[c + 1];
-      if (pairs) {
-        const int n128 = (valid_len(a.seq_len, a.seq_start, b, a.n_rows) + kTile - 1) / kTile;
-        const int i0 = max(ibeg[c], prefix[b]) - prefix[b];  // b's first pair tile in the item
-        live = live && 2 * i0 + hh < n128;
-        slot = tc::pair_slot(c, b, hh);
-      } else {
-        slot = (int64_t)c + b;
-      }
-    } else {  // extra pair tile e (tensor-core path only)
-      const int n128 = (valid_len(a.seq_len, a.seq_start, b, a.n_rows) + kTile - 1) / kTile;
-      const int e = e0 + k - nm;
-      live = 2 * (NTm + e - prefix[b]) + hh < n128;
-      slot = tc::pair_xslot(n_it, B, e, hh);
-    }
-    float m = -INFINITY, l = 0.f;
-    if (live) {
-      const float2 ml = reinterpret_cast<const float2*>(a.part_ml)[slot * Hq + j];
-      m = ml.x;
-      l = ml.y;
-    }
-    pw[(size_t)i * cap + q] = m;
-    pl[(size_t)i * cap + q] = l;
-    ps[(size_t)i * cap + q] = live ? (int)slot : -1;
-  }
-  if (threadIdx.x < nrow) {
-    const int i = threadIdx.x;
-    pn[i] = (pairs ? 2 : 1) * (rc[4 * i + 1] + rc[4 * i + 3]);
-  }
-  __syncthreads();
+  // (1) one warp per row: each live partial's slot, reference max m (log2
+  // units) and sum l, their loads all in flight together (a lane per
+  // partial); then M = max m, the weights 2^(m - M) and 1/l; (2) this CTA's
+  // rows of u as the weighted sum, all of a row's loads independent.
   {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int i = warp; i < nrow; i += kThreads / 32) {  // one warp per row
-      const int n = pn[i];
+    const int nps = pairs ? 2 : 1;  // slots per item or extra tile
+    for (int i = warp; i < nrow; i += kThreads / 32) {
+      const int b = b0 + i / qpg, j = h * qpg + i % qpg;
+      const int c0 = rc[4 * i], nm = rc[4 * i + 1], e0 = rc[4 * i + 2];
+      const int ns = nps * (nm + rc[4 * i + 3]);
+      const int n128 = rn128[i];
       float M = -INFINITY;
-      for (int q = lane; q < n; q += 32) M = fmaxf(M, pw[(size_t)i * cap + q]);
+      for (int q = lane; q < ns; q += 32) {
+        const int k = q / nps, hh = q % nps;
+        bool live;
+        int64_t slot;
+        if (k < nm) {  // item c0 + k
+          const int c = c0 + k;
+          live = ibeg[c] != ibeg[c + 1];
+          if (pairs) {
+            const int i0 = max(ibeg[c], prefix[b]) - prefix[b];  // b's first pair tile in the item
+            live = live && 2 * i0 + hh < n128;
+            slot = tc::pair_slot(c, b, hh);
+          } else {
+            slot = (int64_t)c + b;
+          }
+        } else {  // extra pair tile e (tensor-core path only)
+          const int e = e0 + k - nm;
+          live = 2 * (NTm + e - prefix[b]) + hh < n128;
+          slot = tc::pair_xslot(n_it, B, e, hh);
+        }
+        float m = -INFINITY, l = 0.f;
+        if (live) {
+          const float2 ml = reinterpret_cast<const float2*>(a.part_ml)[slot * Hq + j];
+          m = ml.x;
+          l = ml.y;
+        }
+        pw[(size_t)i * cap + q] = m;
+        pl[(size_t)i * cap + q] = l;
+        ps[(size_t)i * cap + q] = live ? (int)slot : -1;
+        M = fmaxf(M, m);
+      }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
       float l = 0.f;
-      for (int q = lane; q < n; q += 32) {
+      for (int q = lane; q < ns; q += 32) {  // entries this lane wrote itself
         const float wq = M == -INFINITY ? 0.f : exp2f(pw[(size_t)i * cap + q] - M);  // 0 for slots not live
         pw[(size_t)i * cap + q] = wq;
         l = fmaf(wq, pl[(size_t)i * cap + q], l);
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-      if (lane == 0) sinv[i] = l > 0.f ? 1.f / l : 0.f;
+      if (lane == 0) {
+        sinv[i] = l > 0.f ? 1.f / l : 0.f;
+        pn[i] = ns;
+      }
     }
   }
   __syncthreads();
@@ -276,6 +274,7 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int gid = lane >> 2, tig = lane & 3;
     float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+#pragma unroll 4
     for (int k0 = 0; k0 < rr; k0 += 8) {
       uint32_t af[4];
       af[0] = f32_to_tf32(su[(size_t)gid * ldu + k0 + tig]);
@@ -368,7 +367,7 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   const int cap = 2 * a.n_items;
   const size_t smem = (size_t)rr * ldb<T, D>() * sizeof(T) +
                       sizeof(float) * ((size_t)kMaxRows * (rr + 4) + kMaxRows * D + kMaxRows + 2 * (size_t)kMaxRows * cap) +
-                      sizeof(int) * ((size_t)kMaxRows * cap + kMaxRows + 4 * kMaxRows + a.B + 1 + a.n_items + 1);
+                      sizeof(int) * ((size_t)kMaxRows * cap + kMaxRows + 4 * kMaxRows + kMaxRows + a.B + 1 + a.n_items + 1);
   auto k = combine_kernel<T, D>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
