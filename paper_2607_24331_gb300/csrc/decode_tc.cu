@@ -100,7 +100,12 @@ constexpr int kMaxItems = 256;
 constexpr int kMaxUnits = 32;
 constexpr int kEpiThreads = 256;
 constexpr int kEpiWarps = kEpiThreads / 32;
-constexpr int kPrefetchAhead = 2;   // latent tiles prefetched toward L2 ahead of their loads
+// Latent tiles prefetched toward L2 ahead of their loads: two in query-folded
+// mode; none in key mode, whose TMA loads keep enough of the latent stream in
+// flight themselves and whose prefetches only competed with it (7B GQA layer,
+// 0 / 1 / 2 / 4 tiles ahead: 298 / 301 / 306 / 315 us per step)
+template <bool kFold>
+constexpr int prefetch_ahead() { return kFold ? 2 : 0; }
 constexpr float kRescaleThr = 8.f;  // log2 units: probabilities stay <= 256
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kKCols = 256;    // TMEM columns of one key accumulator
@@ -354,7 +359,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
       const uint64_t pol = policy_evict_first();
       SlotFifo ga;  // the latent ring
       bool ok = true;
-      // L2 prefetch of this half's latent rows, kPrefetchAhead tiles ahead of the
+      // L2 prefetch of this half's latent rows, prefetch_ahead() tiles ahead of the
       // loads (across segment boundaries): the TMA loads then find them in L2
       PairWalker pwalk[2] = {walk_m, walk_x};
       PSegment pseg;
@@ -372,7 +377,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
         const int64_t nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
         if (nr > 0) prefetch_l2(static_cast<const __nv_bfloat16*>(a.kc) + r0 * lt.Rk, (uint32_t)(nr * lt.Rk * 2));
       };
-      for (int q = 0; q < kPrefetchAhead; ++q) prefetch_next();
+      for (int q = 0; q < prefetch_ahead<kFold>(); ++q) prefetch_next();
       griddep_wait();  // the preparation launch may append the step's own latents
       for (int ph = 0; ph < 2 && ok; ++ph)
         for (PairWalker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
