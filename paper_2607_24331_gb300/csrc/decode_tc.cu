@@ -105,7 +105,7 @@ constexpr int kEpiWarps = kEpiThreads / 32;
 // flight themselves and whose prefetches only competed with it (7B GQA layer,
 // 0 / 1 / 2 / 4 tiles ahead: 298 / 301 / 306 / 315 us per step)
 template <bool kFold>
-constexpr int prefetch_ahead() { return kFold ? 2 : 0; }
+__host__ __device__ constexpr int prefetch_ahead() { return kFold ? 2 : 0; }
 constexpr float kRescaleThr = 8.f;  // log2 units: probabilities stay <= 256
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kKCols = 256;    // TMEM columns of one key accumulator
