@@ -41,6 +41,15 @@ constexpr int kRStages = 4;
 constexpr int kRASlot = 16384;         // latent piece [128 rows][<= 64] bf16
 constexpr int kRBSlot = 16384;         // factor piece [<= 64 ranks][128 cols] as two 64-column atoms
 constexpr int kMaxGroupsP = 16;
+constexpr float kTwoPiP = 6.28318530717958647692f;
+// 2^x on the special-function unit (relative error about 2^-22; results below
+// 2^-126 flush to zero): the probabilities are rounded to bf16 right after
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+constexpr float kInvTwoPiP = 0.15915494309189533577f;
 
 // ---------------------------------------------------------------------------
 // 1. reconstruction
@@ -69,6 +78,7 @@ struct RArgs {
 struct RSmem {
   uint8_t a[kRStages][kRASlot];
   uint8_t b[kRStages][kRBSlot];
+  float beta[kPD / 2], om32[kPD / 2];  // RoPE: (t0 w_i) mod 2 pi of the tile's first row, and w_i
   uint64_t full[kRStages], empty[kRStages], acc;
   uint32_t tmem_base;
   int abort_flag;
@@ -106,6 +116,13 @@ __global__ void __launch_bounds__(kRThreads, 1)
     mbar_init(&sm.acc, 1);
     sm.abort_flag = 0;
     fence_mbar_init();
+  }
+  // RoPE angle of row t0 + r and pair i: (t0 w_i reduced mod 2 pi in fp64, once
+  // per tile) + r w_i in fp32; the fp64 work stays off the per-row path
+  if (!is_v && tid < kPD / 2) {
+    const double ang = (double)t0 * ra.om[tid];
+    sm.beta[tid] = (float)(ang - 6.283185307179586 * floor(ang * 0.15915494309189535));
+    sm.om32[tid] = (float)ra.om[tid];
   }
   if (warp == 1) {
     tmem_alloc(&sm.tmem_base, 128);
@@ -169,10 +186,11 @@ __global__ void __launch_bounds__(kRThreads, 1)
         if (!is_v) {
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            // angle pos w_i reduced mod 2 pi in fp64, sine and cosine in fp32
-            const double ang = (double)pos * ra.om[cc + i];
+            // angle (t0 w_i mod 2 pi) + r w_i, reduced to [-pi, pi] in fp32
+            float ph = fmaf((float)r, sm.om32[cc + i], sm.beta[cc + i]);
+            ph = fmaf(-kTwoPiP, rintf(ph * kInvTwoPiP), ph);
             float sn, cs;
-            sincosf((float)(ang - 6.283185307179586 * rint(ang * 0.15915494309189535)), &sn, &cs);
+            sincosf(ph, &sn, &cs);
             const float xr = x[i] * cs - y[i] * sn, yr = x[i] * sn + y[i] * cs;
             x[i] = xr;
             y[i] = yr;
@@ -242,6 +260,7 @@ struct ASmemP {
   uint8_t v[2][2][kAtom];   // V^ ring [stage][d atom][128 keys][128 B] (TMA)
   uint8_t p[2][kAtom];      // P [key atom][128 rows][128 B], K-major, 128B-swizzled
   uint64_t kv_full[2], kv_empty[2], s_full[2], s_free[2], p_ready, o_ready, q_ready;
+  float qbeta[kPD / 2], om32[kPD / 2];  // RoPE: (p0 w_i) mod 2 pi of the tile's first query, and w_i
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -293,6 +312,13 @@ __global__ void __launch_bounds__(kAThreadsP, 1)
     mbar_init(&sm.q_ready, 4);
     sm.abort_flag = 0;
     fence_mbar_init();
+  }
+  // query RoPE angles: (p0 w_i reduced mod 2 pi in fp64, once per tile) + (row
+  // offset) w_i in fp32, p0 the position of the tile's first query
+  if (tid < kPD / 2) {
+    const double ang = (double)(L - Q + i0) * aa.om[tid];
+    sm.qbeta[tid] = (float)(ang - 6.283185307179586 * floor(ang * 0.15915494309189535));
+    sm.om32[tid] = (float)aa.om[tid];
   }
   if (warp == 1) {
     tmem_alloc(&sm.tmem_base, 512);
@@ -370,9 +396,11 @@ __global__ void __launch_bounds__(kAThreadsP, 1)
           float rx[2], ry[2];
 #pragma unroll
           for (int u = 0; u < 2; ++u) {
-            const double ang = (double)pos * aa.om[8 * cc + t + u];
+            const int pi = 8 * cc + t + u;
+            float ph = fmaf((float)(valid ? qi - i0 : 0), sm.om32[pi], sm.qbeta[pi]);
+            ph = fmaf(-kTwoPiP, rintf(ph * kInvTwoPiP), ph);
             float sn, cs;
-            sincosf((float)(ang - 6.283185307179586 * rint(ang * 0.15915494309189535)), &sn, &cs);
+            sincosf(ph, &sn, &cs);
             const float x = valid ? __bfloat162float(xh[t + u]) : 0.f, y = valid ? __bfloat162float(yh[t + u]) : 0.f;
             rx[u] = (x * cs - y * sn) * sc;
             ry[u] = (x * sn + y * cs) * sc;
@@ -396,20 +424,21 @@ __global__ void __launch_bounds__(kAThreadsP, 1)
       const uint32_t sb = tmem + lb + 128 * sl;
       const int kbase = kTile * kt;
       const int vis = valid ? min(pos - kbase + 1, kTile) : 0;  // visible keys of this tile: [0, vis)
-      // pass 1: the tile's max over visible keys
+      // the row's 128 scores in one TMEM round trip, then the tile's max over visible keys
+      float sv[4][32];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(sb + 32 * c, sv[c]);
+      tmem_wait_ld();
       float mt = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        float v[32];
-        tmem_ld32(sb + 32 * c, v);
-        tmem_wait_ld();
+      for (int c = 0; c < 4; ++c)
 #pragma unroll
         for (int i = 0; i < 32; ++i)
-          if (32 * c + i < vis) mt = fmaxf(mt, v[i]);
-      }
-      // PV of the previous tile must be done before P is overwritten and before O is rescaled
-      if (kt >= 1 && !(ok = wwait(&sm.o_ready, (kt - 1) & 1, abort_flag))) break;
-      tc_fence_after();
+          if (32 * c + i < vis) mt = fmaxf(mt, sv[c][i]);
+      // the S buffer has been read
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.s_free[sl]);
       // a new reference max for this row when the tile's max passes the old one by kThr;
       // O and l are rescaled where a reference existed.  The TMEM loads and stores are
       // warp-collective, so the whole warp runs them when any row rescales (factor 1
@@ -417,6 +446,9 @@ __global__ void __launch_bounds__(kAThreadsP, 1)
       const bool upd = mt != -INFINITY && (m == -INFINITY || mt > m + kThr);
       const bool resc = upd && m != -INFINITY;
       const float al = resc ? exp2f(m - mt) : 1.f;
+      // PV of the previous tile must be done before P is overwritten and before O is rescaled
+      if (kt >= 1 && !(ok = wwait(&sm.o_ready, (kt - 1) & 1, abort_flag))) break;
+      tc_fence_after();
       if (__any_sync(0xffffffffu, resc)) {
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
@@ -435,12 +467,10 @@ __global__ void __launch_bounds__(kAThreadsP, 1)
       }
       l *= al;
       if (upd) m = mt;
-      // pass 2: P = 2^(s - m) over visible keys (bf16, the row sum over the rounded values)
+      // P = 2^(s - m) over visible keys (bf16, the row sum over the rounded values)
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
-        float v[32];
-        tmem_ld32(sb + 32 * c, v);
-        tmem_wait_ld();
+        const float* v = sv[c];
 #pragma unroll
         for (int cc = 0; cc < 4; ++cc) {
           uint4 o;
@@ -448,8 +478,8 @@ __global__ void __launch_bounds__(kAThreadsP, 1)
 #pragma unroll
           for (int t = 0; t < 4; ++t) {
             const int k0 = 32 * c + 8 * cc + 2 * t;
-            const float p0 = k0 < vis ? exp2f(v[8 * cc + 2 * t] - m) : 0.f;
-            const float p1 = k0 + 1 < vis ? exp2f(v[8 * cc + 2 * t + 1] - m) : 0.f;
+            const float p0 = k0 < vis ? ex2_approx(v[8 * cc + 2 * t] - m) : 0.f;
+            const float p1 = k0 + 1 < vis ? ex2_approx(v[8 * cc + 2 * t + 1] - m) : 0.f;
             po[t] = __floats2bfloat162_rn(p0, p1);
             const float2 pr = __bfloat1622float2(po[t]);
             l += pr.x + pr.y;
@@ -457,9 +487,6 @@ __global__ void __launch_bounds__(kAThreadsP, 1)
           *reinterpret_cast<uint4*>(&sm.p[0][0] + swz_chunk(r, 4 * c + cc)) = o;
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.s_free[sl]);  // S buffer read
       // keys past the sequence in its last tile: exact zeros in V^ (P is zero there)
       if (kbase + r >= L) {
         uint4* z0 = reinterpret_cast<uint4*>(sm.v[sl][0] + r * 128);
@@ -512,6 +539,9 @@ __global__ void __launch_bounds__(kAThreadsP, 1)
 }
 
 }  // namespace
+
+static_assert(sizeof(RSmem) + 1024 <= 232448, "shared memory of the reconstruction kernel");
+static_assert(sizeof(ASmemP) + 1024 <= 232448, "shared memory of the prefill attention kernel");
 
 // ---------------------------------------------------------------------------
 // host
