@@ -185,6 +185,7 @@ struct Smem {
   double om64[kD / 2];
   float om32[kD / 2];
   float beta[kD / 2];
+  float qcs[kFold ? 1 : kD / 2], qsn[kFold ? 1 : kD / 2];  // key mode: RoPE of the query position
   // latent ring: one full/empty pair per group instance; factor rings: one
   // pair per unit (batch of items) of each MMA thread (see SlotFifo)
   uint64_t g_full[kFifoBars], g_empty[kFifoBars];
@@ -552,15 +553,19 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
       for (PairWalker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
         if (!kFold) {
           // rotated queries of this sequence at position L-1, scaled to log2 units
-          // (angle reduced mod 2 pi in fp64, sine and cosine in fp32)
-          const double Pq = (double)(seg.L - 1);
+          // (the 64 angles reduced mod 2 pi in fp64 once, sine and cosine in fp32;
+          // every query head uses them)
+          if (e < kD / 2) {
+            const double ang = (double)(seg.L - 1) * sm.om64[e];
+            sincosf((float)(ang - 6.283185307179586 * rint(ang * 0.15915494309189535)), &sm.qsn[e], &sm.qcs[e]);
+          }
+          EPI_SYNC();
+          if (!ok) break;
           const float qscale = kLog2e * rsqrtf((float)kD);
           const __nv_bfloat16* qb = static_cast<const __nv_bfloat16*>(a.q) + (int64_t)seg.b * Hq * kD;
           for (int i = e; i < Hq * (kD / 2); i += kEpiThreads) {
             const int j = i / (kD / 2), pi = i % (kD / 2);
-            const double ang = Pq * sm.om64[pi];
-            float sn, cs;
-            sincosf((float)(ang - 6.283185307179586 * rint(ang * 0.15915494309189535)), &sn, &cs);
+            const float sn = sm.qsn[pi], cs = sm.qcs[pi];
             const float x1v = __bfloat162float(qb[j * kD + pi]), x2v = __bfloat162float(qb[j * kD + pi + kD / 2]);
             sm.qr[j * kD + pi] = __float2bfloat16_rn((x1v * cs - x2v * sn) * qscale);
             sm.qr[j * kD + pi + kD / 2] = __float2bfloat16_rn((x1v * sn + x2v * cs) * qscale);
