@@ -747,8 +747,8 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
             uint32_t pk[8];
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
-              const __nv_bfloat162 pv = __floats2bfloat162_rn(own ? exp2f(sc[2 * k] - m_run) : 0.f,
-                                                              own ? exp2f(sc[2 * k + 1] - m_run) : 0.f);
+              const __nv_bfloat162 pv = __floats2bfloat162_rn(own ? ex2_approx(sc[2 * k] - m_run) : 0.f,
+                                                              own ? ex2_approx(sc[2 * k + 1] - m_run) : 0.f);
               const float2 pf = __bfloat1622float2(pv);
               l_part += pf.x + pf.y;
               pk[k] = *reinterpret_cast<const uint32_t*>(&pv);

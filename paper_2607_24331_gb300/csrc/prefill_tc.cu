@@ -42,13 +42,6 @@ constexpr int kRASlot = 16384;         // latent piece [128 rows][<= 64] bf16
 constexpr int kRBSlot = 16384;         // factor piece [<= 64 ranks][128 cols] as two 64-column atoms
 constexpr int kMaxGroupsP = 16;
 constexpr float kTwoPiP = 6.28318530717958647692f;
-// 2^x on the special-function unit (relative error about 2^-22; results below
-// 2^-126 flush to zero): the probabilities are rounded to bf16 right after
-__device__ __forceinline__ float ex2_approx(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
 constexpr float kInvTwoPiP = 0.15915494309189533577f;
 
 // ---------------------------------------------------------------------------
