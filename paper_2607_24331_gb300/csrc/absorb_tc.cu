@@ -19,9 +19,9 @@
 // each hand-off phase follows the MMA threads' own commits.  U = [r_v / 128 chunks][Hq_pad heads] fp32 accumulators, one TMEM
 // lane per r_v row of a chunk.
 //
-// Warps: 0 producer (P images by bulk copy, value chunks by TMA, next tile's
-// values prefetched toward L2), 1 and 6 MMA issuers (lane 0 of each; M = 128
-// r_v rows, N = Hq_pad, K = 16 tokens; 8 per chunk and tile), each taking half
+// Warps: 0 producer (P images by bulk copy, value chunks by TMA), 1 and 6 MMA
+// issuers (lane 0 of each; M = 128 r_v rows, N = Hq_pad, K = 16 tokens; 8 per
+// chunk and tile), each taking half
 // of a tile's r_v chunks from its own ring of value slots (a single thread's
 // MMA issue, commits and barrier tests took longer than the values took to
 // arrive); warp 1 owns TMEM.  2-5 epilogue (one TMEM lane quadrant each:
@@ -216,9 +216,8 @@ __global__ void __launch_bounds__(kAThreads, 1)
   if (warp == 0) {
     // ---- producer ------------------------------------------------------------
     // The value latents do not depend on the scores kernel, which may still be
-    // running (programmatic dependent launch): the first tile's rows are
-    // prefetched and its first chunks loaded before the wait for that kernel's
-    // probabilities and maxima.
+    // running (programmatic dependent launch): the first tile's first chunks
+    // are loaded before the wait for that kernel's probabilities and maxima.
     if (has_work) {
       const uint64_t pol = policy_evict_first();
       int v_cnt[2] = {0, 0}, p_cnt = 0;
@@ -226,30 +225,15 @@ __global__ void __launch_bounds__(kAThreads, 1)
       // reference maxima (lane = head) of the previous tile and, loaded a tile
       // ahead so that their latency hides behind the value loads, of this one
       float m_prev = 0.f, m_pf = 0.f;
-      // L2 prefetch of the value rows two tiles ahead of their loads, across
-      // segments (the first two at once)
-      AWalk pwalk = walk0;
-      ASeg pseg;
-      int pti = 0;
-      bool pvalid = false;
-      auto prefetch_next = [&]() {
-        if (lane != 0) return;
-        while (!pvalid || pti >= pseg.n) {
-          if (!pwalk.next(a, pl, pseg)) return;
-          pvalid = true;
-          pti = 0;
-        }
-        const int64_t r0 = pseg.row(pti++), nr = a.n_rows - r0 < kTile ? a.n_rows - r0 : (int64_t)kTile;
-        if (nr > 0) prefetch_l2(static_cast<const __nv_bfloat16*>(a.vc) + r0 * lt.rv, (uint32_t)(nr * lt.rv * 2));
-      };
-      prefetch_next();
-      prefetch_next();
+      // No L2 prefetch ahead of the loads: the rings keep 192 KB in flight per
+      // SM, which is enough for HBM's rate, and prefetches of later tiles issued
+      // by every CTA at once only queued ahead of the first tile's loads
+      // (clock64 timelines: the first MMAs started 8 us later with them).
       for (AWalk walk = walk0; ok && walk.next(a, pl, seg);) {
         for (int i = 0; i < seg.n && ok; ++i) {
           const int64_t x = seg.x(i);
           const int64_t yrow = seg.row(i);
           const int ca = seg.ca, cb = seg.cb;
-          prefetch_next();
           // chunks go to the two MMA threads' rings alternately (thread 0: [ca, cm),
           // thread 1: [cm, cb)), each chunk one slot filled by two boxes (lanes 0, 1)
           const int cm = chunk_mid(ca, cb), nch = cb - ca;

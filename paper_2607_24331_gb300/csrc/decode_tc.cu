@@ -245,7 +245,6 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
   const int hr = (int)cluster_ctarank();  // the half of every pair tile this CTA holds
   const bool leader = hr == 0;            // the even CTA issues the pair MMAs
   const int P = ta.n_pairs, pair = blockIdx.x >> 1;
-  griddep_launch();  // the absorption kernel may start streaming values as CTAs finish
 
   // ---- setup -------------------------------------------------------------
   if (tid == 0) {
@@ -350,6 +349,15 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
     return true;
   };
   const int64_t img_seq_rows = ta.fimg_seq_bytes >> 7;
+  // Programmatic dependent launch: every thread lets the absorption kernel
+  // launch only after it has seen the preparation kernel complete, so that
+  // the absorption's value loads ahead of its own grid-dependency wait find
+  // the rows a decode step appends.  The latent producer first moves its
+  // first tiles toward L2.
+  if (warp != 0) {
+    griddep_wait();
+    griddep_launch();
+  }
 
   if (warp == 0) {
     // ---- latent pieces (this CTA's 128 rows of each), issued as soon as their
@@ -380,6 +388,7 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
       };
       for (int q = 0; q < prefetch_ahead<kFold>(); ++q) prefetch_next();
       griddep_wait();  // the preparation launch may append the step's own latents
+      griddep_launch();
       for (int ph = 0; ph < 2 && ok; ++ph)
         for (PairWalker walk = ph ? walk_x : walk_m; ok && walk.next(a, seg);) {
           const int64_t img_row0 = kFold ? (int64_t)seg.b * img_seq_rows : 0;
@@ -410,13 +419,15 @@ __global__ void __launch_bounds__(Ring<kFold>::kThreads, 1)
           }
         }
       if (!ok && lane == 0) stop_peer();
+    } else {
+      griddep_wait();
+      griddep_launch();
     }
   } else if (warp == 10) {
     // ---- factor items: several TMA copies per instruction (query-folded
     // mode: the ring of MMA thread 0 only) --------------------------------------
     if (has_work) {
       const uint64_t pol = policy_evict_last();
-      griddep_wait();  // the images are written by the preparation kernel
       SlotFifo fw;         // the factor ring
       bool ok = true;
       for (int ph = 0; ph < 2 && ok; ++ph)
@@ -1377,7 +1388,7 @@ cudaError_t launch_decode_tc(const LayerTable& lt, const DecodeArgs& a, const Tc
   r.mglob = ta.mglob;
   r.max_tiles = ta.max_tiles;
   r.hq_pad = ta.hq_pad;
-  r.early_values = app == nullptr;
+  r.early_values = true;
   e = launch_absorb_tc(lt, a, r, s);
   return e != cudaSuccess ? e : hook_launched(a.hook, s);
 }

@@ -15,8 +15,9 @@ struct TcRegions {
   const float* mglob;    // [max_tiles][Hq]: reference max (log2 units) P of tile x was computed with
   int64_t max_tiles;
   int hq_pad;
-  bool early_values;     // value loads may start before the scores kernel completes (false when the
-                         // call's first launch also appends latents, which those loads could read)
+  bool early_values;     // value loads may start before the scores kernel completes (that kernel lets
+                         // the absorption launch only once the call's first launch, which may append
+                         // latents, is complete)
 };
 
 // A decode step's latent append fused into the decode call (dck_decode_step).
