@@ -54,6 +54,7 @@ constexpr int kVSlot = 32768;  // one r_v chunk: [2 halves][128 tokens][64 rv] b
 constexpr int kNVr = 3;        // value slots of each MMA thread's ring: six chunks in flight
 constexpr int kPSlot = 8192;   // P image of one tile (Hq_pad <= 32)
 constexpr int kNP = 2;
+constexpr int kEpiWarpsA = 4;  // warps 2-5: one per TMEM lane quadrant
 constexpr uint32_t kTmemCols = 512;
 
 struct AMaps {
@@ -165,10 +166,10 @@ __global__ void __launch_bounds__(kAThreads, 1)
       mbar_init(&sm.p_empty[i], 2);  // released by both MMA threads
     }
     mbar_init(&sm.drain, 2);
-    mbar_init(&sm.tile_ok, 4);
+    mbar_init(&sm.tile_ok, kEpiWarpsA);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sm.u_ready[i], 2);
-      mbar_init(&sm.u_free[i], 4);
+      mbar_init(&sm.u_free[i], kEpiWarpsA);
     }
     sm.abort_flag = 0;
     fence_mbar_init();
@@ -185,7 +186,9 @@ __global__ void __launch_bounds__(kAThreads, 1)
   pl.pr = blockIdx.x >> 1;
   pl.hh = blockIdx.x & 1;
   pl.nc = n_chunks;
+  DCK_AB_TRACE(3);
   const int NP = pair_tile_count(a, sm.s256, sm.s128);
+  DCK_AB_TRACE(4);
   const PSplit sp(NP, pl.P);
   pl.NPm = sp.NPm;
   const bool fits = sm.s128[kAThreads - 1] <= aa.max_tiles;  // else the scores kernel has reported the input
@@ -223,8 +226,10 @@ __global__ void __launch_bounds__(kAThreads, 1)
       int v_cnt[2] = {0, 0}, p_cnt = 0;
       bool ok = true, first = true;
       // reference maxima (lane = head) of the previous tile and, loaded a tile
-      // ahead so that their latency hides behind the value loads, of this one
+      // ahead (across segments) so that their latency hides behind the value
+      // loads, of this one
       float m_prev = 0.f, m_pf = 0.f;
+      bool have_pf = false;
       // No L2 prefetch ahead of the loads: the rings keep 192 KB in flight per
       // SM, which is enough for HBM's rate, and prefetches of later tiles issued
       // by every CTA at once only queued ahead of the first tile's loads
@@ -274,14 +279,17 @@ __global__ void __launch_bounds__(kAThreads, 1)
             // does any head's reference max rise at this tile?  (decided here, once,
             // for the MMA thread; the epilogue warps take the same decision)
             bool need = false;
-            float m_now;
-            if (i == 0) {
-              m_now = lane < Hq ? aa.mglob[x * Hq + lane] : 0.f;
-            } else {
-              m_now = m_pf;
-              need = __any_sync(0xffffffffu, m_now > m_prev);
+            const float m_now = have_pf ? m_pf : (lane < Hq ? aa.mglob[x * Hq + lane] : 0.f);
+            if (i > 0) need = __any_sync(0xffffffffu, m_now > m_prev);
+            have_pf = true;
+            if (i + 1 < seg.n) {
+              m_pf = lane < Hq ? aa.mglob[seg.x(i + 1) * Hq + lane] : 0.f;
+            } else {  // the next segment's first tile
+              AWalk nw = walk;
+              ASeg ns;
+              if (nw.next(a, pl, ns)) m_pf = lane < Hq ? aa.mglob[ns.x(0) * Hq + lane] : 0.f;
+              else have_pf = false;
             }
-            if (i + 1 < seg.n) m_pf = lane < Hq ? aa.mglob[seg.x(i + 1) * Hq + lane] : 0.f;
             m_prev = m_now;
             if (lane == 0) {
               const int sl = p_cnt % kNP;
@@ -441,6 +449,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.u_free[sgc % nub]);
+      DCK_AB_TRACE(23);
       ++sgc;
     }
   }

@@ -34,6 +34,10 @@
 
 namespace cg = cooperative_groups;
 
+#ifndef DCK_CB_TRACE
+#define DCK_CB_TRACE(code) ((void)0)
+#endif
+
 namespace dck {
 namespace {
 
@@ -91,6 +95,7 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   const int nrow = nb * qpg;
   const int rr = rv / split;            // rows of u / B_v owned by this CTA (a multiple of 4)
   const int r0 = rank * rr;
+  DCK_CB_TRACE(99);
 
   // shared layout: B_v rows [rr][ldb] T | u rows [kMaxRows][rr + 4] | received partial o [split][kMaxRows * D / split]
   // | 1/l | per row: partial weights [kMaxRows][cap] f32, sums [kMaxRows][cap] f32, slots [kMaxRows][cap] i32,
@@ -167,10 +172,12 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   }
   __syncthreads();
 
+  DCK_CB_TRACE(1);
   // Launched under programmatic dependent launch: everything above reads only the
   // call's inputs; the partials come from the kernels before, complete once the
   // preceding grid is.
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  DCK_CB_TRACE(2);
 
   // (1) one warp per row: each live partial's slot, reference max m (log2
   // units) and sum l, their loads all in flight together (a lane per
@@ -232,6 +239,7 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
     }
   }
   __syncthreads();
+  DCK_CB_TRACE(3);
   const int rr4 = rr / 4;
   for (int idx = threadIdx.x; idx < nrow * rr4; idx += kThreads) {
     const int i = idx / rr4, r4 = idx % rr4;
@@ -264,8 +272,10 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
     reinterpret_cast<float4*>(su + (size_t)i * ldu)[r4] =
         make_float4(acc0.x + acc1.x, acc0.y + acc1.y, acc0.z + acc1.z, acc0.w + acc1.w);
   }
+  DCK_CB_TRACE(4);
   cp_async_wait_all();
   __syncthreads();
+  DCK_CB_TRACE(5);
   const int share = kMaxRows * D / split;
   if constexpr (std::is_same<T, __nv_bfloat16>::value && D == 128) {
     // partial o over this CTA's rows of B_v on the tensor cores: o[16 x 128] =
@@ -342,7 +352,9 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
       }
   }
   }
+  DCK_CB_TRACE(6);
   cluster.sync();
+  DCK_CB_TRACE(7);
   T* out = static_cast<T*>(a.out);
   for (int pos = threadIdx.x; pos * split < nrow * D; pos += kThreads) {
     const int e = pos * split + rank;
@@ -355,28 +367,24 @@ __global__ void __launch_bounds__(kThreads, 2) combine_kernel(const LayerTable l
   }
 }
 
+// Dynamic shared memory of one CTA for an r_v split.
 template <typename T, int D>
-cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) {
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int split = lt.rv % (4 * kMaxSplit) == 0 ? kMaxSplit : kMaxSplit / 2;
-  // as many sequences per cluster as its rows allow: each head's B_v block is staged once per chunk
-  const int bchunk = std::max(1, std::min(a.B, kMaxRows / lt.qpg));
+size_t combine_smem(const LayerTable& lt, const DecodeArgs& a, int split) {
   const int rr = lt.rv / split;
   const int cap = 2 * a.n_items;
-  const size_t smem = (size_t)rr * ldb<T, D>() * sizeof(T) +
-                      sizeof(float) * ((size_t)kMaxRows * (rr + 4) + kMaxRows * D + kMaxRows + 2 * (size_t)kMaxRows * cap) +
-                      sizeof(int) * ((size_t)kMaxRows * cap + kMaxRows + 4 * kMaxRows + kMaxRows + a.B + 1 + a.n_items + 1);
-  auto k = combine_kernel<T, D>;
-  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
+  return (size_t)rr * ldb<T, D>() * sizeof(T) +
+         sizeof(float) * ((size_t)kMaxRows * (rr + 4) + kMaxRows * D + kMaxRows + 2 * (size_t)kMaxRows * cap) +
+         sizeof(int) * ((size_t)kMaxRows * cap + kMaxRows + 4 * kMaxRows + kMaxRows + a.B + 1 + a.n_items + 1);
+}
+
+template <typename T, int D>
+cudaLaunchConfig_t combine_config(const LayerTable& lt, const DecodeArgs& a, int split, int bchunk, size_t smem,
+                                  cudaStream_t s, cudaLaunchAttribute* attr) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(lt.Hkv * split, (a.B + bchunk - 1) / bchunk);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = split;
   attr[0].val.clusterDim.y = 1;
@@ -386,6 +394,30 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
+  return cfg;
+}
+
+template <typename T, int D>
+cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) {
+  // as many sequences per cluster as its rows allow: each head's B_v block is staged once per chunk
+  const int bchunk = std::max(1, std::min(a.B, kMaxRows / lt.qpg));
+  const int n_clusters = lt.Hkv * ((a.B + bchunk - 1) / bchunk);
+  // r_v split over a cluster of 8 CTAs where r_v allows.  Clusters of 8 CTAs
+  // that need two CTAs per SM were not all placed at once (7B MHA layer, B16:
+  // 30 of 32 clusters ran, the other two as a second wave that cost as much
+  // as the first), so where clusters of 4 fit one CTA per SM, 4 it is.
+  int split = lt.rv % (4 * kMaxSplit) == 0 ? kMaxSplit : kMaxSplit / 2;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (split == kMaxSplit && n_clusters * kMaxSplit > sms && n_clusters * (kMaxSplit / 2) <= sms) split = kMaxSplit / 2;
+  auto k = combine_kernel<T, D>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)combine_smem<T, D>(lt, a, split));
+  if (e != cudaSuccess) return e;
+  const size_t smem = combine_smem<T, D>(lt, a, split);
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = combine_config<T, D>(lt, a, split, bchunk, smem, s, attr);
   e = cudaLaunchKernelEx(&cfg, k, lt, a, bchunk, split);
   return e != cudaSuccess ? e : hook_launched(a.hook, s);
 }

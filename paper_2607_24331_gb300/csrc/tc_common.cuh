@@ -228,43 +228,17 @@ __device__ __forceinline__ int pair_tile_count(const DecodeArgs& a, int* s256, i
       if (L < 0 || st < 0 || st + L > a.n_rows) atomicOr(a.err, kErrBadSeq);
     }
   }
-  // inclusive prefixes over the threads (blockDim.x a multiple of 32, at most
-  // 1024): a shuffle scan within each warp, then one over the warps' totals
-  __shared__ int wt256[32], wt128[32];
-  const int lane = tid & 31, wid = tid >> 5, nw = nthr >> 5;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, l256, o), z = __shfl_up_sync(0xffffffffu, l128, o);
-    if (lane >= o) {
-      l256 += y;
-      l128 += z;
-    }
-  }
-  if (lane == 31) {
-    wt256[wid] = l256;
-    wt128[wid] = l128;
-  }
+  s256[tid] = l256;
+  s128[tid] = l128;
   __syncthreads();
-  if (wid == 0) {
-    int y = lane < nw ? wt256[lane] : 0, z = lane < nw ? wt128[lane] : 0;
-    const int y0 = y, z0 = z;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int yy = __shfl_up_sync(0xffffffffu, y, o), zz = __shfl_up_sync(0xffffffffu, z, o);
-      if (lane >= o) {
-        y += yy;
-        z += zz;
-      }
-    }
-    if (lane < nw) {  // exclusive prefix of the warps before
-      wt256[lane] = y - y0;
-      wt128[lane] = z - z0;
-    }
+  for (int off = 1; off < nthr; off <<= 1) {
+    const int v = tid >= off ? s256[tid - off] : 0;
+    const int w = tid >= off ? s128[tid - off] : 0;
+    __syncthreads();
+    s256[tid] += v;
+    s128[tid] += w;
+    __syncthreads();
   }
-  __syncthreads();
-  s256[tid] = l256 + wt256[wid];
-  s128[tid] = l128 + wt128[wid];
-  __syncthreads();
   return s256[nthr - 1];
 }
 
@@ -283,15 +257,24 @@ __device__ __forceinline__ PairWalker pair_walker_at(const DecodeArgs& a, const 
   }
   __syncthreads();
   int r256 = tid ? s256[tid - 1] : 0, r128 = tid ? s128[tid - 1] : 0;
-  for (int b = b0; b < b0 + per && b < a.B; ++b) {
-    const int nt = n256_of(a, b);
-    if (nt > 0 && X >= r256 && X < r256 + nt) {
-      s_b = b;
+  if (per == 1) {  // this thread's sequence (if any): its tile counts are the prefix steps
+    const int nt = s256[tid] - r256;
+    if (b0 < a.B && nt > 0 && X >= r256 && X < r256 + nt) {
+      s_b = b0;
       s_p256 = r256;
       s_p128 = r128;
     }
-    r256 += nt;
-    r128 += n128_of(a, b);
+  } else {
+    for (int b = b0; b < b0 + per && b < a.B; ++b) {
+      const int nt = n256_of(a, b);
+      if (nt > 0 && X >= r256 && X < r256 + nt) {
+        s_b = b;
+        s_p256 = r256;
+        s_p128 = r128;
+      }
+      r256 += nt;
+      r128 += n128_of(a, b);
+    }
   }
   __syncthreads();
   PairWalker w{s_b, s_p256, s_p128, X, X1, single};
