@@ -267,13 +267,15 @@ int32_t dck_set_decode_kernel(int32_t which);
 /*
  * dck_set_timing_events - timing hook of dck_decode_attention: `events` holds
  * n CUDA events (cudaEvent_t, owned by the caller, 2 <= n <= 16).  Each later
- * decode call records events[0] on its stream before its first kernel and
- * events[min(k, n - 1)] after its k-th kernel (k = 1, 2, ...): n = 2 brackets
- * the whole call, n = (kernels + 1) brackets every kernel.  Recording events
- * between kernels can delay a kernel that would otherwise start early
- * (programmatic dependent launch), so per-kernel brackets are for a
- * breakdown, not for timing the call.  n = 0 switches the hook off (events
- * is then ignored); any other invalid argument returns DCK_ERR_INVALID.
+ * decode call records events[0] on its stream before its first kernel,
+ * events[k] after its k-th kernel for k < n - 1 (k = 1, 2, ...) and
+ * events[n - 1] after its last kernel: n = 2 brackets the whole call with
+ * nothing recorded between its kernels, n = (kernels + 1) brackets every
+ * kernel.  Recording events between kernels delays a kernel that would
+ * otherwise start early (programmatic dependent launch), so per-kernel
+ * brackets are for a breakdown, not for timing the call.  n = 0 switches the
+ * hook off (events is then ignored); any other invalid argument returns
+ * DCK_ERR_INVALID.
  */
 dck_status dck_set_timing_events(void* const* events, int32_t n);
 

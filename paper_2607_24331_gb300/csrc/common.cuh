@@ -60,8 +60,9 @@ struct DecodeArgs {
 
 // Host-side record of the kernels one entry-point call puts on its stream.
 // When `n_ev` > 0, ev[0] (a cudaEvent_t) is recorded before the call's first
-// kernel and ev[min(k, n_ev - 1)] after its k-th kernel, so that a caller can
-// time the whole call (n_ev = 2) or every kernel of it (n_ev = kernels + 1).
+// kernel, ev[k] after its k-th kernel for k < n_ev - 1 and ev[n_ev - 1] after
+// its last kernel, so that a caller can time the whole call (n_ev = 2, nothing
+// recorded between the kernels) or every kernel of it (n_ev = kernels + 1).
 struct LaunchHook {
   void* const* ev = nullptr;
   int n_ev = 0;
@@ -69,6 +70,7 @@ struct LaunchHook {
 };
 inline cudaError_t hook_begin(LaunchHook* h, cudaStream_t s);     // before the first kernel
 inline cudaError_t hook_launched(LaunchHook* h, cudaStream_t s);  // after each kernel launch
+inline cudaError_t hook_end(LaunchHook* h, cudaStream_t s);       // after the call's last kernel
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -226,11 +228,20 @@ inline cudaError_t hook_begin(LaunchHook* h, cudaStream_t s) {
   return record_timing_event(h->ev[0], s);
 }
 
+// Events between kernels stop programmatic dependent launch from starting the
+// next kernel early, so only the brackets a caller asked for are recorded:
+// ev[k] after the k-th kernel for k < n_ev - 1, and ev[n_ev - 1] once, after
+// the call's last kernel (hook_end).
 inline cudaError_t hook_launched(LaunchHook* h, cudaStream_t s) {
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || !h) return e;
   ++h->count;
-  if (h->n_ev <= 0) return cudaSuccess;
-  return record_timing_event(h->ev[h->count < h->n_ev - 1 ? h->count : h->n_ev - 1], s);
+  if (h->count >= h->n_ev - 1) return cudaSuccess;
+  return record_timing_event(h->ev[h->count], s);
+}
+
+inline cudaError_t hook_end(LaunchHook* h, cudaStream_t s) {
+  if (!h || h->n_ev <= 0) return cudaSuccess;
+  return record_timing_event(h->ev[h->n_ev - 1], s);
 }
 }  // namespace dck

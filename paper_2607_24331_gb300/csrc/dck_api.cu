@@ -244,9 +244,10 @@ dck_status dck_prefill_attention(const dck_layer_desc* desc, const void* q, cons
   LaunchHook hook;
   hook.ev = t_events;
   hook.n_ev = t_n_events;
-  const cudaError_t e = launch_prefill_tc(lt, q, d_q_len, q_max, kcache, vcache, n_rows, B_k, B_v, d_seq_start,
-                                          d_seq_len, batch, max_seq_len, rope_theta, out, workspace, err, &hook,
-                                          static_cast<cudaStream_t>(stream));
+  cudaError_t e = launch_prefill_tc(lt, q, d_q_len, q_max, kcache, vcache, n_rows, B_k, B_v, d_seq_start,
+                                    d_seq_len, batch, max_seq_len, rope_theta, out, workspace, err, &hook,
+                                    static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) e = hook_end(&hook, static_cast<cudaStream_t>(stream));
   t_last_launches = hook.count;
   return e == cudaSuccess ? DCK_OK : DCK_ERR_CUDA;
 }
@@ -309,6 +310,7 @@ dck_status decode_call(const dck_layer_desc* desc, const void* q, const void* kc
   else e = launch_decode_simt(lt, a, desc->dtype, s);
   if (e != cudaSuccess) return DCK_ERR_CUDA;
   e = launch_combine(lt, a, desc->dtype, s);
+  if (e == cudaSuccess) e = hook_end(&hook, s);
   t_last_launches = hook.count;
   if (e != cudaSuccess) return DCK_ERR_CUDA;
   return DCK_OK;

@@ -92,3 +92,32 @@ def test_step_full_size_mha():
     """The 7B MHA workload, B16 x T4096, sampled heads of the first and last sequence."""
     w = S.workload(1)
     _step(w.layer, w.seq_lens, seed=w.seed, sample_heads=[(0, 0), (0, 17), (15, 5), (15, 31)])
+
+
+def test_timing_hook_brackets():
+    """dck_set_timing_events: with kernels + 1 events every kernel is bracketed, in launch order; with
+    two, the call is bracketed.  The events are recorded once beforehand (so that they exist), then a
+    mark; every event the hooked call records again must come after the mark, in order."""
+    w = S.workload(1)
+    buf = device.DecodeBuffers(w.layer, (700, 300)).synth(seed=7)
+    dck.check(buf.run(), "dck_decode_attention")
+    torch.cuda.synchronize()
+    kernels = dck.dck_last_launch_count()
+    assert kernels == 4
+    for n in (kernels + 1, 2):
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
+        for e_ in evs:
+            e_.record()
+        mark, after = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        mark.record()
+        dck.check(dck.dck_set_timing_events(evs), "timing events")
+        try:
+            dck.check(buf.run(), "dck_decode_attention")
+        finally:
+            dck.check(dck.dck_set_timing_events(None), "timing events")
+        after.record()
+        torch.cuda.synchronize()
+        chain = [mark] + evs + [after]
+        gaps = [chain[i].elapsed_time(chain[i + 1]) for i in range(len(chain) - 1)]
+        assert all(g >= 0 for g in gaps), (n, gaps)
+        assert evs[0].elapsed_time(evs[-1]) > 0
