@@ -47,6 +47,18 @@ def test_append_small(cfg, n_tok):
     _check(spec, n_tok, rows, n_rows, seed=cfg)
 
 
+@pytest.mark.parametrize("cfg,n_tok", [(1, 300), (3, 1000), (2, 257)])
+def test_append_long_ragged(cfg, n_tok):
+    """Appends above the split-K size run as persistent CTA pairs over 256-token x 256-column tiles:
+    token counts that leave a ragged last block, scattered destination rows, a key width (704) whose
+    last tile reaches past R_k."""
+    spec = S.workload(cfg).layer
+    rng = np.random.default_rng(n_tok + cfg)
+    n_rows = 2 * n_tok + 3
+    rows = rng.choice(n_rows, size=n_tok, replace=False)
+    _check(spec, n_tok, rows, n_rows, seed=10 + cfg)
+
+
 def test_append_prefill_8192_tokens_per_sequence():
     """Latent-append prefill of 2 x 8192 tokens of the long-context GQA layer."""
     spec = S.workload(3).layer
