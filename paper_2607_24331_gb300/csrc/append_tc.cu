@@ -15,6 +15,7 @@
 // prefill) with R_k and r_v multiples of 64 run on persistent CTA pairs
 // (append_pair_kernel below).
 #include <algorithm>
+#include <cstring>
 
 #include "common.cuh"
 #include "sm100.cuh"
@@ -39,7 +40,7 @@ struct AppendParams {
   int kblocks;   // ceil(D / 64)
   int ksplit;
   int stages;    // ring depth: min(kStages, K blocks of one CTA)
-  const int64_t* rows;
+  const int64_t* rows;  // cache row of each token (pair kernel: null writes token m to row m)
   __nv_bfloat16* kc;
   __nv_bfloat16* vc;
   int64_t n_rows;
@@ -237,7 +238,9 @@ __host__ __device__ inline int pt_count(int N) { return (N + 255) / 256; }
 __host__ __device__ inline int pt_width(int N, int j) {
   return j + 1 < pt_count(N) || N - 256 * j > 128 ? 256 : 128;
 }
-__host__ __device__ inline int pt_units(int N) { return 2 * (pt_count(N) - 1) + pt_width(N, pt_count(N) - 1) / 128; }
+__host__ __device__ inline int pt_units(int N) {
+  return N > 0 ? 2 * (pt_count(N) - 1) + pt_width(N, pt_count(N) - 1) / 128 : 0;
+}
 
 struct PairTile {
   int m0;    // first token
@@ -401,7 +404,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
       const int m = pt.m0 + hr * kBM + quad * 32 + lane;
       int64_t row = -1;
       if (m < p.n_tok) {
-        row = p.rows[m];
+        row = p.rows ? p.rows[m] : m;
         if (row < 0 || row >= p.n_rows) {
           atomicOr(p.err, kErrBadRow);
           row = -1;
@@ -488,6 +491,54 @@ int plan_ksplit(int n_tok, int D, int Rk, int rv, int sms) {
 }
 
 }  // namespace
+
+// C[M x N] = A[M x K] B[K x N] (bf16 row-major, fp32 accumulation, bf16
+// out) on the persistent CTA pairs of the long append, for N a multiple of 64:
+// the prefill's value reconstruction V^ = C_v B_v.  Returns
+// cudaErrorNotSupported when the pair kernel cannot run on this device.
+cudaError_t launch_gemm_pair(const void* A, int64_t M, int K, const void* Bm, int N, void* C, int* err,
+                             cudaStream_t s) {
+  if (M <= 0 || K <= 0 || N <= 0 || N % 64 || K % 8 || M >= (int64_t(1) << 31)) return cudaErrorInvalidValue;
+  AppendParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.n_tok = (int)M;
+  p.D = K;
+  p.Rk = N;
+  p.rv = 0;
+  p.kblocks = (K + kBK - 1) / kBK;
+  p.ksplit = 1;
+  p.rows = nullptr;  // row m of C is output row m
+  p.kc = static_cast<__nv_bfloat16*>(C);
+  p.vc = nullptr;
+  p.n_rows = M;
+  p.err = err;
+  CUtensorMap ta, tb;
+  if (!make_tmap_2d_bf16(&ta, A, K, M, (uint64_t)K * 2, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_tmap_2d_bf16(&tb, Bm, N, K, (uint64_t)N * 2, 64, kBK, CU_TENSOR_MAP_SWIZZLE_128B))
+    return cudaErrorInvalidValue;
+  const size_t psmem = (size_t)kPStages * kPStageBytes + 1024 + 256;
+  cudaError_t e = cudaFuncSetAttribute(append_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem);
+  if (e != cudaSuccess) return e;
+  const int pairs = append_pairs_of_device(psmem);
+  if (pairs <= 0) return cudaErrorNotSupported;
+  const int64_t units = (M + kPRows - 1) / kPRows * pt_units(N);
+  const int P = (int)std::min<int64_t>(pairs, units);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * P);
+  cfg.blockDim = dim3(kPThreads);
+  cfg.dynamicSmemBytes = psmem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, append_pair_kernel, ta, tb, tb, p);
+}
 
 bool tc_append_supports(int D, int Rk, int rv, int dtype) {
   return dtype == DCK_BF16 && D % 8 == 0 && Rk % 16 == 0 && rv % 16 == 0;

@@ -13,6 +13,8 @@
 //     V^_h = C_v B_v[:, h d : (h+1) d] (tcgen05.mma M = 128 rows, N = 128,
 //     K = r_g or r_v in TMA-staged pieces, fp32 in TMEM), written as bf16 to
 //     the workspace [n_rows][Hkv][d] (keys) and [n_rows][Hkv][d] (values);
+//     the values, where the cache rows are mostly in use, instead as one GEMM
+//     V^ = C_v B_v over all rows on the pair kernel of append_tc.cu;
 //  2. attn_kernel: causal flash attention over them, one CTA per 128 query
 //     rows of one KV head (the qpg query heads of a KV head packed into the
 //     rows: row r = query index r / qpg, head r % qpg), S = Q^ K^T and
@@ -30,6 +32,12 @@
 #include "tmap.h"
 
 namespace dck {
+
+// C[M x N] = A[M x K] B[K x N], bf16 row-major, fp32 accumulation, on the
+// persistent CTA pairs of the long latent append (append_tc.cu).
+cudaError_t launch_gemm_pair(const void* A, int64_t M, int K, const void* Bm, int N, void* C, int* err,
+                             cudaStream_t s);
+
 namespace {
 
 using namespace sm100;
@@ -614,7 +622,25 @@ cudaError_t launch_prefill_tc(const LayerTable& lt, const void* q, const int32_t
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(prefill_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)asmem);
   if (e != cudaSuccess) return e;
-  recon_kernel<<<dim3((max_len + kTile - 1) / kTile, B, 2 * lt.Hkv), kRThreads, rsmem, s>>>(rm, ra);
+  // Values: V^ = C_v B_v is one dense GEMM over the cache rows (no position
+  // enters it), run on the persistent CTA pairs of the long latent append,
+  // where the per-head reconstruction CTAs would each stream the whole latent
+  // tile for one head; taken when the rows in use can be most of the cache
+  // (every row is computed).  Keys (RoPE at each row's position, the head
+  // groups' factors) stay with the reconstruction kernel.
+  bool v_gemm = n_rows <= 2 * (int64_t)B * max_len && n_rows < (int64_t(1) << 31) - 256;
+  if (v_gemm) {
+    e = launch_gemm_pair(vc, n_rows, lt.rv, Bv, lt.Hkv * kPD, vw, err, s);
+    if (e == cudaErrorNotSupported) {
+      cudaGetLastError();
+      v_gemm = false;
+    } else if (e != cudaSuccess) {
+      return e;
+    } else if ((e = hook_launched(hook, s)) != cudaSuccess) {
+      return e;
+    }
+  }
+  recon_kernel<<<dim3((max_len + kTile - 1) / kTile, B, (v_gemm ? 1 : 2) * lt.Hkv), kRThreads, rsmem, s>>>(rm, ra);
   if ((e = hook_launched(hook, s)) != cudaSuccess) return e;
   AArgsP aa;
   std::memset(&aa, 0, sizeof(aa));
