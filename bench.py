@@ -623,6 +623,23 @@ def run_calls(args):
     print(f"{args.calls} decode-step calls of {w.name}: ok", flush=True)
 
 
+def run_append_calls(args):
+    """N latent appends of the long-context GQA layer's prefill (2 x 8192 tokens), L2 flushed before
+    each, then a check of the device error word.  The ncu capture of the append kernel in profiles/
+    uses it with `-s` to skip the first calls."""
+    import torch
+    from paper_2607_24331_gb300 import dck
+    from paper_2607_24331_gb300 import synth as S
+    dev = torch.device("cuda", 0)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    w = S.workload(3)
+    time_prefill_append(w, args.append_calls, 0, dev, flush)
+    torch.cuda.synchronize()
+    if dck.dck_last_device_error() != dck.DCK_OK:
+        raise SystemExit("device error word set")
+    print(f"{args.append_calls} latent appends of {w.name} (2 x {w.append_tokens} tokens): ok", flush=True)
+
+
 # ---------------------------------------------------------------------------
 # the GPU arm
 # ---------------------------------------------------------------------------
@@ -642,6 +659,9 @@ def main():
     ap.add_argument("--oracle-one-core", action="store_true", help=argparse.SUPPRESS)
     ap.add_argument("--calls", type=int, default=0,
                     help="profiling driver: this many plain decode-step calls, no timing and no JSON line")
+    ap.add_argument("--append-calls", type=int, default=0,
+                    help="profiling driver: this many latent appends of the long-context GQA prefill (2 x 8192 "
+                         "tokens), L2 flushed before each, no JSON line")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.oracle_one_core:
@@ -649,6 +669,9 @@ def main():
         return
     if args.calls > 0:
         run_calls(args)
+        return
+    if args.append_calls > 0:
+        run_append_calls(args)
         return
 
     if args.impl == "reference":

@@ -219,9 +219,9 @@ __global__ void append_finalize_kernel(const float* __restrict__ ws, int n_tok, 
 // L2.  Tiles, flattened: for every 256-token block, the key output in
 // 256-column tiles (the last one 128 wide when at most 128 columns remain;
 // columns past R_k load as zeros and are not stored), then the value output
-// likewise.  Pair p takes the tiles whose first 128-column unit falls in
-// [p U / P, (p+1) U / P) of the U units, in order.  Two 256-column TMEM
-// accumulators: the epilogue of one tile overlaps the next tile's MMAs.
+// likewise.  Pair p takes tiles p, p + P, p + 2P, ... of that list.  Two
+// 256-column TMEM accumulators: the epilogue of one tile overlaps the next
+// tile's MMAs.
 // ---------------------------------------------------------------------------
 
 constexpr int kPStages = 6;
@@ -238,10 +238,6 @@ __host__ __device__ inline int pt_count(int N) { return (N + 255) / 256; }
 __host__ __device__ inline int pt_width(int N, int j) {
   return j + 1 < pt_count(N) || N - 256 * j > 128 ? 256 : 128;
 }
-__host__ __device__ inline int pt_units(int N) {
-  return N > 0 ? 2 * (pt_count(N) - 1) + pt_width(N, pt_count(N) - 1) / 128 : 0;
-}
-
 struct PairTile {
   int m0;    // first token
   int out;   // 0: key output, 1: value output
@@ -250,22 +246,8 @@ struct PairTile {
 };
 
 struct PairPlan {
-  int tk, tv, trow, uk, urow;
-  __device__ PairPlan(int Rk, int rv)
-      : tk(pt_count(Rk)), tv(pt_count(rv)), trow(pt_count(Rk) + pt_count(rv)), uk(pt_units(Rk)),
-        urow(pt_units(Rk) + pt_units(rv)) {}
-  // first 128-column unit of flattened tile t
-  __device__ int64_t start(int64_t t) const {
-    const int64_t mt = t / trow;
-    const int j = (int)(t - mt * trow);
-    return mt * urow + (j < tk ? 2 * j : uk + 2 * (j - tk));
-  }
-  // smallest tile whose first unit is >= u (tiles [0, n) only)
-  __device__ int64_t first_at(int64_t u, int64_t n) const {
-    int64_t t = u / urow * trow;
-    while (t < n && start(t) < u) ++t;
-    return t;
-  }
+  int tk, trow;  // key tiles, tiles of a 256-token block
+  __device__ PairPlan(int Rk, int rv) : tk(pt_count(Rk)), trow(pt_count(Rk) + pt_count(rv)) {}
   __device__ PairTile tile(int64_t t, int Rk, int rv) const {
     const int64_t mt = t / trow;
     const int j = (int)(t - mt * trow);
@@ -322,9 +304,13 @@ __global__ void __launch_bounds__(kPThreads, 1)
 
   const PairPlan plan(p.Rk, p.rv);
   const int64_t n_mt = (p.n_tok + kPRows - 1) / kPRows;
-  const int64_t n_tiles = n_mt * plan.trow, n_units = n_mt * plan.urow;
-  const int64_t t0 = plan.first_at(pair * n_units / P, n_tiles);
-  const int64_t t1 = plan.first_at((pair + 1) * n_units / P, n_tiles);
+  const int64_t n_tiles = n_mt * plan.trow;
+  // pair p takes tiles p, p + P, p + 2P, ...: at any time the pairs work on P
+  // consecutive tiles, the column tiles of a few token blocks, so a block's x
+  // is read from HBM once and from L2 by the pairs of its other column tiles
+  // (contiguous ranges per pair re-read x from HBM for every column tile:
+  // 76 pairs' x blocks of 2 MB do not stay in L2 together)
+  const int64_t t0 = pair, t1 = n_tiles, tstep = P;
   const int kb_n = p.kblocks;
 
   if (warp == 0) {
@@ -338,7 +324,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
       pol_a = policy_evict_last();
       int64_t it = 0;
       bool ok = true;
-      for (int64_t t = t0; t < t1 && ok; ++t) {
+      for (int64_t t = t0; t < t1 && ok; t += tstep) {
         const PairTile pt = plan.tile(t, p.Rk, p.rv);
         const CUtensorMap* tb = pt.out ? &tm_av : &tm_ak;
         const int half = pt.w / 2, nbx = half / 64;
@@ -362,7 +348,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
       int64_t it = 0;
       bool ok = true;
       int lt = 0;  // tiles of this pair so far
-      for (int64_t t = t0; t < t1 && ok; ++t, ++lt) {
+      for (int64_t t = t0; t < t1 && ok; t += tstep, ++lt) {
         const PairTile pt = plan.tile(t, p.Rk, p.rv);
         const int buf = lt & 1;
         if (lt >= 2 && !(ok = mbar_wait(&acc_empty[buf], (uint32_t)(((lt >> 1) - 1) & 1), abort_flag))) break;
@@ -394,7 +380,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     int lt = 0;
     bool ok = true;
-    for (int64_t t = t0; t < t1 && ok; ++t, ++lt) {
+    for (int64_t t = t0; t < t1 && ok; t += tstep, ++lt) {
       const PairTile pt = plan.tile(t, p.Rk, p.rv);
       const int buf = lt & 1;
       ok = mbar_wait(&acc_full[buf], (uint32_t)((lt >> 1) & 1), abort_flag);
@@ -521,8 +507,8 @@ cudaError_t launch_gemm_pair(const void* A, int64_t M, int K, const void* Bm, in
   if (e != cudaSuccess) return e;
   const int pairs = append_pairs_of_device(psmem);
   if (pairs <= 0) return cudaErrorNotSupported;
-  const int64_t units = (M + kPRows - 1) / kPRows * pt_units(N);
-  const int P = (int)std::min<int64_t>(pairs, units);
+  const int64_t tiles = (M + kPRows - 1) / kPRows * pt_count(N);
+  const int P = (int)std::min<int64_t>(pairs, tiles);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * P);
   cfg.blockDim = dim3(kPThreads);
@@ -583,8 +569,8 @@ cudaError_t launch_append_tc(const void* x, int n_tok, int D, const void* A_k, c
     const int pairs = append_pairs_of_device(psmem);
     if (pairs > 0) {
       const int64_t n_mt = (n_tok + kPRows - 1) / kPRows;
-      const int64_t units = n_mt * (pt_units(Rk) + pt_units(rv));
-      const int P = (int)std::min<int64_t>(pairs, units);
+      const int64_t tiles = n_mt * (pt_count(Rk) + pt_count(rv));
+      const int P = (int)std::min<int64_t>(pairs, tiles);
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(2 * P);
       cfg.blockDim = dim3(kPThreads);
