@@ -406,11 +406,15 @@ cudaError_t launch_t(const LayerTable& lt, const DecodeArgs& a, cudaStream_t s) 
   // that need two CTAs per SM were not all placed at once (7B MHA layer, B16:
   // 30 of 32 clusters ran, the other two as a second wave that cost as much
   // as the first), so where clusters of 4 fit one CTA per SM, 4 it is.
+  // (The wider r_v slice of a CTA of 4 must still fit its shared memory.)
   int split = lt.rv % (4 * kMaxSplit) == 0 ? kMaxSplit : kMaxSplit / 2;
-  int dev = 0, sms = 0;
+  int dev = 0, sms = 0, smem_optin = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (split == kMaxSplit && n_clusters * kMaxSplit > sms && n_clusters * (kMaxSplit / 2) <= sms) split = kMaxSplit / 2;
+  cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (split == kMaxSplit && n_clusters * kMaxSplit > sms && n_clusters * (kMaxSplit / 2) <= sms &&
+      combine_smem<T, D>(lt, a, kMaxSplit / 2) <= (size_t)smem_optin)
+    split = kMaxSplit / 2;
   auto k = combine_kernel<T, D>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)combine_smem<T, D>(lt, a, split));
